@@ -1,0 +1,292 @@
+// Bandwidth-bound and small kernels of the chunk step: patch embedding,
+// adaLN-Zero LayerNorm modulation, the reuse path (Eq. 4), the conditioning
+// GEMVs, the output head, the Euler update and weight layout conversion.
+#include "xc_common.cuh"
+
+namespace xc {
+
+// ------------------------------------------------------------ patch embed
+// X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][C].
+template <typename T>
+__global__ void patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w,
+                                   const float *__restrict__ b, T *__restrict__ out, int L, int C, int d) {
+    const int runs = d / 16;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= L * runs) return;
+    const int row = idx / runs, col = (idx % runs) * 16;
+    float acc[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) acc[j] = b[col + j];
+    for (int k = 0; k < C; ++k) {
+        const float zv = z[(size_t)row * C + k];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) acc[j] = fmaf(zv, w[(size_t)k * d + col + j], acc[j]);
+    }
+    store16<T>(out + (size_t)row * d + col, acc);
+}
+
+template <typename T>
+cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st) {
+    const int n = L * (d / 16);
+    patch_embed_kernel<T><<<(n + 255) / 256, 256, 0, st>>>(z, w, b, out, L, C, d);
+    return cudaGetLastError();
+}
+template cudaError_t patch_embed<float>(const float *, const float *, const float *, float *, int, int, int, cudaStream_t);
+template cudaError_t patch_embed<bf16>(const float *, const float *, const float *, bf16 *, int, int, int, cudaStream_t);
+
+// ------------------------------------------------------------- row stats
+// Welford over a lane's elements, merged across the warp (Chan et al.).
+struct Moments {
+    float n, mean, m2;
+};
+__device__ __forceinline__ void welford_add(Moments &a, float x) {
+    a.n += 1.0f;
+    const float dlt = x - a.mean;
+    a.mean += dlt / a.n;
+    a.m2 += dlt * (x - a.mean);
+}
+__device__ __forceinline__ Moments welford_merge(Moments a, Moments b) {
+    if (b.n == 0.0f) return a;
+    if (a.n == 0.0f) return b;
+    Moments r;
+    r.n = a.n + b.n;
+    const float dlt = b.mean - a.mean;
+    r.mean = a.mean + dlt * (b.n / r.n);
+    r.m2 = a.m2 + b.m2 + dlt * dlt * (a.n * b.n / r.n);
+    return r;
+}
+__device__ __forceinline__ Moments warp_moments(Moments a) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        Moments b;
+        b.n = __shfl_xor_sync(0xffffffffu, a.n, o);
+        b.mean = __shfl_xor_sync(0xffffffffu, a.mean, o);
+        b.m2 = __shfl_xor_sync(0xffffffffu, a.m2, o);
+        a = welford_merge(a, b);
+    }
+    return a;
+}
+
+// ----------------------------------------------------------------- ln_mod
+// One warp per row: h = round(LN(x) * (1 + scale) + shift).  d % 512 == 0 is
+// not required; rows are walked in 16-element runs (d % 16 == 0).
+template <typename T>
+__global__ void __launch_bounds__(256)
+    ln_mod_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
+                  T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
+    if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= M) return;
+    const T *xr = x + (size_t)warp * d;
+    Moments mo = {0.0f, 0.0f, 0.0f};
+    for (int c = lane * 16; c < d; c += 32 * 16) {
+        float v[16];
+        load16<T>(xr + c, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) welford_add(mo, v[i]);
+    }
+    mo = warp_moments(mo);
+    const float rstd = rsqrtf(mo.m2 / (float)d + eps);
+    T *orow = out + (size_t)warp * d;
+    for (int c = lane * 16; c < d; c += 32 * 16) {
+        float v[16];
+        load16<T>(xr + c, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = (v[i] - mo.mean) * rstd * (1.0f + scale[c + i]) + shift[c + i];
+        store16<T>(orow + c, v);
+    }
+}
+
+template <typename T>
+cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
+                   const uint8_t *skip, cudaStream_t st) {
+    const int warps_per_block = 8;
+    ln_mod_kernel<T><<<(M + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, st>>>(
+        x, shift, scale, out, M, d, eps, skip);
+    return cudaGetLastError();
+}
+template cudaError_t ln_mod<float>(const float *, const float *, const float *, float *, int, int, float,
+                                   const uint8_t *, cudaStream_t);
+template cudaError_t ln_mod<bf16>(const bf16 *, const float *, const float *, bf16 *, int, int, float,
+                                  const uint8_t *, cudaStream_t);
+
+// ------------------------------------------------------------ reuse (Eq. 4)
+// out = round(x + rhat), 16-byte vectors; runs only when the gate chose reuse
+// (need_flag = XC_DEC_SKIP) or unconditionally (skip_flag == nullptr).
+template <typename T>
+__global__ void __launch_bounds__(256)
+    reuse_kernel(const T *__restrict__ x, const T *__restrict__ r, T *__restrict__ out, long n16,
+                 const uint8_t *__restrict__ skip_flag) {
+    if (skip_flag != nullptr && *skip_flag != XC_DEC_SKIP) return;
+    const long stride = (long)gridDim.x * blockDim.x;
+    for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n16; i += stride) {
+        float a[16], b[16];
+        load16<T>(x + i * 16, a);
+        load16<T>(r + i * 16, b);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) a[j] += b[j];
+        store16<T>(out + i * 16, a);
+    }
+}
+
+template <typename T>
+cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t *skip, int n_sm, cudaStream_t st) {
+    const long n16 = n / 16;
+    long blocks = (n16 + 255) / 256;
+    const long cap = (long)n_sm * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    reuse_kernel<T><<<(unsigned)blocks, 256, 0, st>>>(x, r, out, n16, skip);
+    return cudaGetLastError();
+}
+template cudaError_t residual_reuse<float>(const float *, const float *, float *, long, const uint8_t *, int, cudaStream_t);
+template cudaError_t residual_reuse<bf16>(const bf16 *, const bf16 *, bf16 *, long, const uint8_t *, int, cudaStream_t);
+
+// -------------------------------------------------------------- Euler step
+__global__ void euler_kernel(float *__restrict__ x, const float *__restrict__ v, float ds, long n) {
+    const long i = blockIdx.x * (long)blockDim.x + threadIdx.x;
+    if (i < n) x[i] = fmaf(ds, v[i], x[i]);
+}
+cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_t st) {
+    euler_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(x, v, ds, n);
+    return cudaGetLastError();
+}
+
+// ----------------------------------------------------------- conditioning
+// Sinusoidal embedding of the flow time 1000*sigma, computed in double
+// precision (angles reach 1000 rad): e[i] = cos(s f_i), e[half + i] = sin(s f_i),
+// f_i = 10000^(-i/half).
+__global__ void temb_kernel(float sigma, float *__restrict__ e, int dim) {
+    const int half = dim / 2;
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= half) return;
+    const double f = exp(-9.210340371976184 * (double)i / (double)half);   // ln(10000)
+    const double a = 1000.0 * (double)sigma * f;
+    e[i] = (float)cos(a);
+    e[half + i] = (float)sin(a);
+}
+cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st) {
+    temb_kernel<<<(dim / 2 + 127) / 128, 128, 0, st>>>(sigma, e, dim);
+    return cudaGetLastError();
+}
+
+// y[j] = act_out( sum_i in(i) W[i][j] + b[j] + add[j] ), W [n_in][n_out].
+// in_silu: in = SiLU(x) instead of x.  act_out 0: none, 1: SiLU.
+__global__ void gemv_kernel(const float *__restrict__ x, int in_silu, const float *__restrict__ W,
+                            const float *__restrict__ b, const float *__restrict__ add, float *__restrict__ y,
+                            int n_in, int n_out, int act_out) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= n_out) return;
+    float acc = 0.0f;
+    for (int i = 0; i < n_in; ++i) {
+        const float xi = in_silu ? silu(x[i]) : x[i];
+        acc = fmaf(xi, W[(size_t)i * n_out + j], acc);
+    }
+    acc += b[j];
+    if (add != nullptr) acc += add[j];
+    y[j] = act_out == 1 ? silu(acc) : acc;
+}
+
+cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
+                 int n_out, int act_out, cudaStream_t st) {
+    gemv_kernel<<<(n_out + 127) / 128, 128, 0, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
+    return cudaGetLastError();
+}
+
+// mods_all[b][j][c] = m[j*d + c] + blk_mod[b][j][c]   (B x 6 x d)
+__global__ void assemble_mods_kernel(const float *__restrict__ m, const float *__restrict__ tab,
+                                     float *__restrict__ out, int B, int d) {
+    const long i = blockIdx.x * (long)blockDim.x + threadIdx.x;
+    if (i >= (long)B * 6 * d) return;
+    out[i] = m[i % (6 * d)] + tab[i];
+}
+cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, int d, cudaStream_t st) {
+    const long n = (long)B * 6 * d;
+    assemble_mods_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(m, tab, out, B, d);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------- head
+// One warp per row: hf = round(LN(x) (1 + scale) + shift); v = hf W_out + b_out
+// (C = 16 output channels, float32 out).
+template <typename T>
+__global__ void __launch_bounds__(256)
+    head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
+                const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
+    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (warp >= L) return;
+    const T *xr = x + (size_t)warp * d;
+    Moments mo = {0.0f, 0.0f, 0.0f};
+    for (int c = lane * 16; c < d; c += 512) {
+        float t[16];
+        load16<T>(xr + c, t);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) welford_add(mo, t[i]);
+    }
+    mo = warp_moments(mo);
+    const float rstd = rsqrtf(mo.m2 / (float)d + eps);
+    const float *shift = hm, *scale = hm + d;
+    float acc[16];
+#pragma unroll
+    for (int o = 0; o < 16; ++o) acc[o] = 0.0f;
+    for (int c = lane * 16; c < d; c += 512) {
+        float t[16];
+        load16<T>(xr + c, t);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float hv = round_to<T>((t[i] - mo.mean) * rstd * (1.0f + scale[c + i]) + shift[c + i]);
+            const float *wr = w + (size_t)(c + i) * 16;
+#pragma unroll
+            for (int o = 0; o < 16; ++o) acc[o] = fmaf(hv, wr[o], acc[o]);
+        }
+    }
+#pragma unroll
+    for (int o = 0; o < 16; ++o) {
+#pragma unroll
+        for (int s = 16; s > 0; s >>= 1) acc[o] += __shfl_xor_sync(0xffffffffu, acc[o], s);
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int o = 0; o < 16; ++o) v[(size_t)warp * 16 + o] = acc[o] + b[o];
+    }
+}
+
+template <typename T>
+cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
+                 cudaStream_t st) {
+    head_kernel<T><<<(L + 7) / 8, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
+    return cudaGetLastError();
+}
+template cudaError_t head<float>(const float *, const float *, const float *, const float *, float *, int, int, float,
+                                 cudaStream_t);
+template cudaError_t head<bf16>(const bf16 *, const float *, const float *, const float *, float *, int, int, float,
+                                cudaStream_t);
+
+// --------------------------------------------------------- weight layout
+// Wt[n][k] = convert(W[k][n]) for one [K][N] float32 matrix (32x32 tiles).
+template <typename T>
+__global__ void transpose_convert_kernel(const float *__restrict__ W, T *__restrict__ Wt, int K, int N) {
+    __shared__ float tile[32][33];
+    const int n0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int k = k0 + i, n = n0 + threadIdx.x;
+        tile[i][threadIdx.x] = (k < K && n < N) ? W[(size_t)k * N + n] : 0.0f;
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int n = n0 + i, k = k0 + threadIdx.x;
+        if (n < N && k < K) Wt[(size_t)n * K + k] = from_f<T>(tile[threadIdx.x][i]);
+    }
+}
+template <typename T>
+cudaError_t transpose_convert(const float *W, T *Wt, int K, int N, cudaStream_t st) {
+    dim3 grid((N + 31) / 32, (K + 31) / 32), block(32, 8);
+    transpose_convert_kernel<T><<<grid, block, 0, st>>>(W, Wt, K, N);
+    return cudaGetLastError();
+}
+template cudaError_t transpose_convert<float>(const float *, float *, int, int, cudaStream_t);
+template cudaError_t transpose_convert<bf16>(const float *, bf16 *, int, int, cudaStream_t);
+
+}  // namespace xc

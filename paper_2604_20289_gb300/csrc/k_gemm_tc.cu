@@ -1,0 +1,194 @@
+// bf16 GEMM on the 5th-generation tensor core (tcgen05), fed by TMA.
+//
+//   C[M][N] = epilogue(A[M][K] @ Wt[N][K]^T), fp32 accumulation in TMEM.
+//
+// One CTA computes a 128 x BN tile.  Warp roles (192 threads):
+//   warp 0, lane 0 : TMA producer, STAGES-deep ring of (A 128x64, B BNx64)
+//                    tiles in 128B-swizzled shared memory;
+//   warp 1         : allocates TMEM; lane 0 issues tcgen05.mma (M=128, N=BN,
+//                    K=16 per instruction, 4 per 64-wide k-tile) and commits
+//                    each stage back to the producer;
+//   warps 2..5     : epilogue -- tcgen05.ld of their 32-lane TMEM quadrant,
+//                    fused bias / GELU / gated residual / residual-cache /
+//                    RoPE, vectorised stores.
+// The skip flag of the block lets the whole recompute path early-exit when
+// the gate chose reuse (Eq. 4), so decisions never return to the host.
+#include "xc_ptx.cuh"
+
+namespace xc {
+
+constexpr int GEMM_BM = 128;
+constexpr int GEMM_BK = 64;
+
+template <int BN>
+struct GemmTile {
+    static constexpr int STAGES = BN == 256 ? 4 : 6;
+    static constexpr int A_BYTES = GEMM_BM * GEMM_BK * 2;
+    static constexpr int B_BYTES = BN * GEMM_BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int BAR_OFFSET = STAGES * STAGE_BYTES;
+    static constexpr int SMEM_BYTES = BAR_OFFSET + 256 + 1024;   // barriers + alignment slack
+    static constexpr int TMEM_COLS = BN;
+};
+
+__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
+    const uint32_t s = smem_u32(p);
+    return p + ((1024u - (s & 1023u)) & 1023u);
+}
+
+template <int BN, int EPI, typename T>
+__global__ void __launch_bounds__(192, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const EpiParams ep, const int K, const uint8_t *__restrict__ skip_flag, int *err) {
+    using G = GemmTile<BN>;
+    if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = align1024(smem_raw);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + G::BAR_OFFSET);
+    uint64_t *empty = full + G::STAGES;
+    uint64_t *done = empty + G::STAGES;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * GEMM_BM;
+    const int KT = K / GEMM_BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < G::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(done, 1);
+        mbar_fence_init();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, G::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int issued = 0;
+            for (int kt = 0; kt < KT; ++kt) {
+                const int s = kt % G::STAGES;
+                const uint32_t ph = (kt / G::STAGES) & 1;
+                if (!mbar_wait(&empty[s], ph ^ 1, err, ERR_WAIT_PRODUCER)) break;
+                uint8_t *sa = smem + s * G::STAGE_BYTES;
+                mbar_expect_tx(&full[s], G::STAGE_BYTES);
+                tma_load_2d(sa, &tmA, &full[s], kt * GEMM_BK, m0);
+                tma_load_2d(sa + G::A_BYTES, &tmB, &full[s], kt * GEMM_BK, n0);
+                issued = kt + 1;
+            }
+            // Drain: every copy this thread started has landed before exit.
+            for (int kt = issued - G::STAGES < 0 ? 0 : issued - G::STAGES; kt < issued; ++kt)
+                mbar_wait(&full[kt % G::STAGES], (kt / G::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(GEMM_BM, BN, false, false);
+            for (int kt = 0; kt < KT; ++kt) {
+                const int s = kt % G::STAGES;
+                const uint32_t ph = (kt / G::STAGES) & 1;
+                if (!mbar_wait(&full[s], ph, err, ERR_WAIT_MMA)) break;
+                tc_fence_after();
+                const uint32_t a = smem_u32(smem + s * G::STAGE_BYTES);
+                const uint32_t b = a + G::A_BYTES;
+#pragma unroll
+                for (int k = 0; k < GEMM_BK / 16; ++k) {
+                    tc_mma(tmem, sdesc_sw128(a + 32 * k, 16, 1024), sdesc_sw128(b + 32 * k, 16, 1024), idesc,
+                           (kt | k) != 0 ? 1u : 0u);
+                }
+                tc_commit(&empty[s]);
+            }
+            tc_commit(done);
+        }
+    } else {
+        const int q = warp & 3;   // TMEM lane quadrant this warp may access
+        const bool ok = mbar_wait(done, 0, err, ERR_WAIT_EPI);
+        tc_fence_after();
+        if (ok) {
+            const int row = m0 + q * 32 + lane;
+            const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 16) {
+                float v[16];
+                tmem_ld16_sync(tq + c, v);
+                epilogue16<EPI, T>(ep, row, n0 + c, v);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, G::TMEM_COLS);
+    }
+}
+
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (fn == nullptr) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows][cols] matrix, box [box_rows][64],
+// 128-byte swizzle, zero fill outside the matrix.
+bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (fn == nullptr) return false;
+    if ((reinterpret_cast<uintptr_t>(base) & 15) != 0 || (cols * 2) % 16 != 0) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int EPI>
+static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+                             const uint8_t *skip, int *err, cudaStream_t st) {
+    constexpr int BN = 256;
+    using G = GemmTile<BN>;
+    auto kern = gemm_tc_kernel<BN, EPI, bf16>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    dim3 grid(ep.N / BN, (ep.M + GEMM_BM - 1) / GEMM_BM);
+    kern<<<grid, 192, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
+    return cudaGetLastError();
+}
+
+// Entry used by the chunk step and xc_op_linear / xc_op_qkv_rope (bf16 only).
+// `ta` covers A [M][K], `tb` covers Wt [N][K]; N % 256 == 0, K % 64 == 0.
+cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+                    const uint8_t *skip, int *err, cudaStream_t st) {
+    switch (epi) {
+        case EPI_BIAS: return launch_tc<EPI_BIAS>(ta, tb, ep, K, skip, err, st);
+        case EPI_GELU: return launch_tc<EPI_GELU>(ta, tb, ep, K, skip, err, st);
+        case EPI_RESID_GATE: return launch_tc<EPI_RESID_GATE>(ta, tb, ep, K, skip, err, st);
+        case EPI_RESID_CACHE: return launch_tc<EPI_RESID_CACHE>(ta, tb, ep, K, skip, err, st);
+        case EPI_QKV_ROPE: return launch_tc<EPI_QKV_ROPE>(ta, tb, ep, K, skip, err, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace xc

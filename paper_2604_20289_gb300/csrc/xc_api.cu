@@ -1,0 +1,1021 @@
+// Host runtime of the X-Cache chunk step: the C ABI of include/xcache.h and
+// include/xcache_ops.h.  Owns device memory for weights, the rolling KV ring,
+// the per-(t, b) residual / fingerprint caches and scratch; sequences the
+// kernels of one forward pass on the context's stream.  Gate decisions stay
+// on the device: every recompute kernel of block b reads flag[b] and exits
+// early when the gate chose reuse; the reuse kernel runs only then.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "xc_kernels.cuh"
+
+
+using namespace xc;
+
+// ------------------------------------------------------------------ helpers
+namespace {
+
+std::mutex g_err_mu;
+std::string g_global_err = "no error";
+
+struct Fail {
+    xc_status st;
+};
+
+// RoPE pair table: head_dim split hd/8 (camera) : 3hd/8 (absolute frame) :
+// hd/4 (h) : hd/4 (w); pair j of an axis with D dims rotates at theta^(-2j/D).
+void rope_table(int hd, double theta, std::vector<float> &freq, std::vector<int> &axis) {
+    const int dims[4] = {hd / 8, 3 * hd / 8, hd / 4, hd / 4};
+    freq.clear();
+    axis.clear();
+    for (int a = 0; a < 4; ++a)
+        for (int j = 0; j < dims[a] / 2; ++j) {
+            axis.push_back(a);
+            freq.push_back((float)std::pow(theta, -2.0 * j / dims[a]));
+        }
+}
+
+// Spatial sample of the fingerprint (Section 2.3.1): per axis
+// k_a = clamp(floor(dim_a * (K / (F H W))^(1/3)), 1, dim_a), taken exactly as the
+// largest k with k^3 * F*H*W <= K * dim_a^3; indices floor((2j+1) dim / (2k));
+// Cartesian product per camera; cameras with <= K tokens keep every token.
+std::vector<int> fingerprint_rows(int V, int Fr, int gh, int gw, int K, int *kfp) {
+    const long long N = (long long)Fr * gh * gw;
+    std::vector<int> rows;
+    if (N <= K) {
+        *kfp = (int)N;
+        for (int c = 0; c < V; ++c)
+            for (long long i = 0; i < N; ++i) rows.push_back((int)(c * N + i));
+        return rows;
+    }
+    const int dims[3] = {Fr, gh, gw};
+    int k[3];
+    for (int a = 0; a < 3; ++a) {
+        long long kk = 0;
+        const long long dm = dims[a];
+        while (kk + 1 <= dm && (kk + 1) * (kk + 1) * (kk + 1) * N <= (long long)K * dm * dm * dm) ++kk;
+        if (kk < 1) kk = 1;
+        k[a] = (int)kk;
+    }
+    *kfp = k[0] * k[1] * k[2];
+    for (int c = 0; c < V; ++c)
+        for (int i = 0; i < k[0]; ++i) {
+            const int f = (int)(((2LL * i + 1) * Fr) / (2LL * k[0]));
+            for (int j = 0; j < k[1]; ++j) {
+                const int h = (int)(((2LL * j + 1) * gh) / (2LL * k[1]));
+                for (int l = 0; l < k[2]; ++l) {
+                    const int w = (int)(((2LL * l + 1) * gw) / (2LL * k[2]));
+                    rows.push_back((int)(c * N + ((long long)f * gh + h) * gw + w));
+                }
+            }
+        }
+    return rows;
+}
+
+bool is_host_ptr(const void *p) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return true;
+    }
+    return a.type == cudaMemoryTypeHost || a.type == cudaMemoryTypeUnregistered;
+}
+
+}  // namespace
+
+struct xc_ctx {
+    xc_model_cfg cfg;
+    int L, d, F, B, S, H, hd, Wkv, C, A, V, npc;
+    bool bf;
+    size_t esz;
+    cudaStream_t st;
+    int n_sm;
+    std::vector<void *> allocs;
+
+    // weights
+    float *pe_w, *pe_b, *t_w1, *t_b1, *t_w2, *t_b2, *a_w1, *a_b1, *a_w2, *a_b2;
+    float *mod_w, *mod_b, *blk_mod, *head_w, *head_b, *head_tab, *out_w, *out_b;
+    void *qkv_wt, *o_wt, *f1_wt, *f2_wt;      // [B][N][K] activation dtype
+    float *qkv_b, *o_b, *f1_b, *f2_b;          // [B][N]
+    float *rope_freq;
+    int *rope_axis;
+
+    // activations / conditioning
+    void *xb[2], *x1, *hbuf, *q, *o, *u;
+    float *lat, *vout, *act_dev;
+    float *temb, *ht, *ha, *e1, *e, *mshared, *mods, *hmod;
+
+    // rolling KV ring [B][Wkv][L][d] and caches
+    void *ring_k, *ring_v;
+    void *rhat;                                // [S][B][L][d]
+    float *phi;                                // [S][B][2][n_all]
+    float *phi_act;                            // [S][B][2][8]
+    GateCell *cells;                           // [S][B]
+    int *fp_rows;
+    int fp_K, kfp;
+    size_t phi_n_all;
+
+    // per pass
+    uint8_t *flags;
+    float *s_cos, *d_max, *tau;
+    uint8_t *h_flags;
+    float *h_stats;                            // pinned [3][B]
+    int *d_err;
+
+    // gate scratch
+    int g_ns, g_R;
+    float *g_colsum;
+    double *g_sp, *g_gl;
+    unsigned *g_cnt;
+
+    // tensor maps (bf16)
+    CUtensorMap tm_h, tm_o, tm_u, tm_q;
+    std::vector<CUtensorMap> tm_wqkv, tm_wo, tm_w1, tm_w2, tm_rk, tm_rv;
+
+    int n, next_step;
+    void *trace;
+    std::string err;
+};
+
+namespace {
+
+void set_err(xc_ctx *c, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c != nullptr) c->err = buf;
+    std::lock_guard<std::mutex> g(g_err_mu);
+    g_global_err = buf;
+}
+
+#define CK(call)                                                                            \
+    do {                                                                                    \
+        cudaError_t e_ = (call);                                                            \
+        if (e_ != cudaSuccess) {                                                            \
+            set_err(ctx, "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, __LINE__); \
+            throw Fail{e_ == cudaErrorMemoryAllocation ? XC_ENOMEM : XC_ECUDA};             \
+        }                                                                                   \
+    } while (0)
+
+template <typename P>
+P *dalloc(xc_ctx *ctx, size_t bytes) {
+    void *p = nullptr;
+    CK(cudaMalloc(&p, bytes < 16 ? 16 : bytes));
+    ctx->allocs.push_back(p);
+    return reinterpret_cast<P *>(p);
+}
+
+void upload(xc_ctx *ctx, float *dst, const float *src, size_t n) {
+    CK(cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyHostToDevice));
+}
+
+bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
+    auto bad = [&](const char *m) { snprintf(why, n, "invalid model cfg: %s", m); return false; };
+    if (c->n_blocks < 1 || c->n_blocks > XC_MAX_BLOCKS) return bad("n_blocks out of [1, 64]");
+    if (c->d_model < 16 || c->n_heads < 1 || c->head_dim < 16) return bad("sizes too small");
+    if (c->n_heads * c->head_dim != c->d_model) return bad("d_model != n_heads * head_dim");
+    if (c->head_dim % 16 != 0) return bad("head_dim % 16 != 0");
+    if (c->d_model % 64 != 0 || c->d_ffn % 16 != 0 || c->d_ffn < 16) return bad("d_model % 64 or d_ffn % 16");
+    if (c->c_latent != 16) return bad("c_latent must be 16");
+    if (c->action_dim < 1 || c->action_dim > 8) return bad("action_dim out of [1, 8]");
+    if (c->n_cams < 1 || c->frames < 1 || c->grid_h < 1 || c->grid_w < 1) return bad("empty latent grid");
+    if ((long long)c->n_cams * c->frames * c->grid_h * c->grid_w > (1LL << 24)) return bad("chunk too large");
+    if (c->kv_window_chunks < 1 || c->n_denoise_steps < 1 || c->n_denoise_steps > 64) return bad("window / steps");
+    if (c->t_freq_dim < 2 || c->t_freq_dim % 2 != 0) return bad("t_freq_dim must be even");
+    if (!(c->ln_eps > 0.0f) || !(c->rope_theta > 1.0f)) return bad("ln_eps / rope_theta");
+    if (c->dtype == XC_BF16) {
+        if (c->head_dim != 64 && c->head_dim != 128) return bad("bf16 needs head_dim 64 or 128");
+        if (c->d_model % 256 != 0 || c->d_ffn % 256 != 0) return bad("bf16 needs d_model, d_ffn % 256 == 0");
+    } else if (c->dtype == XC_F32) {
+        if (c->head_dim > 64) return bad("f32 path supports head_dim 16, 32, 64");
+        if (c->head_dim != 16 && c->head_dim != 32 && c->head_dim != 64) return bad("f32 head_dim");
+    } else {
+        return bad("dtype must be XC_F32 or XC_BF16");
+    }
+    return true;
+}
+
+bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
+    auto bad = [&](const char *m) { snprintf(why, n, "invalid gate params: %s", m); return false; };
+    const float f[] = {p->tau_floor, p->margin, p->alpha, p->tau_dev, p->eps_dev, p->step0_strict_tau};
+    for (float v : f)
+        if (std::isnan(v)) return bad("NaN threshold");
+    if (p->alpha < 0.0f || p->alpha > 1.0f) return bad("alpha out of [0, 1]");
+    if (p->front_anchors < 0 || p->back_anchors < 0 || p->warmup_chunks < 0 || p->max_skips < 0)
+        return bad("negative count");
+    if (p->fp_tokens < 1) return bad("fp_tokens < 1");
+    if (p->fp_refresh != 0 && p->fp_refresh != 1) return bad("fp_refresh must be 0 or 1");
+    (void)B;
+    return true;
+}
+
+// (Re)build the spatial sample for a token budget K; resets every gate cell.
+void ensure_fp(xc_ctx *ctx, int K) {
+    if (ctx->fp_K == K) return;
+    int kfp = 0;
+    std::vector<int> rows = fingerprint_rows(ctx->V, ctx->cfg.frames, ctx->cfg.grid_h, ctx->cfg.grid_w, K, &kfp);
+    const size_t n_all = (size_t)ctx->V * kfp * ctx->d + (size_t)ctx->V * ctx->d;
+    if (ctx->fp_rows != nullptr) {
+        CK(cudaStreamSynchronize(ctx->st));
+        for (auto it = ctx->allocs.begin(); it != ctx->allocs.end();) {
+            if (*it == ctx->fp_rows || *it == ctx->phi) {
+                cudaFree(*it);
+                it = ctx->allocs.erase(it);
+            } else {
+                ++it;
+            }
+        }
+    }
+    ctx->fp_rows = dalloc<int>(ctx, rows.size() * sizeof(int));
+    CK(cudaMemcpy(ctx->fp_rows, rows.data(), rows.size() * sizeof(int), cudaMemcpyHostToDevice));
+    ctx->phi = dalloc<float>(ctx, (size_t)ctx->S * ctx->B * 2 * n_all * sizeof(float));
+    CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * n_all * sizeof(float), ctx->st));
+    CK(cudaMemsetAsync(ctx->cells, 0, (size_t)ctx->S * ctx->B * sizeof(GateCell), ctx->st));
+    CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
+    ctx->kfp = kfp;
+    ctx->phi_n_all = n_all;
+    ctx->fp_K = K;
+}
+
+void clear_state(xc_ctx *ctx) {
+    const size_t ring = (size_t)ctx->B * ctx->Wkv * ctx->L * ctx->d * ctx->esz;
+    CK(cudaMemsetAsync(ctx->ring_k, 0, ring, ctx->st));
+    CK(cudaMemsetAsync(ctx->ring_v, 0, ring, ctx->st));
+    CK(cudaMemsetAsync(ctx->rhat, 0, (size_t)ctx->S * ctx->B * ctx->L * ctx->d * ctx->esz, ctx->st));
+    CK(cudaMemsetAsync(ctx->cells, 0, (size_t)ctx->S * ctx->B * sizeof(GateCell), ctx->st));
+    CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
+    if (ctx->phi != nullptr)
+        CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * ctx->phi_n_all * sizeof(float), ctx->st));
+    CK(cudaMemsetAsync(ctx->g_cnt, 0, (size_t)(ctx->V * ctx->g_ns + 1) * sizeof(unsigned), ctx->st));
+    CK(cudaStreamSynchronize(ctx->st));
+    ctx->n = 0;
+    ctx->next_step = 0;
+}
+
+// Per-block weight upload: W [K][N] float32 (host) -> Wt [N][K] activation dtype.
+void upload_blocks(xc_ctx *ctx, void *dst, const float *src, int K, int N, float *tmp) {
+    for (int b = 0; b < ctx->B; ++b) {
+        CK(cudaMemcpy(tmp, src + (size_t)b * K * N, (size_t)K * N * sizeof(float), cudaMemcpyHostToDevice));
+        char *out = reinterpret_cast<char *>(dst) + (size_t)b * K * N * ctx->esz;
+        if (ctx->bf)
+            CK(transpose_convert<bf16>(tmp, reinterpret_cast<bf16 *>(out), K, N, ctx->st));
+        else
+            CK(transpose_convert<float>(tmp, reinterpret_cast<float *>(out), K, N, ctx->st));
+        CK(cudaStreamSynchronize(ctx->st));
+    }
+}
+
+void tmap(xc_ctx *ctx, CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box) {
+    if (!make_tmap_bf16(m, base, rows, cols, box)) {
+        set_err(ctx, "cuTensorMapEncodeTiled failed (rows %llu cols %llu)", (unsigned long long)rows,
+                (unsigned long long)cols);
+        throw Fail{XC_ECUDA};
+    }
+}
+
+template <typename T>
+void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigma, int t, bool kv,
+              const xc_gate_params &p, float *v_dev) {
+    const int L = ctx->L, d = ctx->d, F = ctx->F, B = ctx->B, hd = ctx->hd;
+    cudaStream_t st = ctx->st;
+    const size_t Ld = (size_t)L * d;
+    const int n = ctx->n;
+    const int slot = n % ctx->Wkv;
+    const int n_res = (n + 1 < ctx->Wkv ? n + 1 : ctx->Wkv);
+    const int n_keys = n_res * L;
+
+    // conditioning c_t: timestep + action embeddings -> adaLN-Zero vectors
+    CK(cudaMemcpyAsync(ctx->act_dev, action, ctx->A * sizeof(float), cudaMemcpyHostToDevice, st));
+    CK(timestep_embedding(sigma, ctx->temb, ctx->cfg.t_freq_dim, st));
+    CK(gemv(ctx->temb, 0, ctx->t_w1, ctx->t_b1, nullptr, ctx->ht, ctx->cfg.t_freq_dim, d, 1, st));
+    CK(gemv(ctx->act_dev, 0, ctx->a_w1, ctx->a_b1, nullptr, ctx->ha, ctx->A, d, 1, st));
+    CK(gemv(ctx->ht, 0, ctx->t_w2, ctx->t_b2, nullptr, ctx->e1, d, d, 0, st));
+    CK(gemv(ctx->ha, 0, ctx->a_w2, ctx->a_b2, ctx->e1, ctx->e, d, d, 0, st));
+    CK(gemv(ctx->e, 1, ctx->mod_w, ctx->mod_b, nullptr, ctx->mshared, d, 6 * d, 0, st));
+    CK(gemv(ctx->e, 1, ctx->head_w, ctx->head_b, ctx->head_tab, ctx->hmod, d, 2 * d, 0, st));
+    CK(assemble_mods(ctx->mshared, ctx->blk_mod, ctx->mods, B, d, st));
+
+    T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
+    CK(patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
+    CK(cudaMemsetAsync(ctx->flags, 0, B, st));
+    CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
+
+    const bool gating = p.enabled != 0 && !kv;
+    const bool eval_mode = n >= p.warmup_chunks && !(p.protect_step0 && t == 0);
+    T *x1 = reinterpret_cast<T *>(ctx->x1);
+    T *hb = reinterpret_cast<T *>(ctx->hbuf);
+    T *qb = reinterpret_cast<T *>(ctx->q);
+    T *ob = reinterpret_cast<T *>(ctx->o);
+    T *ub = reinterpret_cast<T *>(ctx->u);
+
+    for (int b = 0; b < B; ++b) {
+        T *xin = X[b & 1], *xout = X[(b + 1) & 1];
+        const uint8_t *flag = ctx->flags + b;
+        const bool gated = gating && b >= p.front_anchors && b < B - p.back_anchors;
+        const float *mb = ctx->mods + (size_t)b * 6 * d;   // shift1 scale1 gate1 shift2 scale2 gate2
+        T *rk = reinterpret_cast<T *>(ctx->ring_k) + ((size_t)b * ctx->Wkv + slot) * Ld;
+        T *rv = reinterpret_cast<T *>(ctx->ring_v) + ((size_t)b * ctx->Wkv + slot) * Ld;
+        T *rh = gated ? reinterpret_cast<T *>(ctx->rhat) + ((size_t)t * B + b) * Ld : nullptr;
+
+        if (gated) {
+            GateArgs g;
+            memset(&g, 0, sizeof g);
+            g.x = xin;
+            g.d = d;
+            g.V = ctx->V;
+            g.npc = ctx->npc;
+            g.fp_rows = ctx->fp_rows;
+            g.kfp = ctx->kfp;
+            g.n_slices = ctx->g_ns;
+            g.R = ctx->g_R;
+            const size_t cell = (size_t)t * B + b;
+            g.phi = ctx->phi + cell * 2 * ctx->phi_n_all;
+            g.phi_act = ctx->phi_act + cell * 16;
+            for (int i = 0; i < ctx->A; ++i) g.action[i] = action[i];
+            g.A = ctx->A;
+            g.cell = ctx->cells + cell;
+            g.mode = eval_mode ? 1 : 0;
+            g.step = t;
+            g.tau_floor = p.tau_floor;
+            g.margin = p.margin;
+            g.alpha = p.alpha;
+            g.tau_dev = p.tau_dev;
+            g.eps_dev = p.eps_dev;
+            g.strict_tau = p.step0_strict_tau;
+            g.max_skips = p.max_skips;
+            g.fp_refresh = p.fp_refresh;
+            g.replay = p.replay_skip != nullptr ? (p.replay_skip[b] != 0 ? 1 : 0) : -1;
+            g.flag = ctx->flags + b;
+            g.s_cos = ctx->s_cos + b;
+            g.d_max = ctx->d_max + b;
+            g.tau_out = ctx->tau + b;
+            g.colsum = ctx->g_colsum;
+            g.sp_part = ctx->g_sp;
+            g.gl_part = ctx->g_gl;
+            g.cnt_cs = ctx->g_cnt;
+            g.cnt_all = ctx->g_cnt + ctx->V * ctx->g_ns;
+            CK(gate_launch<T>(g, st));
+        }
+
+        // ---- recompute path (early-exits when flag[b] == skip)
+        CK(ln_mod<T>(xin, mb + 0 * d, mb + 1 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
+        EpiParams ep;
+        memset(&ep, 0, sizeof ep);
+        ep.M = L;
+        ep.N = 3 * d;
+        ep.bias = ctx->qkv_b + (size_t)b * 3 * d;
+        ep.out = qb;
+        ep.out_k = rk;
+        ep.out_v = rv;
+        ep.d = d;
+        ep.head_dim = hd;
+        ep.npc = ctx->npc;
+        ep.gh = ctx->cfg.grid_h;
+        ep.gw = ctx->cfg.grid_w;
+        ep.frames = ctx->cfg.frames;
+        ep.frame0 = n * ctx->cfg.frames;
+        ep.rope_freq = ctx->rope_freq;
+        ep.rope_axis = ctx->rope_axis;
+        if constexpr (sizeof(T) == 2) {
+            CK(gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
+            CK(attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L, n_keys,
+                       ctx->H, d, flag, ctx->d_err, st));
+        } else {
+            const float *W = reinterpret_cast<const float *>(ctx->qkv_wt) + (size_t)b * 3 * d * d;
+            CK(gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+            const float *Kr = reinterpret_cast<const float *>(ctx->ring_k) + (size_t)b * ctx->Wkv * Ld;
+            const float *Vr = reinterpret_cast<const float *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld;
+            CK(attn_simt(hd, reinterpret_cast<const float *>(qb), Kr, Vr, reinterpret_cast<float *>(ob), L, n_keys,
+                         ctx->H, flag, st));
+        }
+        // O projection + gated residual: x1 = x + gate1 * (o W_o + b_o)
+        memset(&ep, 0, sizeof ep);
+        ep.M = L;
+        ep.N = d;
+        ep.bias = ctx->o_b + (size_t)b * d;
+        ep.gate = mb + 2 * d;
+        ep.resid = xin;
+        ep.out = x1;
+        if constexpr (sizeof(T) == 2) {
+            CK(gemm_tc(EPI_RESID_GATE, ctx->tm_o, ctx->tm_wo[b], ep, d, flag, ctx->d_err, st));
+        } else {
+            const float *W = reinterpret_cast<const float *>(ctx->o_wt) + (size_t)b * d * d;
+            CK(gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
+        }
+        CK(ln_mod<T>(x1, mb + 3 * d, mb + 4 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
+        // FFN up: u = GELU_tanh(h2 W1 + b1)
+        memset(&ep, 0, sizeof ep);
+        ep.M = L;
+        ep.N = F;
+        ep.bias = ctx->f1_b + (size_t)b * F;
+        ep.out = ub;
+        if constexpr (sizeof(T) == 2) {
+            CK(gemm_tc(EPI_GELU, ctx->tm_h, ctx->tm_w1[b], ep, d, flag, ctx->d_err, st));
+        } else {
+            const float *W = reinterpret_cast<const float *>(ctx->f1_wt) + (size_t)b * F * d;
+            CK(gemm_simt(EPI_GELU, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+        }
+        // FFN down + gated residual; residual cache write r_hat = x2 - x (Eq. 2-3)
+        memset(&ep, 0, sizeof ep);
+        ep.M = L;
+        ep.N = d;
+        ep.bias = ctx->f2_b + (size_t)b * d;
+        ep.gate = mb + 5 * d;
+        ep.resid = x1;
+        ep.xin = xin;
+        ep.out = xout;
+        ep.rhat = rh;
+        if constexpr (sizeof(T) == 2) {
+            CK(gemm_tc(EPI_RESID_CACHE, ctx->tm_u, ctx->tm_w2[b], ep, F, flag, ctx->d_err, st));
+        } else {
+            const float *W = reinterpret_cast<const float *>(ctx->f2_wt) + (size_t)b * d * F;
+            CK(gemm_simt(EPI_RESID_CACHE, ep, reinterpret_cast<const float *>(ub), W, F, flag, st));
+        }
+        // ---- reuse path (Eq. 4), only when the gate chose skip
+        if (gated) CK(residual_reuse<T>(xin, rh, xout, (long)Ld, flag, ctx->n_sm, st));
+        if (ctx->trace != nullptr)
+            CK(cudaMemcpyAsync(reinterpret_cast<char *>(ctx->trace) + (size_t)b * Ld * sizeof(T), xout,
+                               Ld * sizeof(T), cudaMemcpyDeviceToDevice, st));
+    }
+    CK(head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
+}
+
+}  // namespace
+
+// ======================================================================= ABI
+extern "C" {
+
+void xc_gate_params_default(xc_gate_params *p) {
+    if (p == nullptr) return;
+    memset(p, 0, sizeof *p);
+    p->enabled = 1;
+    p->tau_floor = 0.97f;
+    p->margin = 0.02f;
+    p->alpha = 0.30f;
+    p->tau_dev = 2.0f;
+    p->eps_dev = 1e-6f;
+    p->front_anchors = 1;
+    p->back_anchors = 0;
+    p->warmup_chunks = 1;
+    p->max_skips = 0;
+    p->protect_step0 = 0;
+    p->step0_strict_tau = 0.0f;
+    p->fp_tokens = 32;
+    p->fp_refresh = 0;
+    p->replay_skip = nullptr;
+}
+
+const char *xc_last_error(const xc_ctx *ctx) {
+    if (ctx != nullptr) return ctx->err.c_str();
+    std::lock_guard<std::mutex> g(g_err_mu);
+    return g_global_err.c_str();
+}
+
+void xc_destroy(xc_ctx *ctx) {
+    if (ctx == nullptr) return;
+    cudaStreamSynchronize(ctx->st);
+    for (void *p : ctx->allocs) cudaFree(p);
+    if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
+    if (ctx->h_stats) cudaFreeHost(ctx->h_stats);
+    delete ctx;
+}
+
+xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_stream, xc_ctx **out) {
+    xc_ctx *ctx = nullptr;
+    if (out == nullptr || cfg == nullptr || w == nullptr) {
+        set_err(nullptr, "xc_init: NULL argument");
+        return XC_EINVAL;
+    }
+    *out = nullptr;
+    char why[256];
+    if (!cfg_ok(cfg, why, sizeof why)) {
+        set_err(nullptr, "%s", why);
+        return XC_EINVAL;
+    }
+    const float *const req[] = {w->pe_w, w->pe_b, w->t_w1, w->t_b1, w->t_w2, w->t_b2, w->a_w1, w->a_b1, w->a_w2,
+                                w->a_b2, w->mod_w, w->mod_b, w->blk_mod, w->qkv_w, w->qkv_b, w->o_w, w->o_b,
+                                w->f1_w, w->f1_b, w->f2_w, w->f2_b, w->head_w, w->head_b, w->head_tab, w->out_w,
+                                w->out_b};
+    for (const float *p : req)
+        if (p == nullptr) {
+            set_err(nullptr, "xc_init: NULL weight pointer");
+            return XC_EINVAL;
+        }
+    ctx = new xc_ctx();
+    try {
+        ctx->cfg = *cfg;
+        ctx->B = cfg->n_blocks;
+        ctx->d = cfg->d_model;
+        ctx->F = cfg->d_ffn;
+        ctx->H = cfg->n_heads;
+        ctx->hd = cfg->head_dim;
+        ctx->S = cfg->n_denoise_steps;
+        ctx->Wkv = cfg->kv_window_chunks;
+        ctx->C = cfg->c_latent;
+        ctx->A = cfg->action_dim;
+        ctx->V = cfg->n_cams;
+        ctx->npc = cfg->frames * cfg->grid_h * cfg->grid_w;
+        ctx->L = ctx->V * ctx->npc;
+        ctx->bf = cfg->dtype == XC_BF16;
+        ctx->esz = ctx->bf ? 2 : 4;
+        ctx->st = reinterpret_cast<cudaStream_t>(cuda_stream);
+        int dev = 0;
+        CK(cudaGetDevice(&dev));
+        CK(cudaDeviceGetAttribute(&ctx->n_sm, cudaDevAttrMultiProcessorCount, dev));
+        const int L = ctx->L, d = ctx->d, F = ctx->F, B = ctx->B, C = ctx->C, A = ctx->A, Tf = cfg->t_freq_dim;
+        const size_t Ld = (size_t)L * d, es = ctx->esz;
+
+        // weights
+        auto up = [&](float *&dst, const float *src, size_t n) {
+            dst = dalloc<float>(ctx, n * sizeof(float));
+            upload(ctx, dst, src, n);
+        };
+        up(ctx->pe_w, w->pe_w, (size_t)C * d);
+        up(ctx->pe_b, w->pe_b, d);
+        up(ctx->t_w1, w->t_w1, (size_t)Tf * d);
+        up(ctx->t_b1, w->t_b1, d);
+        up(ctx->t_w2, w->t_w2, (size_t)d * d);
+        up(ctx->t_b2, w->t_b2, d);
+        up(ctx->a_w1, w->a_w1, (size_t)A * d);
+        up(ctx->a_b1, w->a_b1, d);
+        up(ctx->a_w2, w->a_w2, (size_t)d * d);
+        up(ctx->a_b2, w->a_b2, d);
+        up(ctx->mod_w, w->mod_w, (size_t)d * 6 * d);
+        up(ctx->mod_b, w->mod_b, 6 * (size_t)d);
+        up(ctx->blk_mod, w->blk_mod, (size_t)B * 6 * d);
+        up(ctx->head_w, w->head_w, (size_t)d * 2 * d);
+        up(ctx->head_b, w->head_b, 2 * (size_t)d);
+        up(ctx->head_tab, w->head_tab, 2 * (size_t)d);
+        up(ctx->out_w, w->out_w, (size_t)d * C);
+        up(ctx->out_b, w->out_b, C);
+        up(ctx->qkv_b, w->qkv_b, (size_t)B * 3 * d);
+        up(ctx->o_b, w->o_b, (size_t)B * d);
+        up(ctx->f1_b, w->f1_b, (size_t)B * F);
+        up(ctx->f2_b, w->f2_b, (size_t)B * d);
+        ctx->qkv_wt = dalloc<void>(ctx, (size_t)B * 3 * d * d * es);
+        ctx->o_wt = dalloc<void>(ctx, (size_t)B * d * d * es);
+        ctx->f1_wt = dalloc<void>(ctx, (size_t)B * F * d * es);
+        ctx->f2_wt = dalloc<void>(ctx, (size_t)B * d * F * es);
+        {
+            size_t mx = (size_t)3 * d * d;
+            if ((size_t)d * F > mx) mx = (size_t)d * F;
+            float *tmp = nullptr;
+            CK(cudaMalloc(&tmp, mx * sizeof(float)));
+            try {
+                upload_blocks(ctx, ctx->qkv_wt, w->qkv_w, d, 3 * d, tmp);
+                upload_blocks(ctx, ctx->o_wt, w->o_w, d, d, tmp);
+                upload_blocks(ctx, ctx->f1_wt, w->f1_w, d, F, tmp);
+                upload_blocks(ctx, ctx->f2_wt, w->f2_w, F, d, tmp);
+            } catch (...) {
+                cudaFree(tmp);
+                throw;
+            }
+            cudaFree(tmp);
+        }
+        {
+            std::vector<float> fr;
+            std::vector<int> ax;
+            rope_table(ctx->hd, cfg->rope_theta, fr, ax);
+            ctx->rope_freq = dalloc<float>(ctx, fr.size() * sizeof(float));
+            ctx->rope_axis = dalloc<int>(ctx, ax.size() * sizeof(int));
+            CK(cudaMemcpy(ctx->rope_freq, fr.data(), fr.size() * sizeof(float), cudaMemcpyHostToDevice));
+            CK(cudaMemcpy(ctx->rope_axis, ax.data(), ax.size() * sizeof(int), cudaMemcpyHostToDevice));
+        }
+
+        // activations
+        ctx->xb[0] = dalloc<void>(ctx, Ld * es);
+        ctx->xb[1] = dalloc<void>(ctx, Ld * es);
+        ctx->x1 = dalloc<void>(ctx, Ld * es);
+        ctx->hbuf = dalloc<void>(ctx, Ld * es);
+        ctx->q = dalloc<void>(ctx, Ld * es);
+        ctx->o = dalloc<void>(ctx, Ld * es);
+        ctx->u = dalloc<void>(ctx, (size_t)L * F * es);
+        ctx->lat = dalloc<float>(ctx, (size_t)L * C * sizeof(float));
+        ctx->vout = dalloc<float>(ctx, (size_t)L * C * sizeof(float));
+        ctx->act_dev = dalloc<float>(ctx, 8 * sizeof(float));
+        ctx->temb = dalloc<float>(ctx, Tf * sizeof(float));
+        ctx->ht = dalloc<float>(ctx, d * sizeof(float));
+        ctx->ha = dalloc<float>(ctx, d * sizeof(float));
+        ctx->e1 = dalloc<float>(ctx, d * sizeof(float));
+        ctx->e = dalloc<float>(ctx, d * sizeof(float));
+        ctx->mshared = dalloc<float>(ctx, 6 * (size_t)d * sizeof(float));
+        ctx->mods = dalloc<float>(ctx, (size_t)B * 6 * d * sizeof(float));
+        ctx->hmod = dalloc<float>(ctx, 2 * (size_t)d * sizeof(float));
+
+        // ring and caches
+        ctx->ring_k = dalloc<void>(ctx, (size_t)B * ctx->Wkv * Ld * es);
+        ctx->ring_v = dalloc<void>(ctx, (size_t)B * ctx->Wkv * Ld * es);
+        ctx->rhat = dalloc<void>(ctx, (size_t)ctx->S * B * Ld * es);
+        ctx->cells = dalloc<GateCell>(ctx, (size_t)ctx->S * B * sizeof(GateCell));
+        ctx->phi_act = dalloc<float>(ctx, (size_t)ctx->S * B * 16 * sizeof(float));
+        ctx->fp_K = -1;
+        ctx->fp_rows = nullptr;
+        ctx->phi = nullptr;
+        ensure_fp(ctx, 32);
+
+        // per pass
+        ctx->flags = dalloc<uint8_t>(ctx, XC_MAX_BLOCKS);
+        ctx->s_cos = dalloc<float>(ctx, 3 * XC_MAX_BLOCKS * sizeof(float));
+        ctx->d_max = ctx->s_cos + B;
+        ctx->tau = ctx->s_cos + 2 * B;
+        ctx->d_err = dalloc<int>(ctx, sizeof(int));
+        CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
+        CK(cudaMallocHost(reinterpret_cast<void **>(&ctx->h_flags), XC_MAX_BLOCKS));
+        CK(cudaMallocHost(reinterpret_cast<void **>(&ctx->h_stats), 3 * XC_MAX_BLOCKS * sizeof(float)));
+
+        // gate scratch
+        gate_geometry(ctx->V, ctx->npc, d, ctx->n_sm, &ctx->g_ns, &ctx->g_R);
+        ctx->g_colsum = dalloc<float>(ctx, (size_t)ctx->V * ctx->g_R * d * sizeof(float));
+        ctx->g_sp = dalloc<double>(ctx, (size_t)ctx->V * ctx->g_ns * ctx->g_R * 5 * sizeof(double));
+        ctx->g_gl = dalloc<double>(ctx, (size_t)ctx->V * ctx->g_ns * 3 * sizeof(double));
+        ctx->g_cnt = dalloc<unsigned>(ctx, (size_t)(ctx->V * ctx->g_ns + 1) * sizeof(unsigned));
+
+        // tensor maps of the bf16 path
+        if (ctx->bf) {
+            tmap(ctx, &ctx->tm_h, ctx->hbuf, L, d, 128);
+            tmap(ctx, &ctx->tm_o, ctx->o, L, d, 128);
+            tmap(ctx, &ctx->tm_u, ctx->u, L, F, 128);
+            tmap(ctx, &ctx->tm_q, ctx->q, L, d, 128);
+            ctx->tm_wqkv.resize(B);
+            ctx->tm_wo.resize(B);
+            ctx->tm_w1.resize(B);
+            ctx->tm_w2.resize(B);
+            ctx->tm_rk.resize(B);
+            ctx->tm_rv.resize(B);
+            for (int b = 0; b < B; ++b) {
+                const char *wq = reinterpret_cast<const char *>(ctx->qkv_wt) + (size_t)b * 3 * d * d * es;
+                const char *wo = reinterpret_cast<const char *>(ctx->o_wt) + (size_t)b * d * d * es;
+                const char *w1 = reinterpret_cast<const char *>(ctx->f1_wt) + (size_t)b * F * d * es;
+                const char *w2 = reinterpret_cast<const char *>(ctx->f2_wt) + (size_t)b * d * F * es;
+                tmap(ctx, &ctx->tm_wqkv[b], wq, 3 * (uint64_t)d, d, 256);
+                tmap(ctx, &ctx->tm_wo[b], wo, d, d, 256);
+                tmap(ctx, &ctx->tm_w1[b], w1, F, d, 256);
+                tmap(ctx, &ctx->tm_w2[b], w2, d, F, 256);
+                const char *rk = reinterpret_cast<const char *>(ctx->ring_k) + (size_t)b * ctx->Wkv * Ld * es;
+                const char *rv = reinterpret_cast<const char *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld * es;
+                tmap(ctx, &ctx->tm_rk[b], rk, (uint64_t)ctx->Wkv * L, d, 128);
+                tmap(ctx, &ctx->tm_rv[b], rv, (uint64_t)ctx->Wkv * L, d, 128);
+            }
+        }
+        ctx->trace = nullptr;
+        clear_state(ctx);
+        CK(cudaDeviceSynchronize());
+    } catch (Fail &f) {
+        std::string msg = ctx->err;
+        xc_destroy(ctx);
+        set_err(nullptr, "%s", msg.c_str());
+        return f.st;
+    }
+    ctx->err = "no error";
+    *out = ctx;
+    return XC_OK;
+}
+
+xc_status xc_reset(xc_ctx *ctx) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_reset: NULL context");
+        return XC_ESTATE;
+    }
+    try {
+        clear_state(ctx);
+    } catch (Fail &f) {
+        return f.st;
+    }
+    return XC_OK;
+}
+
+int xc_chunk_index(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->n; }
+
+xc_status xc_set_block_trace(xc_ctx *ctx, void *dev_buf) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_set_block_trace: NULL context");
+        return XC_ESTATE;
+    }
+    ctx->trace = dev_buf;
+    return XC_OK;
+}
+
+xc_status xc_sync(xc_ctx *ctx) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_sync: NULL context");
+        return XC_ESTATE;
+    }
+    try {
+        CK(cudaStreamSynchronize(ctx->st));
+        int e = 0;
+        CK(cudaMemcpy(&e, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+        if (e != 0) {
+            CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
+            set_err(ctx, "device wait expired (error bits 0x%x)", e);
+            return XC_ETIMEOUT;
+        }
+    } catch (Fail &f) {
+        return f.st;
+    }
+    return XC_OK;
+}
+
+xc_status xc_euler_update(xc_ctx *ctx, float *x, const float *v, float dsigma, long n) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_euler_update: NULL context");
+        return XC_ESTATE;
+    }
+    if (x == nullptr || v == nullptr || n < 0) {
+        set_err(ctx, "xc_euler_update: bad argument");
+        return XC_EINVAL;
+    }
+    if (n == 0) return XC_OK;
+    try {
+        CK(euler_update(x, v, dsigma, n, ctx->st));
+    } catch (Fail &f) {
+        return f.st;
+    }
+    return XC_OK;
+}
+
+xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, float sigma, int step_index,
+                        int is_kv_update, const xc_gate_params *gate, float *v_out, xc_step_stats *stats) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_chunk_step: NULL context");
+        return XC_ESTATE;
+    }
+    if (latent == nullptr || action == nullptr) {
+        set_err(ctx, "xc_chunk_step: NULL latent or action");
+        return XC_EINVAL;
+    }
+    xc_gate_params p;
+    if (gate != nullptr)
+        p = *gate;
+    else
+        xc_gate_params_default(&p);
+    char why[256];
+    if (!gate_ok(&p, ctx->B, why, sizeof why)) {
+        set_err(ctx, "%s", why);
+        return XC_EINVAL;
+    }
+    for (int i = 0; i < ctx->A; ++i)
+        if (!std::isfinite(action[i])) {
+            set_err(ctx, "xc_chunk_step: non-finite action");
+            return XC_ENUMERIC;
+        }
+    if (!std::isfinite(sigma)) {
+        set_err(ctx, "xc_chunk_step: non-finite sigma");
+        return XC_ENUMERIC;
+    }
+    const bool kv = is_kv_update != 0;
+    if (kv) {
+        if (ctx->next_step != 0 && ctx->next_step != ctx->S) {
+            set_err(ctx, "KV-update pass before all %d denoising passes of chunk %d", ctx->S, ctx->n);
+            return XC_ESTATE;
+        }
+    } else if (step_index != ctx->next_step || step_index >= ctx->S) {
+        set_err(ctx, "denoising pass %d out of order (expected %d)", step_index, ctx->next_step);
+        return XC_ESTATE;
+    }
+    const int t = kv ? 0 : step_index;
+    try {
+        ensure_fp(ctx, p.fp_tokens);
+        const size_t lat_bytes = (size_t)ctx->L * ctx->C * sizeof(float);
+        const float *lat_dev = latent;
+        if (is_host_ptr(latent)) {
+            CK(cudaMemcpyAsync(ctx->lat, latent, lat_bytes, cudaMemcpyHostToDevice, ctx->st));
+            lat_dev = ctx->lat;
+        }
+        const bool v_host = v_out != nullptr && is_host_ptr(v_out);
+        float *v_dev = (v_out == nullptr || v_host) ? ctx->vout : v_out;
+        if (ctx->bf)
+            run_pass<bf16>(ctx, lat_dev, action, sigma, t, kv, p, v_dev);
+        else
+            run_pass<float>(ctx, lat_dev, action, sigma, t, kv, p, v_dev);
+        if (v_host) CK(cudaMemcpyAsync(v_out, ctx->vout, lat_bytes, cudaMemcpyDeviceToHost, ctx->st));
+        if (stats != nullptr) {
+            CK(cudaMemcpyAsync(ctx->h_flags, ctx->flags, ctx->B, cudaMemcpyDeviceToHost, ctx->st));
+            CK(cudaMemcpyAsync(ctx->h_stats, ctx->s_cos, 3 * ctx->B * sizeof(float), cudaMemcpyDeviceToHost,
+                               ctx->st));
+            CK(cudaStreamSynchronize(ctx->st));
+            int e = 0;
+            CK(cudaMemcpy(&e, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+            if (e != 0) {
+                CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
+                set_err(ctx, "device wait expired (error bits 0x%x)", e);
+                return XC_ETIMEOUT;
+            }
+            memset(stats, 0, sizeof *stats);
+            stats->n_blocks = ctx->B;
+            stats->chunk_index = ctx->n;
+            for (int b = 0; b < ctx->B; ++b) {
+                stats->decision[b] = ctx->h_flags[b];
+                stats->s_cos[b] = ctx->h_stats[b];
+                stats->d_max[b] = ctx->h_stats[ctx->B + b];
+                stats->tau_cos[b] = ctx->h_stats[2 * ctx->B + b];
+            }
+        }
+    } catch (Fail &f) {
+        return f.st;
+    }
+    if (kv) {
+        ctx->n += 1;
+        ctx->next_step = 0;
+    } else {
+        ctx->next_step = step_index + 1;
+    }
+    return XC_OK;
+}
+
+// ---------------------------------------------------------------- op entries
+static int *op_err_word() {
+    static int *p = nullptr;
+    if (p == nullptr) {
+        if (cudaMalloc(&p, sizeof(int)) != cudaSuccess) return nullptr;
+        cudaMemset(p, 0, sizeof(int));
+    }
+    return p;
+}
+
+int xc_op_device_error(void) {
+    int *p = op_err_word();
+    if (p == nullptr) return -1;
+    cudaDeviceSynchronize();
+    int e = 0;
+    cudaMemcpy(&e, p, sizeof(int), cudaMemcpyDeviceToHost);
+    cudaMemset(p, 0, sizeof(int));
+    return e;
+}
+
+#define OP_FAIL(code, ...)              \
+    do {                                \
+        set_err(nullptr, __VA_ARGS__);  \
+        return code;                    \
+    } while (0)
+#define OP_CK(call)                                                                        \
+    do {                                                                                   \
+        cudaError_t e_ = (call);                                                           \
+        if (e_ != cudaSuccess) OP_FAIL(XC_ECUDA, "%s: %s", #call, cudaGetErrorString(e_)); \
+    } while (0)
+
+xc_status xc_op_linear(int dtype, int epilogue, int M, int N, int K, const void *A, const void *Wt,
+                       const float *bias, const float *gate, const void *resid, const void *xin, void *out,
+                       void *rhat, void *stream) {
+    if (M < 1 || N < 16 || K < 1 || A == nullptr || Wt == nullptr || bias == nullptr || out == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_linear: bad shape or NULL pointer");
+    if (epilogue < XC_EPI_BIAS || epilogue > XC_EPI_RESID_CACHE) OP_FAIL(XC_EINVAL, "xc_op_linear: epilogue");
+    if ((epilogue == XC_EPI_RESID_GATE || epilogue == XC_EPI_RESID_CACHE) && (gate == nullptr || resid == nullptr))
+        OP_FAIL(XC_EINVAL, "xc_op_linear: gated residual needs gate and resid");
+    if (epilogue == XC_EPI_RESID_CACHE && rhat != nullptr && xin == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_linear: residual cache needs xin");
+    EpiParams ep;
+    memset(&ep, 0, sizeof ep);
+    ep.M = M;
+    ep.N = N;
+    ep.bias = bias;
+    ep.gate = gate;
+    ep.resid = resid;
+    ep.xin = xin;
+    ep.out = out;
+    ep.rhat = rhat;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == XC_BF16) {
+        if (N % 256 != 0 || K % 64 != 0) OP_FAIL(XC_EINVAL, "xc_op_linear: bf16 needs N %% 256 == 0, K %% 64 == 0");
+        CUtensorMap ta, tb;
+        if (!make_tmap_bf16(&ta, A, M, K, 128) || !make_tmap_bf16(&tb, Wt, N, K, 256))
+            OP_FAIL(XC_EINVAL, "xc_op_linear: tensor map (alignment?)");
+        OP_CK(gemm_tc(epilogue, ta, tb, ep, K, nullptr, op_err_word(), st));
+    } else if (dtype == XC_F32) {
+        if (N % 16 != 0) OP_FAIL(XC_EINVAL, "xc_op_linear: f32 needs N %% 16 == 0");
+        OP_CK(gemm_simt(epilogue, ep, reinterpret_cast<const float *>(A), reinterpret_cast<const float *>(Wt), K,
+                        nullptr, st));
+    } else {
+        OP_FAIL(XC_EINVAL, "xc_op_linear: dtype");
+    }
+    return XC_OK;
+}
+
+xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int chunk, int d, int head_dim,
+                         float rope_theta, const void *A, const void *Wt, const float *bias, void *q, void *k,
+                         void *v, void *stream) {
+    if (n_cams < 1 || frames < 1 || gh < 1 || gw < 1 || chunk < 0 || head_dim < 16 || head_dim % 16 != 0 ||
+        d % head_dim != 0 || A == nullptr || Wt == nullptr || bias == nullptr || q == nullptr || k == nullptr ||
+        v == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: bad argument");
+    static float *freq = nullptr;
+    static int *axis = nullptr;
+    static int table_hd = -1;
+    static float table_theta = 0.0f;
+    if (table_hd != head_dim || table_theta != rope_theta) {
+        std::vector<float> fr;
+        std::vector<int> ax;
+        rope_table(head_dim, rope_theta, fr, ax);
+        cudaDeviceSynchronize();
+        if (freq) cudaFree(freq);
+        if (axis) cudaFree(axis);
+        OP_CK(cudaMalloc(&freq, fr.size() * sizeof(float)));
+        OP_CK(cudaMalloc(&axis, ax.size() * sizeof(int)));
+        OP_CK(cudaMemcpy(freq, fr.data(), fr.size() * sizeof(float), cudaMemcpyHostToDevice));
+        OP_CK(cudaMemcpy(axis, ax.data(), ax.size() * sizeof(int), cudaMemcpyHostToDevice));
+        table_hd = head_dim;
+        table_theta = rope_theta;
+    }
+    const int npc = frames * gh * gw, M = n_cams * npc;
+    EpiParams ep;
+    memset(&ep, 0, sizeof ep);
+    ep.M = M;
+    ep.N = 3 * d;
+    ep.bias = bias;
+    ep.out = q;
+    ep.out_k = k;
+    ep.out_v = v;
+    ep.d = d;
+    ep.head_dim = head_dim;
+    ep.npc = npc;
+    ep.gh = gh;
+    ep.gw = gw;
+    ep.frames = frames;
+    ep.frame0 = chunk * frames;
+    ep.rope_freq = freq;
+    ep.rope_axis = axis;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == XC_BF16) {
+        if ((3 * d) % 256 != 0 || d % 64 != 0) OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: bf16 needs 3d %% 256, d %% 64");
+        CUtensorMap ta, tb;
+        if (!make_tmap_bf16(&ta, A, M, d, 128) || !make_tmap_bf16(&tb, Wt, 3 * (uint64_t)d, d, 256))
+            OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: tensor map");
+        OP_CK(gemm_tc(EPI_QKV_ROPE, ta, tb, ep, d, nullptr, op_err_word(), st));
+    } else if (dtype == XC_F32) {
+        OP_CK(gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(A), reinterpret_cast<const float *>(Wt), d,
+                        nullptr, st));
+    } else {
+        OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: dtype");
+    }
+    return XC_OK;
+}
+
+xc_status xc_op_attention(int dtype, int Lq, int n_keys, int n_heads, int head_dim, const void *q, const void *k,
+                          const void *v, void *o, void *stream) {
+    if (Lq < 1 || n_keys < 1 || n_heads < 1 || q == nullptr || k == nullptr || v == nullptr || o == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_attention: bad argument");
+    const int d = n_heads * head_dim;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == XC_BF16) {
+        if (head_dim != 64 && head_dim != 128) OP_FAIL(XC_EINVAL, "xc_op_attention: bf16 head_dim 64 or 128");
+        CUtensorMap tq, tk, tv;
+        if (!make_tmap_bf16(&tq, q, Lq, d, 128) || !make_tmap_bf16(&tk, k, n_keys, d, 128) ||
+            !make_tmap_bf16(&tv, v, n_keys, d, 128))
+            OP_FAIL(XC_EINVAL, "xc_op_attention: tensor map");
+        OP_CK(attn_tc(head_dim, tq, tk, tv, reinterpret_cast<bf16 *>(o), Lq, n_keys, n_heads, d, nullptr,
+                      op_err_word(), st));
+    } else if (dtype == XC_F32) {
+        OP_CK(attn_simt(head_dim, reinterpret_cast<const float *>(q), reinterpret_cast<const float *>(k),
+                        reinterpret_cast<const float *>(v), reinterpret_cast<float *>(o), Lq, n_keys, n_heads,
+                        nullptr, st));
+    } else {
+        OP_FAIL(XC_EINVAL, "xc_op_attention: dtype");
+    }
+    return XC_OK;
+}
+
+xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x, const float *shift, const float *scale,
+                       void *out, void *stream) {
+    if (M < 1 || d < 16 || d % 16 != 0 || x == nullptr || shift == nullptr || scale == nullptr || out == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_ln_mod: bad argument");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == XC_BF16)
+        OP_CK(ln_mod<bf16>(reinterpret_cast<const bf16 *>(x), shift, scale, reinterpret_cast<bf16 *>(out), M, d, eps,
+                           nullptr, st));
+    else if (dtype == XC_F32)
+        OP_CK(ln_mod<float>(reinterpret_cast<const float *>(x), shift, scale, reinterpret_cast<float *>(out), M, d,
+                            eps, nullptr, st));
+    else
+        OP_FAIL(XC_EINVAL, "xc_op_ln_mod: dtype");
+    return XC_OK;
+}
+
+xc_status xc_op_residual_reuse(int dtype, long n, const void *x, const void *rhat, void *out, void *stream) {
+    if (n < 0 || n % 16 != 0 || x == nullptr || rhat == nullptr || out == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_residual_reuse: bad argument (n %% 16 == 0 required)");
+    if (n == 0) return XC_OK;
+    int dev = 0, n_sm = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == XC_BF16)
+        OP_CK(residual_reuse<bf16>(reinterpret_cast<const bf16 *>(x), reinterpret_cast<const bf16 *>(rhat),
+                                   reinterpret_cast<bf16 *>(out), n, nullptr, n_sm, st));
+    else if (dtype == XC_F32)
+        OP_CK(residual_reuse<float>(reinterpret_cast<const float *>(x), reinterpret_cast<const float *>(rhat),
+                                    reinterpret_cast<float *>(out), n, nullptr, n_sm, st));
+    else
+        OP_FAIL(XC_EINVAL, "xc_op_residual_reuse: dtype");
+    return XC_OK;
+}
+
+}  // extern "C"

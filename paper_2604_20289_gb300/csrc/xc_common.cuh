@@ -1,0 +1,168 @@
+// Common device helpers of the X-Cache CUDA path (sm_103a).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/xcache.h"
+#include "../../include/xcache_ops.h"
+
+namespace xc {
+
+typedef __nv_bfloat16 bf16;
+
+// Device error word bits (bounded waits that expired, bad launch state).
+enum : int {
+    ERR_WAIT_TMA = 1,
+    ERR_WAIT_MMA = 2,
+    ERR_WAIT_EPI = 4,
+    ERR_WAIT_SOFTMAX = 8,
+    ERR_WAIT_PRODUCER = 16,
+    ERR_BAD_LAUNCH = 32,
+};
+
+// Wait limit of every spin on an mbarrier: 2 s of global time, and a hard
+// iteration cap in case the timer does not advance.
+constexpr unsigned long long WAIT_NS = 2000000000ull;
+constexpr unsigned int WAIT_MAX_ITERS = 1u << 30;
+
+// ---------------------------------------------------------------- storage
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// Round a float to the storage type and back (the value a store would keep).
+template <typename T> __device__ __forceinline__ float round_to(float v) { return to_f(from_f<T>(v)); }
+
+// Load / store a run of 16 consecutive elements (row-major, 16-element aligned).
+template <typename T> __device__ __forceinline__ void load16(const T *p, float (&v)[16]);
+template <> __device__ __forceinline__ void load16<float>(const float *p, float (&v)[16]) {
+    const float4 *q = reinterpret_cast<const float4 *>(p);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float4 t = q[i];
+        v[4 * i] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+    }
+}
+template <> __device__ __forceinline__ void load16<bf16>(const bf16 *p, float (&v)[16]) {
+    const uint4 *q = reinterpret_cast<const uint4 *>(p);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        uint4 t = q[i];
+        uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162 *>(&w[j]);
+            float2 f = __bfloat1622float2(h);
+            v[8 * i + 2 * j] = f.x;
+            v[8 * i + 2 * j + 1] = f.y;
+        }
+    }
+}
+template <typename T> __device__ __forceinline__ void store16(T *p, const float (&v)[16]);
+template <> __device__ __forceinline__ void store16<float>(float *p, const float (&v)[16]) {
+    float4 *q = reinterpret_cast<float4 *>(p);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) q[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+template <> __device__ __forceinline__ void store16<bf16>(bf16 *p, const float (&v)[16]) {
+    uint4 *q = reinterpret_cast<uint4 *>(p);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
+            w[j] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        q[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+__device__ __forceinline__ float gelu_tanh(float x) {
+    const float k0 = 0.7978845608028654f;   // sqrt(2/pi)
+    return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
+
+// ------------------------------------------------------------ GEMM epilogue
+// Everything a fused GEMM epilogue may need.  One call processes the run of
+// 16 consecutive output columns [col, col + 16) of one row.
+struct EpiParams {
+    int M, N;
+    const float *bias;         // [N]
+    const float *gate;         // [N]   adaLN-Zero gate (resid kinds)
+    const void *resid;         // [M][N] residual stream input
+    const void *xin;           // [M][N] block input (residual cache)
+    void *out;                 // [M][N]  (q for the QKV kind)
+    void *out_k;               // [M][d]  QKV kind
+    void *out_v;               // [M][d]  QKV kind
+    void *rhat;                // [M][N]  residual cache slot or nullptr
+    // RoPE geometry (QKV kind)
+    int d, head_dim, npc, gh, gw, frames, frame0;
+    const float *rope_freq;    // [head_dim/2] rotation frequency of each pair
+    const int *rope_axis;      // [head_dim/2] 0 camera, 1 frame, 2 h, 3 w
+};
+
+enum { EPI_BIAS = XC_EPI_BIAS, EPI_GELU = XC_EPI_GELU, EPI_RESID_GATE = XC_EPI_RESID_GATE,
+       EPI_RESID_CACHE = XC_EPI_RESID_CACHE, EPI_QKV_ROPE = 16 };
+
+template <int EPI, typename T>
+__device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col, float (&acc)[16]) {
+    if (row >= p.M) return;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) acc[i] += p.bias[col + i];
+    const size_t off = (size_t)row * p.N + col;
+    if constexpr (EPI == EPI_BIAS) {
+        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+    } else if constexpr (EPI == EPI_GELU) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh(acc[i]);
+        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+    } else if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
+        float r[16];
+        load16<T>(reinterpret_cast<const T *>(p.resid) + off, r);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) acc[i] = r[i] + p.gate[col + i] * acc[i];
+        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+        if constexpr (EPI == EPI_RESID_CACHE) {
+            if (p.rhat != nullptr) {
+                float xi[16];
+                load16<T>(reinterpret_cast<const T *>(p.xin) + off, xi);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) acc[i] = round_to<T>(acc[i]) - xi[i];
+                store16<T>(reinterpret_cast<T *>(p.rhat) + off, acc);
+            }
+        }
+    } else if constexpr (EPI == EPI_QKV_ROPE) {
+        const int d = p.d;
+        const int part = col / d;          // 0 q, 1 k, 2 v (16-runs never straddle: d % 16 == 0)
+        const int c = col - part * d;
+        if (part < 2) {
+            const int cam = row / p.npc;
+            const int rem = row - cam * p.npc;
+            const int f = rem / (p.gh * p.gw);
+            const int hh = (rem / p.gw) % p.gh;
+            const int ww = rem % p.gw;
+            const float pos[4] = {(float)cam, (float)(p.frame0 + f), (float)hh, (float)ww};
+            const int pair0 = (c % p.head_dim) >> 1;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int pr = pair0 + j;
+                const float ang = pos[p.rope_axis[pr]] * p.rope_freq[pr];
+                float sn, cs;
+                sincosf(ang, &sn, &cs);
+                const float x0 = acc[2 * j], x1 = acc[2 * j + 1];
+                acc[2 * j] = x0 * cs - x1 * sn;
+                acc[2 * j + 1] = x0 * sn + x1 * cs;
+            }
+        }
+        T *dst = reinterpret_cast<T *>(part == 0 ? p.out : (part == 1 ? p.out_k : p.out_v));
+        store16<T>(dst + (size_t)row * d + c, acc);
+    }
+}
+
+}  // namespace xc

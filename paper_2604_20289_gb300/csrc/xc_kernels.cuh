@@ -1,0 +1,65 @@
+// Launchers of the X-Cache kernels (k_*.cu) and the gate's device structs.
+#pragma once
+#include <cuda.h>
+
+#include "xc_common.cuh"
+
+namespace xc {
+// Per-(t, b) gate state: EMA of the cosine (Eq. 8), has-history bit,
+// consecutive-skip counter, cache-valid bit, active fingerprint half.
+struct GateCell {
+    double ema;
+    int has_hist, stale, valid, active;
+    int pad[2];
+};
+struct GateArgs {
+    const void *x;
+    int d, V, npc;
+    const int *fp_rows;
+    int kfp;
+    int n_slices, R;
+    float *phi;
+    float *phi_act;
+    float action[8];
+    int A;
+    GateCell *cell;
+    int mode;
+    int step;
+    float tau_floor, margin, alpha, tau_dev, eps_dev, strict_tau;
+    int max_skips, fp_refresh, replay;
+    uint8_t *flag;
+    float *s_cos, *d_max, *tau_out;
+    float *colsum;
+    double *sp_part;
+    double *gl_part;
+    unsigned *cnt_cs;
+    unsigned *cnt_all;
+};
+void gate_geometry(int V, int npc, int d, int n_sm, int *n_slices, int *R);
+template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);
+bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+                    const uint8_t *skip, int *err, cudaStream_t st);
+cudaError_t attn_tc(int head_dim, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, bf16 *o,
+                    int Lq, int n_keys, int n_heads, int d, const uint8_t *skip, int *err, cudaStream_t st);
+cudaError_t gemm_simt(int epi, const EpiParams &ep, const float *A, const float *Wt, int K, const uint8_t *skip,
+                      cudaStream_t st);
+cudaError_t attn_simt(int head_dim, const float *q, const float *k, const float *v, float *o, int Lq, int n_keys,
+                      int H, const uint8_t *skip, cudaStream_t st);
+template <typename T>
+cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st);
+template <typename T>
+cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
+                   const uint8_t *skip, cudaStream_t st);
+template <typename T>
+cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t *skip, int n_sm, cudaStream_t st);
+cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_t st);
+cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st);
+cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
+                 int n_out, int act_out, cudaStream_t st);
+cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, int d, cudaStream_t st);
+template <typename T>
+cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
+                 cudaStream_t st);
+template <typename T> cudaError_t transpose_convert(const float *W, T *Wt, int K, int N, cudaStream_t st);
+}  // namespace xc

@@ -1,0 +1,222 @@
+"""Chunk-step parity: AR rollouts through xc_chunk_step against the CPU oracle.
+
+Tolerances (the benchmark spec): fp32 model max|err| <= 1e-4 x output RMS; bf16
+model per-block rel-L2 <= 1e-2 and final-latent rel-L2 <= 3e-2; gate
+decisions identical except where the oracle's metric lies within 1e-3
+relative of its threshold.  Numerics are compared in decision-replay mode
+(the GPU takes the oracle's decisions), decisions in free-running mode.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+import oracle as O  # noqa: E402
+import xc_inputs as X  # noqa: E402
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2604_20289_gb300 import xcache as xb  # noqa: E402
+from paper_2604_20289_gb300.rollout import rollout as gpu_rollout  # noqa: E402
+
+FORCE_RECOMPUTE = dict(tau_floor=2.0)
+FORCE_REUSE = dict(tau_floor=-2.0, margin=10.0, tau_dev=1e30)
+
+
+def params(**kw):
+    """The same knobs for both sides, rounded to the C ABI's float32."""
+    kw = {k: (float(np.float32(v)) if isinstance(v, float) else v) for k, v in kw.items()}
+    return O.GateParams(**kw), xb.gate_params(**kw)
+
+
+_MODELS = {}
+
+
+def model(cfg):
+    if cfg.name not in _MODELS:
+        w = X.make_weights(cfg)
+        _MODELS[cfg.name] = (w, xb.XCache(cfg, w))
+    w, xc = _MODELS[cfg.name]
+    xc.reset()
+    return w, xc
+
+
+def rel_l2(a, b):
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def decisions(stats):
+    return np.array([[s["decision"] for s in ch] for ch in stats])
+
+
+def excused(o_st, b, p):
+    """Oracle metric within 1e-3 relative of its threshold (decision excused)."""
+    s, d, tau = o_st["s_cos"][b], o_st["d_max"][b], o_st["tau"][b]
+    return abs(s - tau) <= 1e-3 * abs(tau) or abs(d - p.tau_dev) <= 1e-3 * abs(p.tau_dev)
+
+
+def compare_decisions(o_stats, g_stats, p):
+    """Decisions agree pass by pass until the first excused disagreement
+    (after which the two rollouts legitimately diverge)."""
+    for n, (och, gch) in enumerate(zip(o_stats, g_stats)):
+        for t, (os_, gs) in enumerate(zip(och, gch)):
+            for b in range(len(os_["decision"])):
+                if os_["decision"][b] != gs["decision"][b]:
+                    assert os_["decision"][b] != O.Decision.FORCED and excused(os_, b, p), (n, t, b, os_, gs)
+                    return n, t
+                if os_["decision"][b] != O.Decision.FORCED:
+                    assert abs(gs["s_cos"][b] - os_["s_cos"][b]) <= 2e-3, (n, t, b)
+    return None
+
+
+def replay_of(o_stats):
+    return [[[d == O.Decision.SKIP for d in s["decision"]] for s in ch[:-1]] for ch in o_stats]
+
+
+# ------------------------------------------------------ fp32 tiny model
+@pytest.mark.parametrize("mode", ["recompute", "reuse", "mixed", "off", "safety"])
+def test_tiny_f32_rollout_parity(mode):
+    cfg = X.TINY_F32
+    kw = {"recompute": FORCE_RECOMPUTE, "reuse": FORCE_REUSE, "off": dict(enabled=False),
+          "mixed": dict(tau_floor=0.93, tau_dev=10.0),
+          "safety": dict(tau_floor=0.5, margin=1.0, tau_dev=100.0, max_skips=1, protect_step0=True,
+                         back_anchors=0, front_anchors=0)}[mode]
+    op, gp = params(**kw)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg)
+    ref = O.rollout(cfg, w, traj, op, cfg.n_chunks)
+    free = gpu_rollout(xc, traj, cfg.n_chunks, gp)
+    compare_decisions(ref["stats"], free["stats"], op)
+    xc.reset()
+    rep = gpu_rollout(xc, traj, cfg.n_chunks, gp, replay=replay_of(ref["stats"]))
+    np.testing.assert_array_equal(decisions(rep["stats"]), decisions(ref["stats"]))
+    for n in range(cfg.n_chunks):
+        want, got = ref["final"][n], rep["final"][n]
+        rms = np.sqrt(np.mean(want ** 2))
+        assert np.max(np.abs(got - want)) <= 1e-4 * rms, (n, np.max(np.abs(got - want)) / rms)
+    dec = decisions(ref["stats"])
+    if mode == "mixed":
+        assert (dec == O.Decision.SKIP).any() and (dec == O.Decision.COMPUTE).any()
+    if mode == "reuse":
+        assert (dec[1:, :4, 1:] == O.Decision.SKIP).all()
+
+
+# ------------------------------------------------------ bf16 mid models
+@pytest.mark.parametrize("cfg", [X.MID_HD64, X.MID_HD128], ids=lambda c: c.name)
+def test_mid_bf16_per_block_parity(cfg):
+    op, gp = params(tau_floor=0.92, tau_dev=10.0)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg)
+    ref = O.rollout(cfg, w, traj, op, cfg.n_chunks, keep_trace=True)
+    rep = gpu_rollout(xc, traj, cfg.n_chunks, gp, replay=replay_of(ref["stats"]), keep_trace=True)
+    worst = 0.0
+    for n in range(cfg.n_chunks):
+        for t in range(cfg.n_steps):
+            for b in range(cfg.n_blocks):
+                e = rel_l2(rep["trace"][n][t][b], ref["trace"][n][t][b])
+                worst = max(worst, e)
+                assert e <= 1e-2, (n, t, b, e)
+        assert rel_l2(rep["final"][n], ref["final"][n]) <= 3e-2
+    dec = decisions(ref["stats"])
+    assert (dec == O.Decision.SKIP).any()
+    xc.reset()
+    free = gpu_rollout(xc, traj, cfg.n_chunks, gp)
+    compare_decisions(ref["stats"], free["stats"], op)
+
+
+# ----------------------------------------------------- GPU invariants
+@pytest.mark.parametrize("cfg", [X.TINY_F32, X.MID_HD64], ids=lambda c: c.name)
+def test_force_recompute_bitwise_equals_no_cache(cfg):
+    _, g_off = params(enabled=False)
+    _, g_fc = params(**FORCE_RECOMPUTE)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=3)
+    a = gpu_rollout(xc, traj, 3, g_off)
+    xc.reset()
+    b = gpu_rollout(xc, traj, 3, g_fc)
+    for x, y in zip(a["final"], b["final"]):
+        np.testing.assert_array_equal(x, y)
+    dec = decisions(b["stats"])
+    assert not (dec == xb.XC_DEC_SKIP).any()
+    assert (dec[:, 4, :] == xb.XC_DEC_FORCED).all()          # KV-update passes
+    assert (dec[0] == xb.XC_DEC_FORCED).all()                # warmup chunk
+
+
+@pytest.mark.parametrize("cfg", [X.TINY_F32, X.MID_HD64], ids=lambda c: c.name)
+def test_force_reuse_block_output_is_input_plus_residual(cfg):
+    _, gp = params(**FORCE_REUSE)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=3)
+    r = gpu_rollout(xc, traj, 3, gp, keep_trace=True)
+    Rd = O.to_bf16 if cfg.dtype == "bf16" else (lambda v: v.astype(np.float32).astype(np.float64))
+    dec = decisions(r["stats"])
+    assert (dec[:, 4, :] == xb.XC_DEC_FORCED).all()
+    for n in (1, 2):
+        for t in range(cfg.n_steps):
+            for b in range(1, cfg.n_blocks):
+                assert dec[n, t, b] == xb.XC_DEC_SKIP
+                r_hat = Rd(r["trace"][0][t][b] - r["trace"][0][t][b - 1])
+                want = Rd(r["trace"][n][t][b - 1] + r_hat)
+                np.testing.assert_array_equal(r["trace"][n][t][b], want)
+
+
+def test_host_buffers_match_device_buffers():
+    cfg = X.MID_HD64
+    w, xc = model(cfg)
+    _, gp = params(tau_floor=0.92, tau_dev=10.0)
+    traj = X.Trajectory(cfg, n_chunks=2)
+    dev_r = gpu_rollout(xc, traj, 2, gp)
+    xc.reset()
+    S = cfg.n_steps
+    sig = (1.0, 0.75, 0.5, 0.25, 0.0)
+    finals = []
+    for n in range(2):
+        x = traj.noise(n).astype(np.float32).copy()
+        v = np.empty_like(x)
+        for t in range(S):
+            xc.chunk_step(x, traj.action(n), sig[t], t, False, gp, v_out=v)
+            x = (x + np.float32(sig[t + 1] - sig[t]) * v).astype(np.float32)
+        xc.chunk_step(traj.clean(n).astype(np.float32), traj.action(n), 0.0, S, True, gp)
+        finals.append(x.astype(np.float64))
+    for a, b in zip(dev_r["final"], finals):
+        np.testing.assert_allclose(b, a, rtol=0, atol=1e-5 * np.abs(a).max())
+
+
+def test_call_order_and_argument_errors():
+    cfg = X.TINY_F32
+    w, xc = model(cfg)
+    x = torch.zeros(cfg.tokens, cfg.c_latent, device="cuda")
+    a = np.zeros(2, np.float32)
+    with pytest.raises(xb.XCacheError) as e:
+        xc.chunk_step(x, a, 0.75, 1, False)
+    assert e.value.status == xb.XC_ESTATE
+    xc.chunk_step(x, a, 1.0, 0, False)
+    with pytest.raises(xb.XCacheError) as e:
+        xc.chunk_step(x, a, 0.0, 0, True)                     # KV pass before all 4 passes
+    assert e.value.status == xb.XC_ESTATE
+    with pytest.raises(xb.XCacheError) as e:
+        xc.chunk_step(x, np.array([np.nan, 0], np.float32), 0.75, 1, False)
+    assert e.value.status == xb.XC_ENUMERIC
+    with pytest.raises(xb.XCacheError) as e:
+        xc.chunk_step(x, a, 0.75, 1, False, xb.gate_params(alpha=2.0))
+    assert e.value.status == xb.XC_EINVAL
+    xc.sync()
+    xc.reset()
+    assert xc.chunk_index == 0
+    xc.chunk_step(x, a, 0.0, 0, True)                         # a KV-only priming chunk is allowed
+    assert xc.chunk_index == 1
+
+
+def test_reset_reproduces_rollout():
+    cfg = X.MID_HD64
+    w, xc = model(cfg)
+    _, gp = params(tau_floor=0.92, tau_dev=10.0)
+    traj = X.Trajectory(cfg, n_chunks=3)
+    a = gpu_rollout(xc, traj, 3, gp)
+    xc.reset()
+    b = gpu_rollout(xc, traj, 3, gp)
+    for x, y in zip(a["final"], b["final"]):
+        np.testing.assert_array_equal(x, y)
+    np.testing.assert_array_equal(decisions(a["stats"]), decisions(b["stats"]))

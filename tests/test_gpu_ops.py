@@ -1,0 +1,241 @@
+"""Operator parity: each kernel of the chunk step (through the C ABI) against
+the CPU oracle's primitives on the same seeded inputs -- mid sizes that span
+several tiles plus ragged tails, edge cases, and the full workload sizes on
+sampled outputs.
+
+Tolerances (written here, derived from the arithmetic):
+* bf16 outputs: both sides round the same fp32/fp64 value to bf16, so they
+  differ by at most one bf16 ulp where the fp32 accumulation lands on the
+  other side of a rounding boundary: rel-L2 <= 2e-3 (GEMM, LN) and a max
+  error of 1.5 bf16 ulps of the output scale.
+* attention: P is rounded to bf16 before P V (fp32 row sums), so each output
+  carries ~2^-9 relative noise averaged over the keys: rel-L2 <= 5e-3.
+* fp32 outputs: fp32 vs fp64 accumulation over K <= 2048 terms: rel-L2 <= 2e-6.
+"""
+import math
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+import oracle as O  # noqa: E402
+import xc_inputs as X  # noqa: E402
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2604_20289_gb300 import xcache as xb  # noqa: E402
+
+DEV = torch.device("cuda")
+
+
+def rt(name, shape, std=1.0, bf16=True, seed=7):
+    return X.random_tensor(seed, name, shape, std=std, bf16=bf16)
+
+
+def dev(a, dtype):
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(DEV)
+    return t.to(torch.bfloat16) if dtype == "bf16" else t
+
+
+def host(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def rel_l2(a, b):
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def R(dtype):
+    return O.to_bf16 if dtype == "bf16" else (lambda a: np.asarray(a, np.float64))
+
+
+def assert_close(got, want, dtype, rel=2e-3, ulps=1.5):
+    if dtype == "bf16":
+        assert rel_l2(got, want) <= rel, rel_l2(got, want)
+        scale = np.max(np.abs(want))
+        assert np.max(np.abs(got - want)) <= ulps * scale * 2.0 ** -7
+    else:
+        assert rel_l2(got, want) <= 2e-6, rel_l2(got, want)
+    assert xb.op_device_error() == 0
+
+
+# ------------------------------------------------------------------- GEMM
+GEMM_CASES = [("bf16", 840, 768, 256), ("bf16", 1000, 256, 1024), ("bf16", 77, 512, 64),
+              ("f32", 64, 192, 64), ("f32", 70, 256, 256)]
+
+
+@pytest.mark.parametrize("dtype,M,N,K", GEMM_CASES)
+@pytest.mark.parametrize("epi", [xb.XC_EPI_BIAS, xb.XC_EPI_GELU, xb.XC_EPI_RESID_GATE,
+                                 xb.XC_EPI_RESID_CACHE])
+def test_linear_epilogues(dtype, M, N, K, epi):
+    bf = dtype == "bf16"
+    A = rt(f"A{M}{K}", (M, K), bf16=bf)
+    Wt = rt(f"W{N}{K}", (N, K), std=1 / math.sqrt(K), bf16=bf)
+    b = rt(f"b{N}", (N,), std=0.1, bf16=False)
+    g = rt(f"g{N}", (N,), std=0.5, bf16=False)
+    res = rt(f"r{M}{N}", (M, N), bf16=bf)
+    xin = rt(f"x{M}{N}", (M, N), bf16=bf)
+    out = torch.empty(M, N, device=DEV, dtype=torch.bfloat16 if bf else torch.float32)
+    rh = torch.empty_like(out)
+    xb.op_linear(dtype, epi, dev(A, dtype), dev(Wt, dtype), dev(b, "f32"), out, gate=dev(g, "f32"),
+                 resid=dev(res, dtype), xin=dev(xin, dtype), rhat=rh)
+    torch.cuda.synchronize()
+    Rd = R(dtype)
+    y = A.astype(np.float64) @ Wt.astype(np.float64).T + b
+    if epi == xb.XC_EPI_BIAS:
+        want = Rd(y)
+    elif epi == xb.XC_EPI_GELU:
+        want = Rd(O.gelu_tanh(y))
+    else:
+        want = Rd(res + g * y)
+    assert_close(host(out), want, dtype)
+    if epi == xb.XC_EPI_RESID_CACHE:
+        # r_hat = round(x_out) - x_in, from the stored output (Eq. 2-3)
+        if bf:
+            want_r = Rd(host(out) - xin)
+        else:
+            want_r = (host(out).astype(np.float32) - xin.astype(np.float32)).astype(np.float64)
+        np.testing.assert_array_equal(host(rh), want_r)
+
+
+# ------------------------------------------------------------- QKV + RoPE
+@pytest.mark.parametrize("dtype,cams,frames,gh,gw,d,hd,chunk", [
+    ("bf16", 2, 3, 10, 14, 256, 64, 5), ("bf16", 2, 3, 10, 14, 256, 128, 0),
+    ("bf16", 1, 3, 16, 28, 512, 64, 41), ("f32", 2, 2, 4, 4, 64, 16, 7)])
+def test_qkv_rope(dtype, cams, frames, gh, gw, d, hd, chunk):
+    bf = dtype == "bf16"
+    M = cams * frames * gh * gw
+    A = rt(f"qa{M}{d}", (M, d), bf16=bf)
+    Wt = rt(f"qw{d}", (3 * d, d), std=1 / math.sqrt(d), bf16=bf)
+    b = rt(f"qb{d}", (3 * d,), std=0.1, bf16=False)
+    q, k, v = (torch.empty(M, d, device=DEV, dtype=torch.bfloat16 if bf else torch.float32)
+               for _ in range(3))
+    xb.op_qkv_rope(dtype, cams, frames, gh, gw, chunk, hd, 1e4, dev(A, dtype), dev(Wt, dtype),
+                   dev(b, "f32"), q, k, v)
+    torch.cuda.synchronize()
+    y = A.astype(np.float64) @ Wt.astype(np.float64).T + b
+    pos = O.token_positions(cams, frames, gh, gw, chunk)
+    H = d // hd
+    Rd = R(dtype)
+    wq = Rd(O.apply_rope(y[:, :d].reshape(M, H, hd), pos, 1e4).reshape(M, d))
+    wk = Rd(O.apply_rope(y[:, d:2 * d].reshape(M, H, hd), pos, 1e4).reshape(M, d))
+    wv = Rd(y[:, 2 * d:])
+    for got, want in ((q, wq), (k, wk), (v, wv)):
+        assert_close(host(got), want, dtype, rel=3e-3)
+
+
+# -------------------------------------------------------------- attention
+ATTN_CASES = [("bf16", 840, 2520, 4, 64), ("bf16", 840, 2520, 2, 128), ("bf16", 100, 60, 2, 64),
+              ("bf16", 1, 1, 1, 128), ("bf16", 129, 257, 3, 64), ("f32", 64, 192, 4, 16),
+              ("f32", 33, 70, 2, 64)]
+
+
+@pytest.mark.parametrize("dtype,Lq,Lk,H,hd", ATTN_CASES)
+def test_attention(dtype, Lq, Lk, H, hd):
+    bf = dtype == "bf16"
+    d = H * hd
+    q = rt(f"aq{Lq}{d}", (Lq, d), bf16=bf)
+    k = rt(f"ak{Lk}{d}", (Lk, d), bf16=bf)
+    v = rt(f"av{Lk}{d}", (Lk, d), bf16=bf)
+    o = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16 if bf else torch.float32)
+    xb.op_attention(dtype, H, hd, dev(q, dtype), dev(k, dtype), dev(v, dtype), o)
+    torch.cuda.synchronize()
+    want = R(dtype)(O.attention(q.reshape(Lq, H, hd).astype(np.float64), k.reshape(Lk, H, hd).astype(np.float64),
+                                v.reshape(Lk, H, hd).astype(np.float64)).reshape(Lq, d))
+    got = host(o)
+    if bf:
+        assert rel_l2(got, want) <= 5e-3, rel_l2(got, want)
+    else:
+        assert rel_l2(got, want) <= 2e-6
+    assert xb.op_device_error() == 0
+
+
+def test_attention_sharp_softmax_rescaling():
+    """Scores with a growing running max across key tiles exercise the O
+    rescale; one dominant key per query makes the output that key's value."""
+    Lq, Lk, H, hd = 128, 1024, 1, 64
+    q = rt("sq", (Lq, hd), bf16=True)
+    k = rt("sk", (Lk, hd), std=0.05, bf16=True)
+    hot = np.arange(Lq) * 5 + 300                       # later tiles hold the maxima
+    k[hot] = X.bf16_representable((q * 4.0).astype(np.float32))
+    v = rt("sv", (Lk, hd), bf16=True)
+    o = torch.empty(Lq, hd, device=DEV, dtype=torch.bfloat16)
+    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o)
+    torch.cuda.synchronize()
+    want = O.to_bf16(O.attention(q[:, None].astype(np.float64), k[:, None].astype(np.float64),
+                                 v[:, None].astype(np.float64))[:, 0])
+    assert rel_l2(host(o), want) <= 5e-3
+
+
+# --------------------------------------------------- LN modulation, reuse
+@pytest.mark.parametrize("dtype,M,d", [("bf16", 840, 256), ("bf16", 301, 1536), ("bf16", 17, 5120),
+                                       ("f32", 64, 64)])
+def test_ln_mod(dtype, M, d):
+    bf = dtype == "bf16"
+    x = rt(f"lx{M}{d}", (M, d), std=2.0, bf16=bf) + 0.5
+    x = X.bf16_representable(x) if bf else x
+    sh = rt(f"lsh{d}", (d,), std=0.3, bf16=False)
+    sc = rt(f"lsc{d}", (d,), std=0.3, bf16=False)
+    out = torch.empty(M, d, device=DEV, dtype=torch.bfloat16 if bf else torch.float32)
+    xb.op_ln_mod(dtype, dev(x, dtype), dev(sh, "f32"), dev(sc, "f32"), out, eps=1e-6)
+    torch.cuda.synchronize()
+    want = R(dtype)(O.layer_norm(x, 1e-6) * (1 + sc) + sh)
+    assert_close(host(out), want, dtype)
+
+
+@pytest.mark.parametrize("dtype,n", [("bf16", 840 * 256), ("bf16", 16), ("f32", 64 * 64)])
+def test_residual_reuse_exact(dtype, n):
+    bf = dtype == "bf16"
+    x = rt(f"rx{n}", (n,), bf16=bf)
+    r = rt(f"rr{n}", (n,), std=0.3, bf16=bf)
+    out = torch.empty(n, device=DEV, dtype=torch.bfloat16 if bf else torch.float32)
+    xb.op_residual_reuse(dtype, dev(x, dtype), dev(r, dtype), out)
+    torch.cuda.synchronize()
+    want = O.to_bf16(x.astype(np.float64) + r) if bf else (x + r).astype(np.float32).astype(np.float64)
+    np.testing.assert_array_equal(host(out), want)
+
+
+# ------------------------------------------- full workload sizes, sampled
+@pytest.mark.parametrize("Lq,Lk,H,hd", [(8064, 32256, 8, 64), (12960, 38880, 12, 128)])
+def test_attention_full_size_sampled(Lq, Lk, H, hd):
+    d = H * hd
+    q = rt(f"Fq{Lq}{d}", (Lq, d))
+    k = rt(f"Fk{Lk}{d}", (Lk, d))
+    v = rt(f"Fv{Lk}{d}", (Lk, d))
+    o = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
+    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o)
+    torch.cuda.synchronize()
+    rows = np.unique(np.r_[0, 127, 128, Lq - 1, np.random.default_rng(3).integers(0, Lq, 60)])
+    want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64),
+                                 k.reshape(Lk, H, hd).astype(np.float64),
+                                 v.reshape(Lk, H, hd).astype(np.float64)).reshape(len(rows), d))
+    assert rel_l2(host(o)[rows], want) <= 5e-3
+    assert xb.op_device_error() == 0
+
+
+@pytest.mark.parametrize("M,N,K,epi", [(8064, 2048, 512, xb.XC_EPI_GELU),
+                                       (12960, 1536, 8960, xb.XC_EPI_RESID_CACHE),
+                                       (12960, 4608, 1536, xb.XC_EPI_BIAS)])
+def test_linear_full_size_sampled(M, N, K, epi):
+    A = rt(f"FA{M}{K}", (M, K))
+    Wt = rt(f"FW{N}{K}", (N, K), std=1 / math.sqrt(K))
+    b = rt(f"Fb{N}", (N,), std=0.1, bf16=False)
+    g = rt(f"Fg{N}", (N,), std=0.5, bf16=False)
+    res = rt(f"Fr{M}{N}", (M, N))
+    out = torch.empty(M, N, device=DEV, dtype=torch.bfloat16)
+    rh = torch.empty_like(out)
+    xb.op_linear("bf16", epi, dev(A, "bf16"), dev(Wt, "bf16"), dev(b, "f32"), out, gate=dev(g, "f32"),
+                 resid=dev(res, "bf16"), xin=dev(res, "bf16"), rhat=rh)
+    torch.cuda.synchronize()
+    rows = np.unique(np.r_[0, 127, 128, M - 1, np.random.default_rng(4).integers(0, M, 100)])
+    y = A[rows].astype(np.float64) @ Wt.astype(np.float64).T + b
+    if epi == xb.XC_EPI_GELU:
+        want = O.to_bf16(O.gelu_tanh(y))
+    elif epi == xb.XC_EPI_BIAS:
+        want = O.to_bf16(y)
+    else:
+        want = O.to_bf16(res[rows] + g * y)
+    assert_close(host(out)[rows], want, "bf16")

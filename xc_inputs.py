@@ -24,6 +24,8 @@ from __future__ import annotations
 
 import dataclasses
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass
 
 import numpy as np
@@ -62,14 +64,24 @@ def uniform(seed: int, name: str, n: int, offset: int = 0) -> np.ndarray:
 
 
 def normal(seed: int, name: str, n: int, offset: int = 0) -> np.ndarray:
-    """n standard normals; normal j uses uniforms 2(offset+j), 2(offset+j)+1."""
+    """n standard normals; normal j uses uniforms 2(offset+j), 2(offset+j)+1.
+    Large requests are filled in parallel blocks (numpy releases the GIL);
+    the values do not depend on the number of threads."""
     out = np.empty(n, dtype=np.float64)
-    step = 1 << 22
-    for a in range(0, n, step):
+    step = 1 << 20
+
+    def fill(a: int):
         m = min(step, n - a)
         u = uniform(seed, name, 2 * m, 2 * (offset + a))
-        u1, u2 = u[0::2], u[1::2]
-        out[a:a + m] = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * math.pi * u2)
+        out[a:a + m] = np.sqrt(-2.0 * np.log(u[0::2])) * np.cos(2.0 * math.pi * u[1::2])
+
+    starts = range(0, n, step)
+    if n <= 2 * step:
+        for a in starts:
+            fill(a)
+    else:
+        with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+            list(ex.map(fill, starts))
     return out
 
 
