@@ -19,7 +19,9 @@
  *  - Work is asynchronous on the stream given to xc_init (a cudaStream_t,
  *    NULL = legacy default stream) unless a call says otherwise.
  *  - Pointers marked "host or device" are classified with
- *    cudaPointerGetAttributes; host buffers are staged through the context.
+ *    cudaPointerGetAttributes; host buffers are staged through the context
+ *    and a call given a host buffer synchronises with its stream before it
+ *    returns, so the caller may reuse or read that buffer immediately.
  *  - The context owns its copies of the weights, the KV ring, the residual
  *    and fingerprint caches and all scratch; callers own every buffer they pass.
  */
@@ -179,6 +181,36 @@ xc_status xc_sync(xc_ctx *ctx);
 
 /* Chunk counter n (number of completed KV-update passes since reset). */
 int xc_chunk_index(const xc_ctx *ctx);
+
+/* ---- measurement (no counterpart in the paper; used by the benchmark) ---- */
+
+/* Kernel kinds of one forward pass. */
+typedef enum {
+    XC_K_COND = 0, XC_K_EMBED, XC_K_GATE, XC_K_LN, XC_K_QKV, XC_K_ATTN, XC_K_OPROJ,
+    XC_K_FFN1, XC_K_FFN2, XC_K_REUSE, XC_K_HEAD, XC_K_COUNT
+} xc_kernel_kind;
+
+/* One timed launch: CUDA-event duration on the context's stream, the block
+ * and pass it belongs to, the gate decision of that block in that pass
+ * (xc_decision; kernels of a skipped block exit at once), the chunk index
+ * and the number of resident keys the pass attended to. */
+typedef struct {
+    int kind, block, pass_seq, decision, chunk, n_keys;
+    float ms;
+} xc_profile_rec;
+
+/* Starts recording events around every launch whose kind bit is set in
+ * kind_mask (1 << xc_kernel_kind), for at most `capacity` launches; resets
+ * the pass sequence.  Errors: XC_EINVAL (capacity < 1), XC_ENOMEM. */
+xc_status xc_profile_start(xc_ctx *ctx, unsigned kind_mask, int capacity);
+
+/* Stops recording, synchronises and copies up to `max` records to `out`
+ * (host); *n_out receives the number recorded.  Frees the events. */
+xc_status xc_profile_stop(xc_ctx *ctx, xc_profile_rec *out, int max, int *n_out);
+
+/* Number of kernel launches this context has issued since xc_init
+ * (including early-exit launches of skipped blocks). */
+long long xc_launch_count(const xc_ctx *ctx);
 
 #ifdef __cplusplus
 }

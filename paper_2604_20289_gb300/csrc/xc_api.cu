@@ -143,6 +143,15 @@ struct xc_ctx {
     int n, next_step;
     void *trace;
     std::string err;
+
+    // measurement: launch counter, optional per-launch CUDA events
+    long long launches;
+    bool prof_on;
+    unsigned prof_mask;
+    int prof_cap, prof_n, pass_seq, cur_keys;
+    std::vector<cudaEvent_t> prof_ev;
+    std::vector<xc_profile_rec> prof_rec;
+    uint8_t *dec_log;                          // device [prof_cap][B]
 };
 
 namespace {
@@ -283,6 +292,34 @@ void tmap(xc_ctx *ctx, CUtensorMap *m, const void *base, uint64_t rows, uint64_t
     }
 }
 
+// Profiling hooks: an event pair around one launch when its kind is selected.
+int prof_begin(xc_ctx *ctx, int kind, int block) {
+    if (!ctx->prof_on || !(ctx->prof_mask & (1u << kind)) || ctx->prof_n >= ctx->prof_cap) return -1;
+    const int i = ctx->prof_n++;
+    CK(cudaEventRecord(ctx->prof_ev[2 * i], ctx->st));
+    xc_profile_rec &r = ctx->prof_rec[i];
+    r.kind = kind;
+    r.block = block;
+    r.pass_seq = ctx->pass_seq;
+    r.decision = -1;
+    r.chunk = ctx->n;
+    r.n_keys = ctx->cur_keys;
+    r.ms = 0.0f;
+    return i;
+}
+void prof_end(xc_ctx *ctx, int i) {
+    if (i >= 0) CK(cudaEventRecord(ctx->prof_ev[2 * i + 1], ctx->st));
+}
+
+// Launch `call` (n_launch kernels) with optional events and the launch count.
+#define LAUNCH(kind, block, n_launch, call)        \
+    do {                                           \
+        const int pi_ = prof_begin(ctx, kind, block); \
+        CK(call);                                  \
+        prof_end(ctx, pi_);                        \
+        ctx->launches += (n_launch);               \
+    } while (0)
+
 template <typename T>
 void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigma, int t, bool kv,
               const xc_gate_params &p, float *v_dev) {
@@ -293,20 +330,26 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     const int slot = n % ctx->Wkv;
     const int n_res = (n + 1 < ctx->Wkv ? n + 1 : ctx->Wkv);
     const int n_keys = n_res * L;
+    ctx->cur_keys = n_keys;
 
     // conditioning c_t: timestep + action embeddings -> adaLN-Zero vectors
     CK(cudaMemcpyAsync(ctx->act_dev, action, ctx->A * sizeof(float), cudaMemcpyHostToDevice, st));
-    CK(timestep_embedding(sigma, ctx->temb, ctx->cfg.t_freq_dim, st));
-    CK(gemv(ctx->temb, 0, ctx->t_w1, ctx->t_b1, nullptr, ctx->ht, ctx->cfg.t_freq_dim, d, 1, st));
-    CK(gemv(ctx->act_dev, 0, ctx->a_w1, ctx->a_b1, nullptr, ctx->ha, ctx->A, d, 1, st));
-    CK(gemv(ctx->ht, 0, ctx->t_w2, ctx->t_b2, nullptr, ctx->e1, d, d, 0, st));
-    CK(gemv(ctx->ha, 0, ctx->a_w2, ctx->a_b2, ctx->e1, ctx->e, d, d, 0, st));
-    CK(gemv(ctx->e, 1, ctx->mod_w, ctx->mod_b, nullptr, ctx->mshared, d, 6 * d, 0, st));
-    CK(gemv(ctx->e, 1, ctx->head_w, ctx->head_b, ctx->head_tab, ctx->hmod, d, 2 * d, 0, st));
-    CK(assemble_mods(ctx->mshared, ctx->blk_mod, ctx->mods, B, d, st));
+    {
+        const int pi = prof_begin(ctx, XC_K_COND, -1);
+        CK(timestep_embedding(sigma, ctx->temb, ctx->cfg.t_freq_dim, st));
+        CK(gemv(ctx->temb, 0, ctx->t_w1, ctx->t_b1, nullptr, ctx->ht, ctx->cfg.t_freq_dim, d, 1, st));
+        CK(gemv(ctx->act_dev, 0, ctx->a_w1, ctx->a_b1, nullptr, ctx->ha, ctx->A, d, 1, st));
+        CK(gemv(ctx->ht, 0, ctx->t_w2, ctx->t_b2, nullptr, ctx->e1, d, d, 0, st));
+        CK(gemv(ctx->ha, 0, ctx->a_w2, ctx->a_b2, ctx->e1, ctx->e, d, d, 0, st));
+        CK(gemv(ctx->e, 1, ctx->mod_w, ctx->mod_b, nullptr, ctx->mshared, d, 6 * d, 0, st));
+        CK(gemv(ctx->e, 1, ctx->head_w, ctx->head_b, ctx->head_tab, ctx->hmod, d, 2 * d, 0, st));
+        CK(assemble_mods(ctx->mshared, ctx->blk_mod, ctx->mods, B, d, st));
+        prof_end(ctx, pi);
+        ctx->launches += 8;
+    }
 
     T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
-    CK(patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
+    LAUNCH(XC_K_EMBED, -1, 1, patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
     CK(cudaMemsetAsync(ctx->flags, 0, B, st));
     CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
 
@@ -364,11 +407,11 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.gl_part = ctx->g_gl;
             g.cnt_cs = ctx->g_cnt;
             g.cnt_all = ctx->g_cnt + ctx->V * ctx->g_ns;
-            CK(gate_launch<T>(g, st));
+            LAUNCH(XC_K_GATE, b, 1, gate_launch<T>(g, st));
         }
 
         // ---- recompute path (early-exits when flag[b] == skip)
-        CK(ln_mod<T>(xin, mb + 0 * d, mb + 1 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
+        LAUNCH(XC_K_LN, b, 1, ln_mod<T>(xin, mb + 0 * d, mb + 1 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
         EpiParams ep;
         memset(&ep, 0, sizeof ep);
         ep.M = L;
@@ -387,15 +430,15 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.rope_freq = ctx->rope_freq;
         ep.rope_axis = ctx->rope_axis;
         if constexpr (sizeof(T) == 2) {
-            CK(gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
-            CK(attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L, n_keys,
-                       ctx->H, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_ATTN, b, 1, attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L,
+                                            n_keys, ctx->H, d, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->qkv_wt) + (size_t)b * 3 * d * d;
-            CK(gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+            LAUNCH(XC_K_QKV, b, 1, gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
             const float *Kr = reinterpret_cast<const float *>(ctx->ring_k) + (size_t)b * ctx->Wkv * Ld;
             const float *Vr = reinterpret_cast<const float *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld;
-            CK(attn_simt(hd, reinterpret_cast<const float *>(qb), Kr, Vr, reinterpret_cast<float *>(ob), L, n_keys,
+            LAUNCH(XC_K_ATTN, b, 1, attn_simt(hd, reinterpret_cast<const float *>(qb), Kr, Vr, reinterpret_cast<float *>(ob), L, n_keys,
                          ctx->H, flag, st));
         }
         // O projection + gated residual: x1 = x + gate1 * (o W_o + b_o)
@@ -407,12 +450,12 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.resid = xin;
         ep.out = x1;
         if constexpr (sizeof(T) == 2) {
-            CK(gemm_tc(EPI_RESID_GATE, ctx->tm_o, ctx->tm_wo[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_OPROJ, b, 1, gemm_tc(EPI_RESID_GATE, ctx->tm_o, ctx->tm_wo[b], ep, d, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->o_wt) + (size_t)b * d * d;
-            CK(gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
+            LAUNCH(XC_K_OPROJ, b, 1, gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
         }
-        CK(ln_mod<T>(x1, mb + 3 * d, mb + 4 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
+        LAUNCH(XC_K_LN, b, 1, ln_mod<T>(x1, mb + 3 * d, mb + 4 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
         // FFN up: u = GELU_tanh(h2 W1 + b1)
         memset(&ep, 0, sizeof ep);
         ep.M = L;
@@ -420,10 +463,10 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.bias = ctx->f1_b + (size_t)b * F;
         ep.out = ub;
         if constexpr (sizeof(T) == 2) {
-            CK(gemm_tc(EPI_GELU, ctx->tm_h, ctx->tm_w1[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_FFN1, b, 1, gemm_tc(EPI_GELU, ctx->tm_h, ctx->tm_w1[b], ep, d, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->f1_wt) + (size_t)b * F * d;
-            CK(gemm_simt(EPI_GELU, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+            LAUNCH(XC_K_FFN1, b, 1, gemm_simt(EPI_GELU, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
         }
         // FFN down + gated residual; residual cache write r_hat = x2 - x (Eq. 2-3)
         memset(&ep, 0, sizeof ep);
@@ -436,18 +479,23 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.out = xout;
         ep.rhat = rh;
         if constexpr (sizeof(T) == 2) {
-            CK(gemm_tc(EPI_RESID_CACHE, ctx->tm_u, ctx->tm_w2[b], ep, F, flag, ctx->d_err, st));
+            LAUNCH(XC_K_FFN2, b, 1, gemm_tc(EPI_RESID_CACHE, ctx->tm_u, ctx->tm_w2[b], ep, F, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->f2_wt) + (size_t)b * d * F;
-            CK(gemm_simt(EPI_RESID_CACHE, ep, reinterpret_cast<const float *>(ub), W, F, flag, st));
+            LAUNCH(XC_K_FFN2, b, 1, gemm_simt(EPI_RESID_CACHE, ep, reinterpret_cast<const float *>(ub), W, F, flag, st));
         }
         // ---- reuse path (Eq. 4), only when the gate chose skip
-        if (gated) CK(residual_reuse<T>(xin, rh, xout, (long)Ld, flag, ctx->n_sm, st));
+        if (gated) LAUNCH(XC_K_REUSE, b, 1, residual_reuse<T>(xin, rh, xout, (long)Ld, flag, ctx->n_sm, st));
         if (ctx->trace != nullptr)
             CK(cudaMemcpyAsync(reinterpret_cast<char *>(ctx->trace) + (size_t)b * Ld * sizeof(T), xout,
                                Ld * sizeof(T), cudaMemcpyDeviceToDevice, st));
     }
-    CK(head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
+    LAUNCH(XC_K_HEAD, -1, 1, head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
+    if (ctx->prof_on) {
+        if (ctx->pass_seq < ctx->prof_cap)
+            CK(cudaMemcpyAsync(ctx->dec_log + (size_t)ctx->pass_seq * B, ctx->flags, B, cudaMemcpyDeviceToDevice, st));
+        ctx->pass_seq += 1;
+    }
 }
 
 }  // namespace
@@ -481,9 +529,12 @@ const char *xc_last_error(const xc_ctx *ctx) {
     return g_global_err.c_str();
 }
 
+static void prof_free(xc_ctx *ctx);
+
 void xc_destroy(xc_ctx *ctx) {
     if (ctx == nullptr) return;
     cudaStreamSynchronize(ctx->st);
+    prof_free(ctx);
     for (void *p : ctx->allocs) cudaFree(p);
     if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
     if (ctx->h_stats) cudaFreeHost(ctx->h_stats);
@@ -696,6 +747,76 @@ xc_status xc_reset(xc_ctx *ctx) {
 
 int xc_chunk_index(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->n; }
 
+long long xc_launch_count(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->launches; }
+
+static void prof_free(xc_ctx *ctx) {
+    for (cudaEvent_t e : ctx->prof_ev) cudaEventDestroy(e);
+    ctx->prof_ev.clear();
+    ctx->prof_rec.clear();
+    if (ctx->dec_log != nullptr) cudaFree(ctx->dec_log);
+    ctx->dec_log = nullptr;
+    ctx->prof_on = false;
+    ctx->prof_cap = ctx->prof_n = 0;
+}
+
+xc_status xc_profile_start(xc_ctx *ctx, unsigned kind_mask, int capacity) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_profile_start: NULL context");
+        return XC_ESTATE;
+    }
+    if (capacity < 1) {
+        set_err(ctx, "xc_profile_start: capacity < 1");
+        return XC_EINVAL;
+    }
+    try {
+        CK(cudaStreamSynchronize(ctx->st));
+        prof_free(ctx);
+        ctx->prof_ev.resize(2 * (size_t)capacity);
+        for (auto &e : ctx->prof_ev) CK(cudaEventCreate(&e));
+        ctx->prof_rec.resize(capacity);
+        CK(cudaMalloc(&ctx->dec_log, (size_t)capacity * ctx->B));
+        ctx->prof_cap = capacity;
+        ctx->prof_n = 0;
+        ctx->pass_seq = 0;
+        ctx->prof_mask = kind_mask;
+        ctx->prof_on = true;
+    } catch (Fail &f) {
+        prof_free(ctx);
+        return f.st;
+    }
+    return XC_OK;
+}
+
+xc_status xc_profile_stop(xc_ctx *ctx, xc_profile_rec *out, int max, int *n_out) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_profile_stop: NULL context");
+        return XC_ESTATE;
+    }
+    if (!ctx->prof_on) {
+        set_err(ctx, "xc_profile_stop: profiling not started");
+        return XC_ESTATE;
+    }
+    xc_status status = XC_OK;
+    try {
+        CK(cudaStreamSynchronize(ctx->st));
+        const int passes = ctx->pass_seq < ctx->prof_cap ? ctx->pass_seq : ctx->prof_cap;
+        std::vector<uint8_t> dec((size_t)passes * ctx->B + 1);
+        if (passes > 0) CK(cudaMemcpy(dec.data(), ctx->dec_log, (size_t)passes * ctx->B, cudaMemcpyDeviceToHost));
+        const int n = ctx->prof_n < max ? ctx->prof_n : max;
+        for (int i = 0; i < n; ++i) {
+            xc_profile_rec r = ctx->prof_rec[i];
+            CK(cudaEventElapsedTime(&r.ms, ctx->prof_ev[2 * i], ctx->prof_ev[2 * i + 1]));
+            if (r.block >= 0 && r.pass_seq < passes) r.decision = dec[(size_t)r.pass_seq * ctx->B + r.block];
+            if (out != nullptr) out[i] = r;
+        }
+        if (n_out != nullptr) *n_out = ctx->prof_n;
+    } catch (Fail &f) {
+        status = f.st;
+    }
+    prof_free(ctx);
+    return status;
+}
+
 xc_status xc_set_block_trace(xc_ctx *ctx, void *dev_buf) {
     if (ctx == nullptr) {
         set_err(nullptr, "xc_set_block_trace: NULL context");
@@ -737,6 +858,7 @@ xc_status xc_euler_update(xc_ctx *ctx, float *x, const float *v, float dsigma, l
     if (n == 0) return XC_OK;
     try {
         CK(euler_update(x, v, dsigma, n, ctx->st));
+        ctx->launches += 1;
     } catch (Fail &f) {
         return f.st;
     }
@@ -798,6 +920,9 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
         else
             run_pass<float>(ctx, lat_dev, action, sigma, t, kv, p, v_dev);
         if (v_host) CK(cudaMemcpyAsync(v_out, ctx->vout, lat_bytes, cudaMemcpyDeviceToHost, ctx->st));
+        // Host buffers are consumed / produced synchronously: the caller may
+        // reuse them as soon as the call returns.
+        if (v_host || lat_dev != latent) CK(cudaStreamSynchronize(ctx->st));
         if (stats != nullptr) {
             CK(cudaMemcpyAsync(ctx->h_flags, ctx->flags, ctx->B, cudaMemcpyDeviceToHost, ctx->st));
             CK(cudaMemcpyAsync(ctx->h_stats, ctx->s_cos, 3 * ctx->B * sizeof(float), cudaMemcpyDeviceToHost,

@@ -64,6 +64,14 @@ class StepStats(ctypes.Structure):
                 ("tau_cos", ctypes.c_float * XC_MAX_BLOCKS)]
 
 
+class ProfileRec(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("block", ctypes.c_int), ("pass_seq", ctypes.c_int),
+                ("decision", ctypes.c_int), ("chunk", ctypes.c_int), ("n_keys", ctypes.c_int),
+                ("ms", ctypes.c_float)]
+
+
+KERNEL_KINDS = ("cond", "embed", "gate", "ln", "qkv", "attn", "oproj", "ffn1", "ffn2", "reuse", "head")
+
 _P = ctypes.c_void_p
 _I = ctypes.c_int
 _F = ctypes.c_float
@@ -80,6 +88,9 @@ SIGNATURES = {
     "xc_set_block_trace": (_I, [_P, _P]),
     "xc_sync": (_I, [_P]),
     "xc_chunk_index": (_I, [_P]),
+    "xc_launch_count": (ctypes.c_longlong, [_P]),
+    "xc_profile_start": (_I, [_P, ctypes.c_uint, _I]),
+    "xc_profile_stop": (_I, [_P, ctypes.POINTER(ProfileRec), _I, ctypes.POINTER(_I)]),
     "xc_op_linear": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
     "xc_op_qkv_rope": (_I, [_I, _I, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P]),
     "xc_op_attention": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
@@ -213,6 +224,27 @@ class XCache:
     @property
     def chunk_index(self) -> int:
         return LIB.xc_chunk_index(self.ctx)
+
+    @property
+    def launch_count(self) -> int:
+        return LIB.xc_launch_count(self.ctx)
+
+    def profile_start(self, kinds=KERNEL_KINDS, capacity: int = 65536):
+        mask = 0
+        for k in kinds:
+            mask |= 1 << KERNEL_KINDS.index(k)
+        self._prof_cap = capacity
+        check(LIB.xc_profile_start(self.ctx, mask, capacity), self.ctx)
+
+    def profile_stop(self) -> list:
+        """Synchronises; returns dicts (kind, block, pass_seq, decision, chunk, n_keys, ms)."""
+        cap = getattr(self, "_prof_cap", 65536)
+        recs = (ProfileRec * cap)()
+        n = ctypes.c_int()
+        check(LIB.xc_profile_stop(self.ctx, recs, cap, ctypes.byref(n)), self.ctx)
+        return [dict(kind=KERNEL_KINDS[r.kind], block=r.block, pass_seq=r.pass_seq,
+                     decision=r.decision, chunk=r.chunk, n_keys=r.n_keys, ms=r.ms)
+                for r in recs[:min(n.value, cap)]]
 
 
 # --------------------------------------------------------------- operators
