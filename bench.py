@@ -340,7 +340,7 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
         x_np[:] = traj.noise(n)
         for t in range(S):
             xc.chunk_step(x_np, acts[n], SIGMAS[t], t, False, gate, v_out=v_np, want_stats=False)
-            x_np += np.float32(SIGMAS[t + 1] - SIGMAS[t]) * v_np
+            np.add(x_np, np.float32(SIGMAS[t + 1] - SIGMAS[t]) * v_np, out=x_np)
         c_np[:] = traj.clean(n)
         xc.chunk_step(c_np, acts[n], 0.0, S, True, gate, want_stats=False)
 

@@ -4,40 +4,42 @@
 //   the current chunk's queries see every resident key of the rolling KV
 //   cache (past chunks' clean K/V plus the current chunk's own K/V).
 //
-// One CTA = one 128-query tile of one head.  Warp roles (192 threads):
-//   warps 0..3 : softmax; thread r owns query row r = TMEM lane r.  Reads the
-//                score row S (fp32, TMEM), online max / sum in the exp2 domain,
-//                writes P (bf16, 128B-swizzled, K-major) to shared memory and
-//                rescales its O row in TMEM when the running max grows;
-//   warp 4     : TMA producer (Q once; K and V tiles of 128 keys, STAGES deep);
-//   warp 5     : TMEM allocation; lane 0 issues S = Q K^T (M=128, N=128) into
-//                one of two TMEM score buffers and O += P V (M=128, N=hd, V
-//                read MN-major straight from its [keys][hd] tile).
-// TMEM columns: S0 [0,128), S1 [128,256), O [256, 256+hd).
-// S_{j+1} is computed while the softmax warps work on S_j; P V_j overlaps the
-// score read of S_{j+1}.  Keys beyond n_keys are masked to -inf (their K/V
-// rows are finite: the ring is zero-initialised and TMA zero-fills past the
-// end of the tensor).
+// One CTA = two 128-query tiles (Q0, Q1) of one head, 320 threads:
+//   warps 0..3  softmax WG 0 (tile Q0), thread = query row = TMEM lane;
+//   warps 4..7  softmax WG 1 (tile Q1);
+//   warp 8      TMA producer: Q0/Q1 once, then 128-key K and V tiles through
+//               a STAGES-deep ring (separate K and V barriers);
+//   warp 9      TMEM allocation; lane 0 issues every MMA.
+// TMEM (512 columns): S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after.
+// The two tiles ping-pong on the tensor core: while WG 0 turns S0 into
+// probabilities, the MMA warp runs P1 V and the next S1, and vice versa.
+// P (bf16) is written back into TMEM over its own S buffer and consumed by
+// tcgen05.mma with the A operand in tensor memory (no shared-memory round
+// trip); V is read MN-major straight from its [keys][hd] tile.
+// Online softmax in the exp2 domain with lazy rescaling: a row's O and sum
+// are rescaled only when its running max grows by more than 8 (2^8 headroom
+// in fp32 / bf16), so after the first tiles the correction almost never runs.
+// Keys beyond n_keys (ragged last tile) are masked to -inf; their K/V rows are
+// finite (zero-initialised ring, TMA zero fill past the tensor end).
 #include "xc_ptx.cuh"
 
 namespace xc {
 
 template <int HD>
 struct AttnTile {
-    static constexpr int BQ = 128, BKV = 128;
+    static constexpr int BQ = 128, BKV = 128, QT = 2;
     static constexpr int NR = HD / 64;                 // 64-wide swizzle regions per row
-    static constexpr int REGION = 128 * 128;           // [128 rows][64 bf16] bytes
-    static constexpr int Q_BYTES = NR * REGION;
-    static constexpr int KV_BYTES = NR * REGION;
-    static constexpr int STAGES = HD == 64 ? 3 : 2;
-    static constexpr int P_BYTES = 2 * REGION;
-    static constexpr int OFF_K = Q_BYTES;
+    static constexpr int REGION = 128 * 128;           // [128 rows][64 bf16]
+    static constexpr int Q_BYTES = NR * REGION;        // one 128-row Q tile
+    static constexpr int KV_BYTES = NR * REGION;       // one 128-key K or V tile
+    static constexpr int STAGES = HD == 64 ? 4 : 2;
+    static constexpr int OFF_K = QT * Q_BYTES;
     static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
-    static constexpr int OFF_P = OFF_V + STAGES * KV_BYTES;
-    static constexpr int OFF_BAR = OFF_P + P_BYTES;
+    static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
     static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
     static constexpr int TMEM_COLS = 512;
-    static constexpr int O_COL = 256;
+    static constexpr int THREADS = 320;
+    static constexpr float LAZY = 8.0f;                // rescale threshold (log2 units)
 };
 
 __device__ __forceinline__ uint8_t *align1024_a(uint8_t *p) {
@@ -45,8 +47,14 @@ __device__ __forceinline__ uint8_t *align1024_a(uint8_t *p) {
     return p + ((1024u - (s & 1023u)) & 1023u);
 }
 
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 template <int HD>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
                    const int n_keys, const int d, const uint8_t *__restrict__ skip_flag, int *err) {
@@ -57,177 +65,218 @@ __global__ void __launch_bounds__(192, 1)
     uint8_t *sQ = smem;
     uint8_t *sK = smem + A::OFF_K;
     uint8_t *sV = smem + A::OFF_V;
-    uint8_t *sP = smem + A::OFF_P;
     uint64_t *bar = reinterpret_cast<uint64_t *>(smem + A::OFF_BAR);
     uint64_t *q_full = bar;
-    uint64_t *kv_full = bar + 1;
-    uint64_t *kv_empty = kv_full + A::STAGES;
-    uint64_t *s_full = kv_empty + A::STAGES;   // [2]
-    uint64_t *s_free = s_full + 2;             // [2]
-    uint64_t *p_full = s_free + 2;
-    uint64_t *pv_done = p_full + 1;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(pv_done + 1);
+    uint64_t *k_full = bar + 1;
+    uint64_t *k_empty = k_full + A::STAGES;
+    uint64_t *v_full = k_empty + A::STAGES;
+    uint64_t *v_empty = v_full + A::STAGES;
+    uint64_t *s_full = v_empty + A::STAGES;    // [2] per tile
+    uint64_t *p_full = s_full + 2;             // [2]
+    uint64_t *o_done = p_full + 2;             // [2]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(o_done + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int q0 = blockIdx.x * A::BQ;
+    const int q0 = blockIdx.x * (A::QT * A::BQ);
     const int h = blockIdx.y;
     const int nkt = (n_keys + A::BKV - 1) / A::BKV;
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
         for (int s = 0; s < A::STAGES; ++s) {
-            mbar_init(&kv_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 128);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&p_full[i], 128);
+            mbar_init(&o_done[i], 1);
         }
-        mbar_init(p_full, 128);
-        mbar_init(pv_done, 1);
         mbar_fence_init();
     }
-    if (warp == 5) tmem_alloc(tmem_slot, A::TMEM_COLS);
+    if (warp == 9) tmem_alloc(tmem_slot, A::TMEM_COLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 4) {
+    if (warp == 8) {
+        // ------------------------------------------------------ TMA producer
         if (lane == 0) {
-            mbar_expect_tx(q_full, A::Q_BYTES);
-            for (int r = 0; r < A::NR; ++r) tma_load_2d(sQ + r * A::REGION, &tmQ, q_full, h * HD + 64 * r, q0);
-            int issued = 0;
+            mbar_expect_tx(q_full, A::QT * A::Q_BYTES);
+            for (int i = 0; i < A::QT; ++i)
+                for (int r = 0; r < A::NR; ++r)
+                    tma_load_2d(sQ + i * A::Q_BYTES + r * A::REGION, &tmQ, q_full, h * HD + 64 * r, q0 + i * A::BQ);
+            int k_issued = 0, v_issued = 0;
             for (int j = 0; j < nkt; ++j) {
                 const int st = j % A::STAGES;
-                if (!mbar_wait(&kv_empty[st], ((j / A::STAGES) & 1) ^ 1, err, ERR_WAIT_PRODUCER)) break;
-                mbar_expect_tx(&kv_full[st], 2 * A::KV_BYTES);
-                for (int r = 0; r < A::NR; ++r) {
-                    tma_load_2d(sK + st * A::KV_BYTES + r * A::REGION, &tmK, &kv_full[st], h * HD + 64 * r,
+                const uint32_t ph = ((j / A::STAGES) & 1) ^ 1;
+                if (!mbar_wait(&k_empty[st], ph, err, ERR_WAIT_PRODUCER)) break;
+                mbar_expect_tx(&k_full[st], A::KV_BYTES);
+                for (int r = 0; r < A::NR; ++r)
+                    tma_load_2d(sK + st * A::KV_BYTES + r * A::REGION, &tmK, &k_full[st], h * HD + 64 * r,
                                 j * A::BKV);
-                    tma_load_2d(sV + st * A::KV_BYTES + r * A::REGION, &tmV, &kv_full[st], h * HD + 64 * r,
+                k_issued = j + 1;
+                if (!mbar_wait(&v_empty[st], ph, err, ERR_WAIT_PRODUCER)) break;
+                mbar_expect_tx(&v_full[st], A::KV_BYTES);
+                for (int r = 0; r < A::NR; ++r)
+                    tma_load_2d(sV + st * A::KV_BYTES + r * A::REGION, &tmV, &v_full[st], h * HD + 64 * r,
                                 j * A::BKV);
-                }
-                issued = j + 1;
+                v_issued = j + 1;
             }
+            // Drain: every copy this thread started has landed before exit.
             mbar_wait(q_full, 0, err, ERR_WAIT_PRODUCER);
-            for (int j = issued - A::STAGES < 0 ? 0 : issued - A::STAGES; j < issued; ++j)
-                mbar_wait(&kv_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+            for (int j = k_issued - A::STAGES < 0 ? 0 : k_issued - A::STAGES; j < k_issued; ++j)
+                mbar_wait(&k_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+            for (int j = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; j < v_issued; ++j)
+                mbar_wait(&v_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
-    } else if (warp == 5) {
+    } else if (warp == 9) {
+        // ---------------------------------------------------------- MMA issue
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);
             constexpr uint32_t idesc_o = idesc_bf16(128, HD, false, true);
-            bool ok = mbar_wait(q_full, 0, err, ERR_WAIT_MMA);
-            const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV), aP = smem_u32(sP);
-            for (int j = 0; ok && j <= nkt; ++j) {
-                if (j < nkt) {
-                    const int st = j % A::STAGES;
-                    const int sb = j & 1;
-                    if (!mbar_wait(&kv_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                    if (j >= 2 && !mbar_wait(&s_free[sb], ((j - 2) >> 1) & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
+            const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV);
+            auto issue_s = [&](int i, int j) {        // S_i = Q_i K_j^T
+                const int st = j % A::STAGES;
 #pragma unroll
-                    for (int ks = 0; ks < HD / 16; ++ks) {
-                        const uint32_t off = (ks >> 2) * A::REGION + (ks & 3) * 32;
-                        tc_mma(tmem + sb * 128, sdesc_sw128(aQ + off, 16, 1024),
-                               sdesc_sw128(aK + st * A::KV_BYTES + off, 16, 1024), idesc_s, ks > 0 ? 1u : 0u);
-                    }
-                    tc_commit(&s_full[sb]);
+                for (int ks = 0; ks < HD / 16; ++ks) {
+                    const uint32_t off = (ks >> 2) * A::REGION + (ks & 3) * 32;
+                    tc_mma(tmem + 128 * i, sdesc_sw128(aQ + i * A::Q_BYTES + off, 16, 1024),
+                           sdesc_sw128(aK + st * A::KV_BYTES + off, 16, 1024), idesc_s, ks > 0 ? 1u : 0u);
                 }
-                if (j >= 1) {
-                    const int jj = j - 1;
-                    const int st = jj % A::STAGES;
-                    if (!mbar_wait(p_full, jj & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
+                tc_commit(&s_full[i]);
+            };
+            auto issue_pv = [&](int i, int j) {       // O_i += P_i V_j, P_i in TMEM over S_i
+                const int st = j % A::STAGES;
 #pragma unroll
-                    for (int ks = 0; ks < A::BKV / 16; ++ks) {
-                        const uint32_t pa = aP + (ks >> 2) * A::REGION + (ks & 3) * 32;
-                        const uint32_t vb = aV + st * A::KV_BYTES + ks * 16 * 128;
-                        tc_mma(tmem + A::O_COL, sdesc_sw128(pa, 16, 1024), sdesc_sw128(vb, A::REGION, 1024),
-                               idesc_o, (jj > 0 || ks > 0) ? 1u : 0u);
-                    }
-                    tc_commit(pv_done);
-                    tc_commit(&kv_empty[st]);
+                for (int ks = 0; ks < A::BKV / 16; ++ks)
+                    tc_mma_tmem_a(tmem + 256 + HD * i, tmem + 128 * i + 8 * ks,
+                                  sdesc_sw128(aV + st * A::KV_BYTES + ks * 16 * 128, A::REGION, 1024), idesc_o,
+                                  (j > 0 || ks > 0) ? 1u : 0u);
+            };
+            bool ok = mbar_wait(q_full, 0, err, ERR_WAIT_MMA) && mbar_wait(&k_full[0], 0, err, ERR_WAIT_MMA);
+            if (ok) {
+                tc_fence_after();
+                issue_s(0, 0);
+                issue_s(1, 0);
+                tc_commit(&k_empty[0]);
+            }
+            for (int j = 0; ok && j < nkt; ++j) {
+                const int st = j % A::STAGES;
+                const int st1 = (j + 1) % A::STAGES;
+                const bool more = j + 1 < nkt;
+                if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
+                tc_fence_after();
+                issue_pv(0, j);
+                if (!more) tc_commit(&o_done[0]);
+                if (more) {
+                    if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                    tc_fence_after();
+                    issue_s(0, j + 1);
+                }
+                if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
+                tc_fence_after();
+                issue_pv(1, j);
+                tc_commit(&v_empty[st]);
+                if (!more) tc_commit(&o_done[1]);
+                if (more) {
+                    issue_s(1, j + 1);
+                    tc_commit(&k_empty[st1]);
                 }
             }
         }
     } else {
-        // ---------------------------------------------------------- softmax
-        const int r = warp * 32 + lane;
-        const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+        // ------------------------------------------------------------ softmax
+        const int wg = warp >> 2;                          // tile of this warpgroup
+        const int q = warp & 3;                            // TMEM lane quadrant
+        const int row = q0 + wg * A::BQ + q * 32 + lane;
+        const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
+        const uint32_t tS = tl + 128 * wg;
+        const uint32_t tO = tl + 256 + HD * wg;
         const float sl2 = rsqrtf((float)HD) * 1.4426950408889634f;
+        const int tail = n_keys - (nkt - 1) * A::BKV;      // valid keys in the last tile
         float m = -INFINITY, l = 0.0f;
         bool ok = true;
-        for (int j = 0; j < nkt && ok; ++j) {
-            const int sb = j & 1;
-            ok = mbar_wait(&s_full[sb], (j >> 1) & 1, err, ERR_WAIT_SOFTMAX);
+        for (int j = 0; j < nkt; ++j) {
+            ok = mbar_wait(&s_full[wg], j & 1, err, ERR_WAIT_SOFTMAX);
             __syncwarp();
             if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             tc_fence_after();
             float s[128];
-            tmem_ld128_sync(tl + sb * 128, s);
-            tc_fence_before();
-            mbar_arrive(&s_free[sb]);
-            const int kbase = j * A::BKV;
-            float mx = -INFINITY;
+            tmem_ld128_sync(tS, s);
+            if (j == nkt - 1 && tail < A::BKV) {
 #pragma unroll
-            for (int c = 0; c < 128; ++c) {
-                if (kbase + c >= n_keys) s[c] = -INFINITY;
-                mx = fmaxf(mx, s[c]);
+                for (int c = 0; c < 128; ++c)
+                    if (c >= tail) s[c] = -INFINITY;
             }
-            const float m_new = fmaxf(m, mx * sl2);
-            if (j >= 1) {
-                ok = mbar_wait(pv_done, (j - 1) & 1, err, ERR_WAIT_SOFTMAX);
-                __syncwarp();
-                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-                tc_fence_after();
-                if (__any_sync(0xffffffffu, m_new > m)) {
-                    const float alpha = exp2f(m - m_new);
+            float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+#pragma unroll
+            for (int c = 4; c < 128; c += 4) {
+                mx0 = fmaxf(mx0, s[c]);
+                mx1 = fmaxf(mx1, s[c + 1]);
+                mx2 = fmaxf(mx2, s[c + 2]);
+                mx3 = fmaxf(mx3, s[c + 3]);
+            }
+            const float m_new = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+            if (j == 0) {
+                m = m_new;
+            } else {
+                const bool grow = m_new > m + A::LAZY;
+                if (__any_sync(0xffffffffu, grow)) {
+                    // O_i is stable: the commit behind s_full covers P V of tile j-1.
+                    const float alpha = grow ? ex2_approx(m - m_new) : 1.0f;
 #pragma unroll 1
                     for (int c = 0; c < HD / 16; ++c) {
                         float t[16];
-                        tmem_ld16_sync(tl + A::O_COL + 16 * c, t);
+                        tmem_ld16_sync(tO + 16 * c, t);
 #pragma unroll
                         for (int i = 0; i < 16; ++i) t[i] *= alpha;
-                        tmem_st16_sync(tl + A::O_COL + 16 * c, t);
+                        tmem_st16_sync(tO + 16 * c, t);
                     }
                     l *= alpha;
+                    if (grow) m = m_new;
                 }
             }
-            m = m_new;
-            float rs = 0.0f;
-            uint8_t *prow = sP + r * 128;
+            const float nm = -m;
+            float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
 #pragma unroll
-            for (int c16 = 0; c16 < 16; ++c16) {
-                uint32_t w[4];
+            for (int half = 0; half < 2; ++half) {
+                uint32_t w[32];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float p0 = exp2f(fmaf(s[8 * c16 + 2 * i], sl2, -m));
-                    const float p1 = exp2f(fmaf(s[8 * c16 + 2 * i + 1], sl2, -m));
-                    rs += p0 + p1;
-                    __nv_bfloat162 hh = __floats2bfloat162_rn(p0, p1);
-                    w[i] = *reinterpret_cast<uint32_t *>(&hh);
+                for (int i = 0; i < 32; i += 2) {
+                    const int c = 64 * half + 2 * i;
+                    const float p0 = ex2_approx(fmaf(s[c], sl2, nm));
+                    const float p1 = ex2_approx(fmaf(s[c + 1], sl2, nm));
+                    const float p2 = ex2_approx(fmaf(s[c + 2], sl2, nm));
+                    const float p3 = ex2_approx(fmaf(s[c + 3], sl2, nm));
+                    r0 += p0;
+                    r1 += p1;
+                    r2 += p2;
+                    r3 += p3;
+                    __nv_bfloat162 h0 = __floats2bfloat162_rn(p0, p1);
+                    __nv_bfloat162 h1 = __floats2bfloat162_rn(p2, p3);
+                    w[i] = *reinterpret_cast<uint32_t *>(&h0);
+                    w[i + 1] = *reinterpret_cast<uint32_t *>(&h1);
                 }
-                const int region = c16 >> 3, cc = c16 & 7;
-                *reinterpret_cast<uint4 *>(prow + region * A::REGION + ((cc ^ (r & 7)) << 4)) =
-                    make_uint4(w[0], w[1], w[2], w[3]);
+                tmem_st32_sync(tS + 32 * half, w);
             }
-            l += rs;
-            fence_proxy_async_smem();
+            l += (r0 + r1) + (r2 + r3);
             tc_fence_before();
-            mbar_arrive(p_full);
+            mbar_arrive(&p_full[wg]);
         }
-        if (ok) ok = mbar_wait(pv_done, (nkt - 1) & 1, err, ERR_WAIT_SOFTMAX);
+        if (ok) ok = mbar_wait(&o_done[wg], 0, err, ERR_WAIT_SOFTMAX);
         __syncwarp();
         if (__all_sync(0xffffffffu, ok)) {
             tc_fence_after();
             const float inv = 1.0f / l;
-            const int row = q0 + r;
 #pragma unroll 1
             for (int c = 0; c < HD / 16; ++c) {
                 float t[16];
-                tmem_ld16_sync(tl + A::O_COL + 16 * c, t);
+                tmem_ld16_sync(tO + 16 * c, t);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) t[i] *= inv;
                 if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
@@ -236,7 +285,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == 9) {
         tc_fence_after();
         tmem_dealloc(tmem, A::TMEM_COLS);
     }
@@ -256,8 +305,8 @@ static cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, con
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    dim3 grid((Lq + A::BQ - 1) / A::BQ, n_heads);
-    attn_tc_kernel<HD><<<grid, 192, A::SMEM_BYTES, st>>>(tq, tk, tv, o, Lq, n_keys, d, skip, err);
+    dim3 grid((Lq + A::QT * A::BQ - 1) / (A::QT * A::BQ), n_heads);
+    attn_tc_kernel<HD><<<grid, A::THREADS, A::SMEM_BYTES, st>>>(tq, tk, tv, o, Lq, n_keys, d, skip, err);
     return cudaGetLastError();
 }
 

@@ -6,53 +6,56 @@
 namespace xc {
 
 // ------------------------------------------------------------ patch embed
-// X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][C].
+// X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][16].
+// One thread per (row, 16-column run); float4 loads of z and pe_w (L1-resident).
 template <typename T>
-__global__ void patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w,
-                                   const float *__restrict__ b, T *__restrict__ out, int L, int C, int d) {
+__global__ void __launch_bounds__(256)
+    patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w, const float *__restrict__ b,
+                       T *__restrict__ out, int L, int d) {
     const int runs = d / 16;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= L * runs) return;
     const int row = idx / runs, col = (idx % runs) * 16;
+    float zr[16];
+    load16<float>(z + (size_t)row * 16, zr);
     float acc[16];
+    load16<float>(b + col, acc);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) acc[j] = b[col + j];
-    for (int k = 0; k < C; ++k) {
-        const float zv = z[(size_t)row * C + k];
+    for (int k = 0; k < 16; ++k) {
+        float wr[16];
+        load16<float>(w + (size_t)k * d + col, wr);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) acc[j] = fmaf(zv, w[(size_t)k * d + col + j], acc[j]);
+        for (int j = 0; j < 16; ++j) acc[j] = fmaf(zr[k], wr[j], acc[j]);
     }
     store16<T>(out + (size_t)row * d + col, acc);
 }
 
 template <typename T>
 cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st) {
+    if (C != 16) return cudaErrorInvalidValue;
     const int n = L * (d / 16);
-    patch_embed_kernel<T><<<(n + 255) / 256, 256, 0, st>>>(z, w, b, out, L, C, d);
+    patch_embed_kernel<T><<<(n + 255) / 256, 256, 0, st>>>(z, w, b, out, L, d);
     return cudaGetLastError();
 }
 template cudaError_t patch_embed<float>(const float *, const float *, const float *, float *, int, int, int, cudaStream_t);
 template cudaError_t patch_embed<bf16>(const float *, const float *, const float *, bf16 *, int, int, int, cudaStream_t);
 
 // ------------------------------------------------------------- row stats
-// Welford over a lane's elements, merged across the warp (Chan et al.).
+// A row is walked in 16-element runs; lane l owns runs l, l + 32, ...  Each
+// lane reduces its own values to (count, mean, M2) in registers, the warp
+// merges the lanes pairwise (Chan, Golub & LeVeque), so no per-element divide.
 struct Moments {
     float n, mean, m2;
 };
-__device__ __forceinline__ void welford_add(Moments &a, float x) {
-    a.n += 1.0f;
-    const float dlt = x - a.mean;
-    a.mean += dlt / a.n;
-    a.m2 += dlt * (x - a.mean);
-}
-__device__ __forceinline__ Moments welford_merge(Moments a, Moments b) {
+__device__ __forceinline__ Moments merge(Moments a, Moments b) {
     if (b.n == 0.0f) return a;
     if (a.n == 0.0f) return b;
     Moments r;
     r.n = a.n + b.n;
     const float dlt = b.mean - a.mean;
-    r.mean = a.mean + dlt * (b.n / r.n);
-    r.m2 = a.m2 + b.m2 + dlt * dlt * (a.n * b.n / r.n);
+    const float f = b.n / r.n;
+    r.mean = a.mean + dlt * f;
+    r.m2 = a.m2 + b.m2 + dlt * dlt * a.n * f;
     return r;
 }
 __device__ __forceinline__ Moments warp_moments(Moments a) {
@@ -62,49 +65,90 @@ __device__ __forceinline__ Moments warp_moments(Moments a) {
         b.n = __shfl_xor_sync(0xffffffffu, a.n, o);
         b.mean = __shfl_xor_sync(0xffffffffu, a.mean, o);
         b.m2 = __shfl_xor_sync(0xffffffffu, a.m2, o);
-        a = welford_merge(a, b);
+        a = merge(a, b);
     }
     return a;
 }
+// Moments of the first n_valid of the NCH runs a lane holds in registers.
+template <int NCH>
+__device__ __forceinline__ Moments lane_moments(const float (&v)[NCH][16], int n_valid) {
+    float s = 0.0f;
+#pragma unroll
+    for (int k = 0; k < NCH; ++k)
+        if (k < n_valid) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) s += v[k][i];
+        }
+    Moments m = {16.0f * n_valid, 0.0f, 0.0f};
+    if (n_valid == 0) return m;
+    m.mean = s / m.n;
+#pragma unroll
+    for (int k = 0; k < NCH; ++k)
+        if (k < n_valid) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const float t = v[k][i] - m.mean;
+                m.m2 = fmaf(t, t, m.m2);
+            }
+        }
+    return m;
+}
 
 // ----------------------------------------------------------------- ln_mod
-// One warp per row: h = round(LN(x) * (1 + scale) + shift).  d % 512 == 0 is
-// not required; rows are walked in 16-element runs (d % 16 == 0).
-template <typename T>
+// One warp per row, the row held in registers (d <= 512 * NCH):
+// h = round(LN(x) * (1 + scale) + shift).
+template <typename T, int NCH>
 __global__ void __launch_bounds__(256)
     ln_mod_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
                   T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
-    if (warp >= M) return;
-    const T *xr = x + (size_t)warp * d;
-    Moments mo = {0.0f, 0.0f, 0.0f};
-    for (int c = lane * 16; c < d; c += 32 * 16) {
-        float v[16];
-        load16<T>(xr + c, v);
+    if (row >= M) return;
+    const T *xr = x + (size_t)row * d;
+    const int runs = d / 16;
+    const int mine = runs > lane ? (runs - lane + 31) / 32 : 0;
+    float v[NCH][16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) welford_add(mo, v[i]);
-    }
-    mo = warp_moments(mo);
+    for (int k = 0; k < NCH; ++k)
+        if (k < mine) load16<T>(xr + 16 * (lane + 32 * k), v[k]);
+    const Moments mo = warp_moments(lane_moments<NCH>(v, mine));
     const float rstd = rsqrtf(mo.m2 / (float)d + eps);
-    T *orow = out + (size_t)warp * d;
-    for (int c = lane * 16; c < d; c += 32 * 16) {
-        float v[16];
-        load16<T>(xr + c, v);
+    T *orow = out + (size_t)row * d;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = (v[i] - mo.mean) * rstd * (1.0f + scale[c + i]) + shift[c + i];
-        store16<T>(orow + c, v);
+    for (int k = 0; k < NCH; ++k) {
+        if (k < mine) {
+            const int c = 16 * (lane + 32 * k);
+            float sc[16], sh[16];
+            load16<float>(scale + c, sc);
+            load16<float>(shift + c, sh);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[k][i] = (v[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i];
+            store16<T>(orow + c, v[k]);
+        }
     }
+}
+
+template <typename T, int NCH>
+static cudaError_t ln_mod_n(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
+                            const uint8_t *skip, cudaStream_t st) {
+    ln_mod_kernel<T, NCH><<<(M + 7) / 8, 256, 0, st>>>(x, shift, scale, out, M, d, eps, skip);
+    return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
                    const uint8_t *skip, cudaStream_t st) {
-    const int warps_per_block = 8;
-    ln_mod_kernel<T><<<(M + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, st>>>(
-        x, shift, scale, out, M, d, eps, skip);
-    return cudaGetLastError();
+    if (d % 16 != 0) return cudaErrorInvalidValue;
+    switch ((d + 511) / 512) {
+        case 1: return ln_mod_n<T, 1>(x, shift, scale, out, M, d, eps, skip, st);
+        case 2: return ln_mod_n<T, 2>(x, shift, scale, out, M, d, eps, skip, st);
+        case 3: return ln_mod_n<T, 3>(x, shift, scale, out, M, d, eps, skip, st);
+        case 4: return ln_mod_n<T, 4>(x, shift, scale, out, M, d, eps, skip, st);
+        case 5: case 6: case 7: case 8: return ln_mod_n<T, 8>(x, shift, scale, out, M, d, eps, skip, st);
+        case 9: case 10: case 11: case 12: return ln_mod_n<T, 12>(x, shift, scale, out, M, d, eps, skip, st);
+        default: return cudaErrorInvalidValue;
+    }
 }
 template cudaError_t ln_mod<float>(const float *, const float *, const float *, float *, int, int, float,
                                    const uint8_t *, cudaStream_t);
@@ -112,8 +156,8 @@ template cudaError_t ln_mod<bf16>(const bf16 *, const float *, const float *, bf
                                   const uint8_t *, cudaStream_t);
 
 // ------------------------------------------------------------ reuse (Eq. 4)
-// out = round(x + rhat), 16-byte vectors; runs only when the gate chose reuse
-// (need_flag = XC_DEC_SKIP) or unconditionally (skip_flag == nullptr).
+// out = round(x + rhat), 16-element vectors; runs only when the gate chose
+// reuse (skip_flag == XC_DEC_SKIP) or unconditionally (skip_flag == nullptr).
 template <typename T>
 __global__ void __launch_bounds__(256)
     reuse_kernel(const T *__restrict__ x, const T *__restrict__ r, T *__restrict__ out, long n16,
@@ -173,24 +217,36 @@ cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st) 
 
 // y[j] = act_out( sum_i in(i) W[i][j] + b[j] + add[j] ), W [n_in][n_out].
 // in_silu: in = SiLU(x) instead of x.  act_out 0: none, 1: SiLU.
-__global__ void gemv_kernel(const float *__restrict__ x, int in_silu, const float *__restrict__ W,
-                            const float *__restrict__ b, const float *__restrict__ add, float *__restrict__ y,
-                            int n_in, int n_out, int act_out) {
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= n_out) return;
+// CTA = 32 output columns x 8 warps; warp w sums rows i = w (mod 8) with
+// coalesced 128-byte row segments, then the warps reduce in shared memory.
+__global__ void __launch_bounds__(256)
+    gemv_kernel(const float *__restrict__ x, int in_silu, const float *__restrict__ W, const float *__restrict__ b,
+                const float *__restrict__ add, float *__restrict__ y, int n_in, int n_out, int act_out) {
+    __shared__ float part[8][33];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + lane;
     float acc = 0.0f;
-    for (int i = 0; i < n_in; ++i) {
-        const float xi = in_silu ? silu(x[i]) : x[i];
-        acc = fmaf(xi, W[(size_t)i * n_out + j], acc);
+    if (j < n_out) {
+        for (int i = warp; i < n_in; i += 8) {
+            const float xi = in_silu ? silu(x[i]) : x[i];
+            acc = fmaf(xi, W[(size_t)i * n_out + j], acc);
+        }
     }
-    acc += b[j];
-    if (add != nullptr) acc += add[j];
-    y[j] = act_out == 1 ? silu(acc) : acc;
+    part[warp][lane] = acc;
+    __syncthreads();
+    if (warp == 0 && j < n_out) {
+        float s = 0.0f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) s += part[w][lane];
+        s += b[j];
+        if (add != nullptr) s += add[j];
+        y[j] = act_out == 1 ? silu(s) : s;
+    }
 }
 
 cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
                  int n_out, int act_out, cudaStream_t st) {
-    gemv_kernel<<<(n_out + 127) / 128, 128, 0, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
+    gemv_kernel<<<(n_out + 31) / 32, 256, 0, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
     return cudaGetLastError();
 }
 
@@ -208,38 +264,45 @@ cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, i
 }
 
 // ------------------------------------------------------------------- head
-// One warp per row: hf = round(LN(x) (1 + scale) + shift); v = hf W_out + b_out
-// (C = 16 output channels, float32 out).
-template <typename T>
+// One warp per row, row in registers: hf = round(LN(x) (1 + scale) + shift);
+// v = hf W_out + b_out (16 output channels, float32 out).  Each lane forms the
+// 16 partial dot products of its runs (float4 reads of W_out), then the warp
+// reduces them.
+template <typename T, int NCH>
 __global__ void __launch_bounds__(256)
     head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
                 const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
-    const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
-    if (warp >= L) return;
-    const T *xr = x + (size_t)warp * d;
-    Moments mo = {0.0f, 0.0f, 0.0f};
-    for (int c = lane * 16; c < d; c += 512) {
-        float t[16];
-        load16<T>(xr + c, t);
+    if (row >= L) return;
+    const T *xr = x + (size_t)row * d;
+    const int runs = d / 16;
+    const int mine = runs > lane ? (runs - lane + 31) / 32 : 0;
+    float val[NCH][16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) welford_add(mo, t[i]);
-    }
-    mo = warp_moments(mo);
+    for (int k = 0; k < NCH; ++k)
+        if (k < mine) load16<T>(xr + 16 * (lane + 32 * k), val[k]);
+    const Moments mo = warp_moments(lane_moments<NCH>(val, mine));
     const float rstd = rsqrtf(mo.m2 / (float)d + eps);
     const float *shift = hm, *scale = hm + d;
     float acc[16];
 #pragma unroll
     for (int o = 0; o < 16; ++o) acc[o] = 0.0f;
-    for (int c = lane * 16; c < d; c += 512) {
-        float t[16];
-        load16<T>(xr + c, t);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const float hv = round_to<T>((t[i] - mo.mean) * rstd * (1.0f + scale[c + i]) + shift[c + i]);
-            const float *wr = w + (size_t)(c + i) * 16;
+    for (int k = 0; k < NCH; ++k) {
+        if (k < mine) {
+            const int c = 16 * (lane + 32 * k);
+            float sc[16], sh[16];
+            load16<float>(scale + c, sc);
+            load16<float>(shift + c, sh);
 #pragma unroll
-            for (int o = 0; o < 16; ++o) acc[o] = fmaf(hv, wr[o], acc[o]);
+            for (int i = 0; i < 16; ++i) {
+                const float hv = round_to<T>((val[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i]);
+                float wr[16];
+                load16<float>(w + (size_t)(c + i) * 16, wr);
+#pragma unroll
+                for (int o = 0; o < 16; ++o) acc[o] = fmaf(hv, wr[o], acc[o]);
+            }
         }
     }
 #pragma unroll
@@ -247,17 +310,36 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
         for (int s = 16; s > 0; s >>= 1) acc[o] += __shfl_xor_sync(0xffffffffu, acc[o], s);
     }
-    if (lane == 0) {
-#pragma unroll
-        for (int o = 0; o < 16; ++o) v[(size_t)warp * 16 + o] = acc[o] + b[o];
+    if (lane < 4) {
+        float4 r;
+        r.x = acc[4 * lane] + b[4 * lane];
+        r.y = acc[4 * lane + 1] + b[4 * lane + 1];
+        r.z = acc[4 * lane + 2] + b[4 * lane + 2];
+        r.w = acc[4 * lane + 3] + b[4 * lane + 3];
+        reinterpret_cast<float4 *>(v + (size_t)row * 16)[lane] = r;
     }
+}
+
+template <typename T, int NCH>
+static cudaError_t head_n(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d,
+                          float eps, cudaStream_t st) {
+    head_kernel<T, NCH><<<(L + 7) / 8, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
+    return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
                  cudaStream_t st) {
-    head_kernel<T><<<(L + 7) / 8, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
-    return cudaGetLastError();
+    if (d % 16 != 0) return cudaErrorInvalidValue;
+    switch ((d + 511) / 512) {
+        case 1: return head_n<T, 1>(x, hm, w, b, v, L, d, eps, st);
+        case 2: return head_n<T, 2>(x, hm, w, b, v, L, d, eps, st);
+        case 3: return head_n<T, 3>(x, hm, w, b, v, L, d, eps, st);
+        case 4: return head_n<T, 4>(x, hm, w, b, v, L, d, eps, st);
+        case 5: case 6: case 7: case 8: return head_n<T, 8>(x, hm, w, b, v, L, d, eps, st);
+        case 9: case 10: case 11: case 12: return head_n<T, 12>(x, hm, w, b, v, L, d, eps, st);
+        default: return cudaErrorInvalidValue;
+    }
 }
 template cudaError_t head<float>(const float *, const float *, const float *, const float *, float *, int, int, float,
                                  cudaStream_t);

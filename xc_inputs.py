@@ -246,7 +246,9 @@ class Trajectory:
             z2 = normal(seed, f"{cfg.name}/eps/{n}", L * C).reshape(L, C)
             if n == 0:
                 xc, eps = z1, z2
-                a = uniform(seed, f"{cfg.name}/a0", A) - 0.5
+                # start from a steady driving state: |a_i| in [0.3, 0.7], random sign
+                u = uniform(seed, f"{cfg.name}/a0", 2 * A)
+                a = (0.3 + 0.4 * u[:A]) * np.where(u[A:] < 0.5, -1.0, 1.0)
             else:
                 s = math.sqrt(1.0 - rho * rho)
                 xc = rho * xc + s * z1
