@@ -10,17 +10,21 @@
 //   warp 8      TMA producer: Q0/Q1 once, then 128-key K and V tiles through
 //               a STAGES-deep ring (separate K and V barriers);
 //   warp 9      TMEM allocation; lane 0 issues every MMA.
-// TMEM (512 columns): S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after.
-// The two tiles ping-pong on the tensor core: while WG 0 turns S0 into
-// probabilities, the MMA warp runs P1 V and the next S1, and vice versa.
-// P (bf16) is written back into TMEM over its own S buffer and consumed by
-// tcgen05.mma with the A operand in tensor memory (no shared-memory round
-// trip); V is read MN-major straight from its [keys][hd] tile.
+// TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after it.  P (bf16)
+// goes back into TMEM and feeds tcgen05.mma as the A operand straight from
+// tensor memory (no shared-memory round trip); V is read MN-major from its
+// [keys][hd] tile.
+//   hd = 64 : P0 / P1 have their own 64 columns ([384,448), [448,512)), so
+//             S_{j+1} is issued as soon as the softmax has READ S_j and runs on
+//             the tensor core while the softmax computes P_j.
+//   hd = 128: TMEM is full (S0 S1 O0 O1 = 512 columns); P_i overwrites S_i and
+//             S_{j+1} waits until P_j V has been issued; the two tiles
+//             ping-pong so the tensor core still has the other tile's work.
 // Online softmax in the exp2 domain with lazy rescaling: a row's O and sum
 // are rescaled only when its running max grows by more than 8 (2^8 headroom
-// in fp32 / bf16), so after the first tiles the correction almost never runs.
-// Keys beyond n_keys (ragged last tile) are masked to -inf; their K/V rows are
-// finite (zero-initialised ring, TMA zero fill past the tensor end).
+// in fp32 / bf16).  Score scaling and row sums use packed fp32 pairs
+// (FFMA2 / FADD2).  Keys beyond n_keys (ragged last tile) are masked to -inf;
+// their K/V rows are finite (zero-initialised ring, TMA zero fill).
 #include "xc_ptx.cuh"
 
 namespace xc {
@@ -39,6 +43,10 @@ struct AttnTile {
     static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
     static constexpr int TMEM_COLS = 512;
     static constexpr int THREADS = 320;
+    static constexpr bool SEP_P = HD == 64;            // P has its own TMEM columns
+    __host__ __device__ static constexpr int S_COL(int i) { return 128 * i; }
+    __host__ __device__ static constexpr int O_COL(int i) { return 256 + HD * i; }
+    __host__ __device__ static constexpr int P_COL(int i) { return SEP_P ? 256 + 2 * HD + 64 * i : 128 * i; }
     static constexpr float LAZY = 8.0f;                // rescale threshold (log2 units)
 };
 
@@ -71,10 +79,11 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t *k_empty = k_full + A::STAGES;
     uint64_t *v_full = k_empty + A::STAGES;
     uint64_t *v_empty = v_full + A::STAGES;
-    uint64_t *s_full = v_empty + A::STAGES;    // [2] per tile
-    uint64_t *p_full = s_full + 2;             // [2]
-    uint64_t *o_done = p_full + 2;             // [2]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(o_done + 2);
+    uint64_t *s_full = v_empty + A::STAGES;    // [2] S_i computed
+    uint64_t *s_cons = s_full + 2;             // [2] S_i read by its softmax WG (hd 64)
+    uint64_t *p_full = s_cons + 2;             // [2] P_i written, O_i corrected
+    uint64_t *pv_done = p_full + 2;            // [2] P_i V done (hd 64: every tile; hd 128: last)
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(pv_done + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * (A::QT * A::BQ);
@@ -91,8 +100,9 @@ __global__ void __launch_bounds__(320, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
+            mbar_init(&s_cons[i], 128);
             mbar_init(&p_full[i], 128);
-            mbar_init(&o_done[i], 1);
+            mbar_init(&pv_done[i], 1);
         }
         mbar_fence_init();
     }
@@ -144,16 +154,16 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                 for (int ks = 0; ks < HD / 16; ++ks) {
                     const uint32_t off = (ks >> 2) * A::REGION + (ks & 3) * 32;
-                    tc_mma(tmem + 128 * i, sdesc_sw128(aQ + i * A::Q_BYTES + off, 16, 1024),
+                    tc_mma(tmem + A::S_COL(i), sdesc_sw128(aQ + i * A::Q_BYTES + off, 16, 1024),
                            sdesc_sw128(aK + st * A::KV_BYTES + off, 16, 1024), idesc_s, ks > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[i]);
             };
-            auto issue_pv = [&](int i, int j) {       // O_i += P_i V_j, P_i in TMEM over S_i
+            auto issue_pv = [&](int i, int j) {       // O_i += P_i V_j, P_i in TMEM
                 const int st = j % A::STAGES;
 #pragma unroll
                 for (int ks = 0; ks < A::BKV / 16; ++ks)
-                    tc_mma_tmem_a(tmem + 256 + HD * i, tmem + 128 * i + 8 * ks,
+                    tc_mma_tmem_a(tmem + A::O_COL(i), tmem + A::P_COL(i) + 8 * ks,
                                   sdesc_sw128(aV + st * A::KV_BYTES + ks * 16 * 128, A::REGION, 1024), idesc_o,
                                   (j > 0 || ks > 0) ? 1u : 0u);
             };
@@ -168,24 +178,48 @@ __global__ void __launch_bounds__(320, 1)
                 const int st = j % A::STAGES;
                 const int st1 = (j + 1) % A::STAGES;
                 const bool more = j + 1 < nkt;
-                if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
-                tc_fence_after();
-                issue_pv(0, j);
-                if (!more) tc_commit(&o_done[0]);
-                if (more) {
-                    if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                if constexpr (A::SEP_P) {
+                    // next scores as soon as the current ones have been read
+                    if (more) {
+                        if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                        if (!mbar_wait(&s_cons[0], j & 1, err, ERR_WAIT_MMA)) break;
+                        tc_fence_after();
+                        issue_s(0, j + 1);
+                        if (!mbar_wait(&s_cons[1], j & 1, err, ERR_WAIT_MMA)) break;
+                        tc_fence_after();
+                        issue_s(1, j + 1);
+                        tc_commit(&k_empty[st1]);
+                    }
+                    if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                    if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
                     tc_fence_after();
-                    issue_s(0, j + 1);
-                }
-                if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
-                tc_fence_after();
-                issue_pv(1, j);
-                tc_commit(&v_empty[st]);
-                if (!more) tc_commit(&o_done[1]);
-                if (more) {
-                    issue_s(1, j + 1);
-                    tc_commit(&k_empty[st1]);
+                    issue_pv(0, j);
+                    tc_commit(&pv_done[0]);
+                    if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
+                    tc_fence_after();
+                    issue_pv(1, j);
+                    tc_commit(&pv_done[1]);
+                    tc_commit(&v_empty[st]);
+                } else {
+                    if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                    if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
+                    tc_fence_after();
+                    issue_pv(0, j);
+                    if (!more) tc_commit(&pv_done[0]);
+                    if (more) {
+                        if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                        tc_fence_after();
+                        issue_s(0, j + 1);
+                    }
+                    if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
+                    tc_fence_after();
+                    issue_pv(1, j);
+                    tc_commit(&v_empty[st]);
+                    if (!more) tc_commit(&pv_done[1]);
+                    if (more) {
+                        issue_s(1, j + 1);
+                        tc_commit(&k_empty[st1]);
+                    }
                 }
             }
         }
@@ -195,8 +229,9 @@ __global__ void __launch_bounds__(320, 1)
         const int q = warp & 3;                            // TMEM lane quadrant
         const int row = q0 + wg * A::BQ + q * 32 + lane;
         const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
-        const uint32_t tS = tl + 128 * wg;
-        const uint32_t tO = tl + 256 + HD * wg;
+        const uint32_t tS = tl + A::S_COL(wg);
+        const uint32_t tP = tl + A::P_COL(wg);
+        const uint32_t tO = tl + A::O_COL(wg);
         const float sl2 = rsqrtf((float)HD) * 1.4426950408889634f;
         const int tail = n_keys - (nkt - 1) * A::BKV;      // valid keys in the last tile
         float m = -INFINITY, l = 0.0f;
@@ -208,6 +243,10 @@ __global__ void __launch_bounds__(320, 1)
             tc_fence_after();
             float s[128];
             tmem_ld128_sync(tS, s);
+            if constexpr (A::SEP_P) {
+                tc_fence_before();
+                mbar_arrive(&s_cons[wg]);
+            }
             if (j == nkt - 1 && tail < A::BKV) {
 #pragma unroll
                 for (int c = 0; c < 128; ++c)
@@ -222,53 +261,58 @@ __global__ void __launch_bounds__(320, 1)
                 mx3 = fmaxf(mx3, s[c + 3]);
             }
             const float m_new = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
-            if (j == 0) {
-                m = m_new;
-            } else {
-                const bool grow = m_new > m + A::LAZY;
-                if (__any_sync(0xffffffffu, grow)) {
-                    // O_i is stable: the commit behind s_full covers P V of tile j-1.
-                    const float alpha = grow ? ex2_approx(m - m_new) : 1.0f;
-#pragma unroll 1
-                    for (int c = 0; c < HD / 16; ++c) {
-                        float t[16];
-                        tmem_ld16_sync(tO + 16 * c, t);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) t[i] *= alpha;
-                        tmem_st16_sync(tO + 16 * c, t);
-                    }
-                    l *= alpha;
-                    if (grow) m = m_new;
+            const bool grow = j > 0 && m_new > m + A::LAZY;
+            const float alpha = grow ? ex2_approx(m - m_new) : 1.0f;
+            if (j == 0 || grow) m = m_new;
+            if constexpr (A::SEP_P) {
+                // P_i buffer free and O_i stable once P V of the previous tile is done
+                if (j >= 1) {
+                    ok = mbar_wait(&pv_done[wg], (j - 1) & 1, err, ERR_WAIT_SOFTMAX);
+                    __syncwarp();
+                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                    tc_fence_after();
                 }
             }
-            const float nm = -m;
-            float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
+            // (hd 128: the commit behind s_full already covers P V of tile j-1)
+            if (__any_sync(0xffffffffu, grow)) {
+#pragma unroll 1
+                for (int c = 0; c < HD / 16; ++c) {
+                    float t[16];
+                    tmem_ld16_sync(tO + 16 * c, t);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) t[i] *= alpha;
+                    tmem_st16_sync(tO + 16 * c, t);
+                }
+            }
+            // probabilities p = 2^(s * sl2 - m), packed bf16 pairs + row sum,
+            // stored to TMEM in two 64-key halves
+            const float2 sc2 = make_float2(sl2, sl2), nm2 = make_float2(-m, -m);
+            float2 rs0 = make_float2(0.f, 0.f), rs1 = make_float2(0.f, 0.f);
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
                 uint32_t w[32];
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    const int c = 64 * half + 2 * i;
-                    const float p0 = ex2_approx(fmaf(s[c], sl2, nm));
-                    const float p1 = ex2_approx(fmaf(s[c + 1], sl2, nm));
-                    const float p2 = ex2_approx(fmaf(s[c + 2], sl2, nm));
-                    const float p3 = ex2_approx(fmaf(s[c + 3], sl2, nm));
-                    r0 += p0;
-                    r1 += p1;
-                    r2 += p2;
-                    r3 += p3;
-                    __nv_bfloat162 h0 = __floats2bfloat162_rn(p0, p1);
-                    __nv_bfloat162 h1 = __floats2bfloat162_rn(p2, p3);
-                    w[i] = *reinterpret_cast<uint32_t *>(&h0);
-                    w[i + 1] = *reinterpret_cast<uint32_t *>(&h1);
+                for (int k = 0; k < 32; k += 2) {
+                    const int c = 64 * half + 2 * k;
+                    const float2 a = __ffma2_rn(make_float2(s[c], s[c + 1]), sc2, nm2);
+                    const float2 b = __ffma2_rn(make_float2(s[c + 2], s[c + 3]), sc2, nm2);
+                    const float2 pa = make_float2(ex2_approx(a.x), ex2_approx(a.y));
+                    const float2 pb = make_float2(ex2_approx(b.x), ex2_approx(b.y));
+                    rs0 = __fadd2_rn(rs0, pa);
+                    rs1 = __fadd2_rn(rs1, pb);
+                    __nv_bfloat162 h0 = __floats2bfloat162_rn(pa.x, pa.y);
+                    __nv_bfloat162 h1 = __floats2bfloat162_rn(pb.x, pb.y);
+                    w[k] = *reinterpret_cast<uint32_t *>(&h0);
+                    w[k + 1] = *reinterpret_cast<uint32_t *>(&h1);
                 }
-                tmem_st32_sync(tS + 32 * half, w);
+                tmem_st32_sync(tP + 32 * half, w);
             }
-            l += (r0 + r1) + (r2 + r3);
+            const float2 rs = __fadd2_rn(rs0, rs1);
+            l = l * alpha + (rs.x + rs.y);
             tc_fence_before();
             mbar_arrive(&p_full[wg]);
         }
-        if (ok) ok = mbar_wait(&o_done[wg], 0, err, ERR_WAIT_SOFTMAX);
+        if (ok) ok = mbar_wait(&pv_done[wg], A::SEP_P ? ((nkt - 1) & 1) : 0, err, ERR_WAIT_SOFTMAX);
         __syncwarp();
         if (__all_sync(0xffffffffu, ok)) {
             tc_fence_after();
