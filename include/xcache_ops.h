@@ -64,6 +64,46 @@ xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x,
 xc_status xc_op_residual_reuse(int dtype, long n, const void *x, const void *rhat, void *out,
                                void *stream);
 
+/* Per-(t, b) gate state kept on the device (32 bytes): EMA of the cosine
+ * (Eq. 8), has-history bit, consecutive-skip counter (Section 2.5 (4)),
+ * cache-valid bit, and which half of the double-buffered cached fingerprint
+ * is active. */
+typedef struct {
+    double ema;
+    int has_hist, stale, valid, active;
+    int pad[2];
+} xc_gate_cell;
+
+/* Bytes of device workspace xc_op_gate needs for this geometry. */
+size_t xc_op_gate_workspace_bytes(int dtype, int n_cams, int tokens_per_cam, int d);
+
+/* One gate evaluation of one (t, b) cell (Section 2.3-2.5): fingerprint of the
+ * block input x (spatial sample, per-camera token mean, action), min-cosine
+ * s_cos (Eq. 5) and max token deviation d_max (Eq. 6) against the cached
+ * fingerprint, adaptive threshold (Eq. 9), decision (Eq. 7), EMA (Eq. 8) and
+ * staleness updates.
+ *   x        device [n_cams * tokens_per_cam][d] activation dtype
+ *   fp_rows  device int [n_cams][kfp]: token rows of the spatial sample
+ *   phi      device float [2][n_cams*kfp*d + n_cams*d]: the two halves of the
+ *            cached fingerprint (spatial entries, then per-camera means); the
+ *            current fingerprint is written into the inactive half
+ *   phi_act  device float [2][8]: cached action halves
+ *   cell     device xc_gate_cell, updated in place
+ *   action   host float [action_dim] (action_dim <= 8)
+ *   mode     1 evaluate the gate, 0 refresh only (forced compute)
+ *   step     denoising step t (strict step-0 threshold)
+ *   gate     knobs (NULL = Table 1); replay_skip[0], when set, replaces the
+ *            decision (decision-replay mode)
+ *   flag     device uint8 decision (xc_decision); s_cos, d_max, tau device float
+ *   workspace device, >= xc_op_gate_workspace_bytes(); its counters are
+ *            cleared by the call (cudaMemsetAsync), nothing is allocated
+ * Asynchronous on `stream`.  Errors: XC_EINVAL. */
+xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows,
+                     int kfp, float *phi, float *phi_act, xc_gate_cell *cell, const float *action,
+                     int action_dim, int mode, int step, const xc_gate_params *gate, uint8_t *flag,
+                     float *s_cos, float *d_max, float *tau, void *workspace, size_t workspace_bytes,
+                     void *stream);
+
 /* Reads and clears the process-wide device error word of operator calls
  * (synchronising).  0 = no error. */
 int xc_op_device_error(void);

@@ -1124,6 +1124,109 @@ xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x, const 
     return XC_OK;
 }
 
+// Workspace of one gate launch: column sums [V][R][d] f32, spatial partials
+// [V*ns*R][5] f64, global partials [V*ns][3] f64, tickets [V*ns + 1] u32.
+struct GateWorkspace {
+    int ns, R;
+    size_t colsum, sp, gl, cnt, cnt_bytes, total;
+};
+static GateWorkspace gate_workspace(int V, int npc, int d) {
+    int dev = 0, n_sm = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    GateWorkspace w;
+    gate_geometry(V, npc, d, n_sm, &w.ns, &w.R);
+    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    size_t off = 0;
+    w.colsum = off;
+    off = al(off + (size_t)V * w.R * d * sizeof(float));
+    w.sp = off;
+    off = al(off + (size_t)V * w.ns * w.R * 5 * sizeof(double));
+    w.gl = off;
+    off = al(off + (size_t)V * w.ns * 3 * sizeof(double));
+    w.cnt = off;
+    w.cnt_bytes = (size_t)(V * w.ns + 1) * sizeof(unsigned);
+    off = al(off + w.cnt_bytes);
+    w.total = off;
+    return w;
+}
+
+size_t xc_op_gate_workspace_bytes(int dtype, int n_cams, int tokens_per_cam, int d) {
+    (void)dtype;
+    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0) return 0;
+    return gate_workspace(n_cams, tokens_per_cam, d).total;
+}
+
+static_assert(sizeof(xc_gate_cell) == sizeof(GateCell), "gate cell layout");
+
+xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows, int kfp,
+                     float *phi, float *phi_act, xc_gate_cell *cell, const float *action, int action_dim, int mode,
+                     int step, const xc_gate_params *gate, uint8_t *flag, float *s_cos, float *d_max, float *tau,
+                     void *workspace, size_t workspace_bytes, void *stream) {
+    if (dtype != XC_F32 && dtype != XC_BF16) OP_FAIL(XC_EINVAL, "xc_op_gate: dtype");
+    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0 || kfp < 1 || kfp > tokens_per_cam ||
+        action_dim < 1 || action_dim > 8 || (mode != 0 && mode != 1) || step < 0)
+        OP_FAIL(XC_EINVAL, "xc_op_gate: bad shape or mode (d %% 64 == 0, 1 <= kfp <= tokens_per_cam, "
+                           "action_dim <= 8)");
+    if (x == nullptr || fp_rows == nullptr || phi == nullptr || phi_act == nullptr || cell == nullptr ||
+        action == nullptr || flag == nullptr || s_cos == nullptr || d_max == nullptr || tau == nullptr ||
+        workspace == nullptr)
+        OP_FAIL(XC_EINVAL, "xc_op_gate: NULL pointer");
+    xc_gate_params p;
+    if (gate != nullptr)
+        p = *gate;
+    else
+        xc_gate_params_default(&p);
+    char why[256];
+    if (!gate_ok(&p, 1, why, sizeof why)) OP_FAIL(XC_EINVAL, "xc_op_gate: %s", why);
+    const GateWorkspace ws = gate_workspace(n_cams, tokens_per_cam, d);
+    if (workspace_bytes < ws.total)
+        OP_FAIL(XC_EINVAL, "xc_op_gate: workspace %zu bytes < %zu needed", workspace_bytes, ws.total);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    char *w = reinterpret_cast<char *>(workspace);
+    OP_CK(cudaMemsetAsync(w + ws.cnt, 0, ws.cnt_bytes, st));
+    GateArgs g;
+    memset(&g, 0, sizeof g);
+    g.x = x;
+    g.d = d;
+    g.V = n_cams;
+    g.npc = tokens_per_cam;
+    g.fp_rows = fp_rows;
+    g.kfp = kfp;
+    g.n_slices = ws.ns;
+    g.R = ws.R;
+    g.phi = phi;
+    g.phi_act = phi_act;
+    for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
+    g.A = action_dim;
+    g.cell = reinterpret_cast<GateCell *>(cell);
+    g.mode = mode;
+    g.step = step;
+    g.tau_floor = p.tau_floor;
+    g.margin = p.margin;
+    g.alpha = p.alpha;
+    g.tau_dev = p.tau_dev;
+    g.eps_dev = p.eps_dev;
+    g.strict_tau = p.step0_strict_tau;
+    g.max_skips = p.max_skips;
+    g.fp_refresh = p.fp_refresh;
+    g.replay = p.replay_skip != nullptr ? (p.replay_skip[0] != 0 ? 1 : 0) : -1;
+    g.flag = flag;
+    g.s_cos = s_cos;
+    g.d_max = d_max;
+    g.tau_out = tau;
+    g.colsum = reinterpret_cast<float *>(w + ws.colsum);
+    g.sp_part = reinterpret_cast<double *>(w + ws.sp);
+    g.gl_part = reinterpret_cast<double *>(w + ws.gl);
+    g.cnt_cs = reinterpret_cast<unsigned *>(w + ws.cnt);
+    g.cnt_all = g.cnt_cs + n_cams * ws.ns;
+    if (dtype == XC_BF16)
+        OP_CK(gate_launch<bf16>(g, st));
+    else
+        OP_CK(gate_launch<float>(g, st));
+    return XC_OK;
+}
+
 xc_status xc_op_residual_reuse(int dtype, long n, const void *x, const void *rhat, void *out, void *stream) {
     if (n < 0 || n % 16 != 0 || x == nullptr || rhat == nullptr || out == nullptr)
         OP_FAIL(XC_EINVAL, "xc_op_residual_reuse: bad argument (n %% 16 == 0 required)");

@@ -97,6 +97,9 @@ SIGNATURES = {
     "xc_op_ln_mod": (_I, [_I, _I, _I, _F, _P, _P, _P, _P, _P]),
     "xc_op_residual_reuse": (_I, [_I, _L, _P, _P, _P, _P]),
     "xc_op_device_error": (_I, []),
+    "xc_op_gate_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I]),
+    "xc_op_gate": (_I, [_I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _P, _I, _I, _I, ctypes.POINTER(GateParams),
+                        _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
 }
 
 
@@ -283,3 +286,25 @@ def op_residual_reuse(dtype, x, rhat, out, stream=None):
 
 def op_device_error() -> int:
     return LIB.xc_op_device_error()
+
+
+class GateCell(ctypes.Structure):
+    """xc_gate_cell: per-(t, b) gate state (32 bytes)."""
+    _fields_ = [("ema", ctypes.c_double), ("has_hist", ctypes.c_int), ("stale", ctypes.c_int),
+                ("valid", ctypes.c_int), ("active", ctypes.c_int), ("pad", ctypes.c_int * 2)]
+
+
+def op_gate_workspace_bytes(dtype, n_cams, tokens_per_cam, d) -> int:
+    return LIB.xc_op_gate_workspace_bytes(dtype_code(dtype), n_cams, tokens_per_cam, d)
+
+
+def op_gate(dtype, n_cams, tokens_per_cam, x, fp_rows, phi, phi_act, cell, action, mode, step,
+            gate, flag, s_cos, d_max, tau, workspace, stream=None):
+    """x, fp_rows [n_cams, kfp] int32, phi, phi_act, cell (uint8 tensor of 32 bytes), flag,
+    s_cos, d_max, tau, workspace: torch CUDA tensors; action: numpy float32."""
+    act = np.ascontiguousarray(action, dtype=np.float32)
+    check(LIB.xc_op_gate(dtype_code(dtype), n_cams, tokens_per_cam, x.shape[1], _ptr(x), _ptr(fp_rows),
+            fp_rows.shape[1], _ptr(phi), _ptr(phi_act), _ptr(cell), act.ctypes.data, act.size, mode,
+            step, ctypes.byref(gate) if gate is not None else None, _ptr(flag), _ptr(s_cos),
+            _ptr(d_max), _ptr(tau), _ptr(workspace), workspace.numel() * workspace.element_size(),
+            _stream(stream)))
