@@ -20,6 +20,11 @@
 // decision is deterministic.  The cached fingerprint is double-buffered per
 // (t, b): the current fingerprint is written to the inactive half, which
 // becomes active when the block recomputes (refresh on compute).
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
 #include "xc_kernels.cuh"
 
 namespace xc {
@@ -274,4 +279,136 @@ cudaError_t gate_launch(const GateArgs &g, cudaStream_t st) {
 template cudaError_t gate_launch<float>(const GateArgs &, cudaStream_t);
 template cudaError_t gate_launch<bf16>(const GateArgs &, cudaStream_t);
 
+// ---------------------------------------------------------------------------
+// Allocation-free gate (xc_op_gate_static).  The gate kernel needs scratch for
+// its column sums, partial metrics and tickets.  Here that scratch is one
+// file-scope device array: every GPU that loads the library holds it until
+// the process exits, and no call allocates or frees anything.  In host code
+// the array's name is only a host-side stand-in, so its device address is
+// looked up once per device with cudaGetSymbolAddress (the first call on a
+// device does this set-up) and passed to the kernel.
+// ---------------------------------------------------------------------------
+constexpr size_t GATE_STATIC_SCRATCH_BYTES = 1u << 20;   // 1 MiB
+static __device__ __align__(256) unsigned char g_gate_scratch[GATE_STATIC_SCRATCH_BYTES];
+
+static std::mutex g_static_mu;
+static void *g_static_ptr[64];                          // device address per device ordinal
+
+// Device address of g_gate_scratch on the current device (set-up once per device).
+static cudaError_t static_scratch(void **out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_static_mu);
+    if (g_static_ptr[dev] == nullptr) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_gate_scratch);
+        if (e != cudaSuccess) return e;
+        g_static_ptr[dev] = p;
+    }
+    *out = g_static_ptr[dev];
+    return cudaSuccess;
+}
+
 }  // namespace xc
+
+using xc::GateArgs;
+using xc::GateCell;
+
+extern "C" xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam, int d, const void *x,
+                                       const int *fp_rows, int kfp, float *phi, float *phi_act,
+                                       xc_gate_cell *cell, const float *action, int action_dim, int mode,
+                                       int step, const xc_gate_params *gate, uint8_t *flag, float *s_cos,
+                                       float *d_max, float *tau, void *stream) {
+    char msg[256];
+    auto fail = [&](xc_status s, const char *m) {
+        snprintf(msg, sizeof msg, "xc_op_gate_static: %s", m);
+        xc::set_global_error(msg);
+        return s;
+    };
+    if (dtype != XC_F32 && dtype != XC_BF16) return fail(XC_EINVAL, "dtype");
+    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0 || kfp < 1 || kfp > tokens_per_cam ||
+        action_dim < 1 || action_dim > 8 || (mode != 0 && mode != 1) || step < 0)
+        return fail(XC_EINVAL, "bad shape or mode (d % 64 == 0, 1 <= kfp <= tokens_per_cam, action_dim <= 8)");
+    if (x == nullptr || fp_rows == nullptr || phi == nullptr || phi_act == nullptr || cell == nullptr ||
+        action == nullptr || flag == nullptr || s_cos == nullptr || d_max == nullptr || tau == nullptr)
+        return fail(XC_EINVAL, "NULL pointer");
+    xc_gate_params p;
+    if (gate != nullptr)
+        p = *gate;
+    else
+        xc_gate_params_default(&p);
+    const float knobs[] = {p.tau_floor, p.margin, p.alpha, p.tau_dev, p.eps_dev, p.step0_strict_tau};
+    for (float v : knobs)
+        if (isnan(v)) return fail(XC_EINVAL, "NaN gate knob");
+    if (p.alpha < 0.0f || p.alpha > 1.0f || p.max_skips < 0 || (p.fp_refresh != 0 && p.fp_refresh != 1))
+        return fail(XC_EINVAL, "gate knob out of range");
+
+    // scratch layout, as for the caller-workspace gate
+    int dev = 0, n_sm = 152;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return fail(XC_ECUDA, "no CUDA device");
+    int ns = 0, R = 0;
+    xc::gate_geometry(n_cams, tokens_per_cam, d, n_sm, &ns, &R);
+    auto al = [](size_t v) { return (v + 255) & ~(size_t)255; };
+    const size_t off_sp = al((size_t)n_cams * R * d * sizeof(float));
+    const size_t off_gl = al(off_sp + (size_t)n_cams * ns * R * 5 * sizeof(double));
+    const size_t off_cnt = al(off_gl + (size_t)n_cams * ns * 3 * sizeof(double));
+    const size_t cnt_bytes = (size_t)(n_cams * ns + 1) * sizeof(unsigned);
+    const size_t need = off_cnt + cnt_bytes;
+    if (need > xc::GATE_STATIC_SCRATCH_BYTES) {
+        snprintf(msg, sizeof msg,
+                 "xc_op_gate_static: this geometry needs %zu bytes of scratch, more than the %zu-byte "
+                 "static maximum (use xc_op_gate with a workspace)",
+                 need, xc::GATE_STATIC_SCRATCH_BYTES);
+        xc::set_global_error(msg);
+        return XC_EINVAL;
+    }
+    void *scratch = nullptr;
+    if (xc::static_scratch(&scratch) != cudaSuccess) return fail(XC_ECUDA, "cudaGetSymbolAddress failed");
+    char *w = reinterpret_cast<char *>(scratch);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // the tickets must start at zero; the rest of the array is overwritten
+    if (cudaMemsetAsync(w + off_cnt, 0, cnt_bytes, st) != cudaSuccess) return fail(XC_ECUDA, "cudaMemsetAsync");
+
+    GateArgs g;
+    memset(&g, 0, sizeof g);
+    g.x = x;
+    g.d = d;
+    g.V = n_cams;
+    g.npc = tokens_per_cam;
+    g.fp_rows = fp_rows;
+    g.kfp = kfp;
+    g.n_slices = ns;
+    g.R = R;
+    g.phi = phi;
+    g.phi_act = phi_act;
+    for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
+    g.A = action_dim;
+    g.cell = reinterpret_cast<GateCell *>(cell);
+    g.mode = mode;
+    g.step = step;
+    g.tau_floor = p.tau_floor;
+    g.margin = p.margin;
+    g.alpha = p.alpha;
+    g.tau_dev = p.tau_dev;
+    g.eps_dev = p.eps_dev;
+    g.strict_tau = p.step0_strict_tau;
+    g.max_skips = p.max_skips;
+    g.fp_refresh = p.fp_refresh;
+    g.replay = p.replay_skip != nullptr ? (p.replay_skip[0] != 0 ? 1 : 0) : -1;
+    g.flag = flag;
+    g.s_cos = s_cos;
+    g.d_max = d_max;
+    g.tau_out = tau;
+    g.colsum = reinterpret_cast<float *>(w);
+    g.sp_part = reinterpret_cast<double *>(w + off_sp);
+    g.gl_part = reinterpret_cast<double *>(w + off_gl);
+    g.cnt_cs = reinterpret_cast<unsigned *>(w + off_cnt);
+    g.cnt_all = g.cnt_cs + n_cams * ns;
+    const cudaError_t e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, st) : xc::gate_launch<float>(g, st);
+    if (e != cudaSuccess) return fail(XC_ECUDA, cudaGetErrorString(e));
+    return XC_OK;
+}

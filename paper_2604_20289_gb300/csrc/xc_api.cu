@@ -167,6 +167,12 @@ void set_err(xc_ctx *c, const char *fmt, ...) {
     g_global_err = buf;
 }
 
+}  // namespace
+
+void xc::set_global_error(const char *msg) { set_err(nullptr, "%s", msg); }
+
+namespace {
+
 #define CK(call)                                                                            \
     do {                                                                                    \
         cudaError_t e_ = (call);                                                            \

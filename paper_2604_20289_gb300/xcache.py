@@ -100,6 +100,8 @@ SIGNATURES = {
     "xc_op_gate_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I]),
     "xc_op_gate": (_I, [_I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _P, _I, _I, _I, ctypes.POINTER(GateParams),
                         _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "xc_op_gate_static": (_I, [_I, _I, _I, _I, _P, _P, _I, _P, _P, _P, _P, _I, _I, _I,
+                               ctypes.POINTER(GateParams), _P, _P, _P, _P, _P]),
 }
 
 
