@@ -250,6 +250,36 @@ cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, co
     return cudaGetLastError();
 }
 
+// RoPE (cos, sin) table of one chunk, double precision.  Axes (camera, frame,
+// h, w) own hd/16, 3hd/16, hd/8, hd/8 consecutive pairs; pair j of an axis
+// with D = 2 * pairs dims rotates at theta^(-2j/D).  Axis a has npos[a]
+// positions (frame: the chunk's frames, absolute frame = frame0 + p); entry
+// base_a + j * npos[a] + p holds (cos, sin)(pos * freq).
+__global__ void rope_table_kernel(int hd, double theta, int frame0, int4 npos, float2 *__restrict__ out, int n) {
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= n) return;
+    const int pairs[4] = {hd / 16, 3 * hd / 16, hd / 8, hd / 8};
+    const int np[4] = {npos.x, npos.y, npos.z, npos.w};
+    int base = 0;
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        const int span = pairs[a] * np[a];
+        if (e < base + span) {
+            const int j = (e - base) / np[a];
+            const int p = (e - base) % np[a];
+            const double freq = pow(theta, -2.0 * j / (2.0 * pairs[a]));
+            const double ang = (double)(p + (a == 1 ? frame0 : 0)) * freq;
+            out[e] = make_float2((float)cos(ang), (float)sin(ang));
+            return;
+        }
+        base += span;
+    }
+}
+cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out, int n, cudaStream_t st) {
+    rope_table_kernel<<<(n + 127) / 128, 128, 0, st>>>(hd, theta, frame0, npos, out, n);
+    return cudaGetLastError();
+}
+
 // mods_all[b][j][c] = m[j*d + c] + blk_mod[b][j][c]   (B x 6 x d)
 __global__ void assemble_mods_kernel(const float *__restrict__ m, const float *__restrict__ tab,
                                      float *__restrict__ out, int B, int d) {

@@ -101,16 +101,30 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     const float *phi_prev = g.phi + (size_t)active * n_all;
     float *phi_next = g.phi + (size_t)(active ^ 1) * n_all;
 
-    // 1. column sums of this CTA's rows (global channel partials)
+    __shared__ int s_i0, s_i1;
+    if (tid == 0) {
+        s_i0 = g.kfp;
+        s_i1 = 0;
+    }
+    __syncthreads();
+    // fingerprint rows of this camera that fall in [rbeg, rend) (rows ascend)
+    for (int i = tid; i < g.kfp; i += GATE_THREADS) {
+        const int row = g.fp_rows[c * g.kfp + i];
+        if (row >= rbeg && row < rend) {
+            atomicMin(&s_i0, i);
+            atomicMax(&s_i1, i + 1);
+        }
+    }
+
+    // 1. column sums of this CTA's rows (global channel partials); 4 rows in
+    //    flight per thread
     {
         const int ty = tid / TPR, tx = tid % TPR;
         float acc[VEC];
 #pragma unroll
         for (int i = 0; i < VEC; ++i) acc[i] = 0.0f;
-        for (int row = rbeg + ty; row < rend; row += RPAR) {
-            const T *p = x + (size_t)row * d + col0 + tx * VEC;
+        auto add16 = [&](const uint4 u) {
             if constexpr (VEC == 8) {
-                const uint4 u = *reinterpret_cast<const uint4 *>(p);
                 const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
@@ -119,10 +133,22 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
                     acc[2 * j + 1] += f.y;
                 }
             } else {
-                const float4 f = *reinterpret_cast<const float4 *>(p);
-                acc[0] += f.x; acc[1] += f.y; acc[2] += f.z; acc[3] += f.w;
+                acc[0] += __uint_as_float(u.x);
+                acc[1] += __uint_as_float(u.y);
+                acc[2] += __uint_as_float(u.z);
+                acc[3] += __uint_as_float(u.w);
             }
+        };
+        const T *base = x + (size_t)col0 + tx * VEC;
+        int row = rbeg + ty;
+        for (; row + 3 * RPAR < rend; row += 4 * RPAR) {
+            uint4 u[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) u[k] = *reinterpret_cast<const uint4 *>(base + (size_t)(row + k * RPAR) * d);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) add16(u[k]);
         }
+        for (; row < rend; row += RPAR) add16(*reinterpret_cast<const uint4 *>(base + (size_t)row * d));
 #pragma unroll
         for (int i = 0; i < VEC; ++i) red[ty * GATE_CW + tx * VEC + i] = acc[i];
         __syncthreads();
@@ -137,10 +163,10 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     //    current fingerprint into the inactive buffer
     {
         double v[5] = {0.0, 0.0, 0.0, 0.0, 0.0};   // dot, |cur|^2, |prev|^2, max|diff|, sum|prev|
-        for (int it = tid; it < g.kfp * GATE_CW; it += GATE_THREADS) {
-            const int i = it / GATE_CW, j = it % GATE_CW;
+        const int i0 = s_i0, n_in = s_i1 > s_i0 ? s_i1 - s_i0 : 0;   // read after the barrier above
+        for (int it = tid; it < n_in * GATE_CW; it += GATE_THREADS) {
+            const int i = i0 + it / GATE_CW, j = it % GATE_CW;
             const int row = g.fp_rows[c * g.kfp + i];
-            if (row < rbeg || row >= rend) continue;
             const size_t e = ((size_t)c * g.kfp + i) * d + col0 + j;
             const double cur = (double)to_f(x[(size_t)row * d + col0 + j]);
             const double prev = (double)phi_prev[e];

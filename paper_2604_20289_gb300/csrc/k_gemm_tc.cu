@@ -2,13 +2,14 @@
 //
 //   C[M][N] = epilogue(A[M][K] @ Wt[N][K]^T), fp32 accumulation in TMEM.
 //
-// One CTA computes a 128 x BN tile.  Warp roles (192 threads):
+// One CTA computes a 128 x BN tile.  Warp roles (320 threads):
 //   warp 0, lane 0 : TMA producer, STAGES-deep ring of (A 128x64, B BNx64)
 //                    tiles in 128B-swizzled shared memory;
 //   warp 1         : allocates TMEM; lane 0 issues tcgen05.mma (M=128, N=BN,
 //                    K=16 per instruction, 4 per 64-wide k-tile) and commits
 //                    each stage back to the producer;
-//   warps 2..5     : epilogue -- tcgen05.ld of their 32-lane TMEM quadrant,
+//   warps 2..9     : epilogue -- tcgen05.ld of their 32-lane TMEM quadrant
+//                    (two warps per quadrant, half of the columns each),
 //                    fused bias / GELU / gated residual / residual-cache /
 //                    RoPE, vectorised stores.
 // The skip flag of the block lets the whole recompute path early-exit when
@@ -37,7 +38,7 @@ __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
 }
 
 template <int BN, int EPI, typename T>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const EpiParams ep, const int K, const uint8_t *__restrict__ skip_flag, int *err) {
     using G = GemmTile<BN>;
@@ -104,14 +105,16 @@ __global__ void __launch_bounds__(192, 1)
             tc_commit(done);
         }
     } else {
+        // warps 2..9: two warps per TMEM lane quadrant, each half of the columns
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
+        const int half = (warp - 2) >> 2;
         const bool ok = mbar_wait(done, 0, err, ERR_WAIT_EPI);
         tc_fence_after();
         if (ok) {
             const int row = m0 + q * 32 + lane;
             const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
-            for (int c = 0; c < BN; c += 16) {
+            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
                 float v[16];
                 tmem_ld16_sync(tq + c, v);
                 epilogue16<EPI, T>(ep, row, n0 + c, v);
@@ -173,7 +176,7 @@ static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const
         attr_set = true;
     }
     dim3 grid(ep.N / BN, (ep.M + GEMM_BM - 1) / GEMM_BM);
-    kern<<<grid, 192, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
+    kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
     return cudaGetLastError();
 }
 

@@ -32,15 +32,21 @@ struct Fail {
 
 // RoPE pair table: head_dim split hd/8 (camera) : 3hd/8 (absolute frame) :
 // hd/4 (h) : hd/4 (w); pair j of an axis with D dims rotates at theta^(-2j/D).
-void rope_table(int hd, double theta, std::vector<float> &freq, std::vector<int> &axis) {
+// For the per-chunk (cos, sin) table (rope_table_kernel): the axis of every
+// pair and the table entry of its position 0; npos = positions per axis
+// (cameras, frames per chunk, h, w).  Returns the number of table entries.
+int rope_layout(int hd, const int npos[4], std::vector<int> &axis, std::vector<int> &off) {
     const int dims[4] = {hd / 8, 3 * hd / 8, hd / 4, hd / 4};
-    freq.clear();
     axis.clear();
+    off.clear();
+    int base = 0;
     for (int a = 0; a < 4; ++a)
         for (int j = 0; j < dims[a] / 2; ++j) {
             axis.push_back(a);
-            freq.push_back((float)std::pow(theta, -2.0 * j / dims[a]));
+            off.push_back(base);
+            base += npos[a];
         }
+    return base;
 }
 
 // Spatial sample of the fingerprint (Section 2.3.1): per axis
@@ -105,8 +111,9 @@ struct xc_ctx {
     float *mod_w, *mod_b, *blk_mod, *head_w, *head_b, *head_tab, *out_w, *out_b;
     void *qkv_wt, *o_wt, *f1_wt, *f2_wt;      // [B][N][K] activation dtype
     float *qkv_b, *o_b, *f1_b, *f2_b;          // [B][N]
-    float *rope_freq;
-    int *rope_axis;
+    int *rope_axis, *rope_off;                 // per pair
+    float2 *rope_cs;                           // per-chunk (cos, sin) table
+    int rope_n;
 
     // activations / conditioning
     void *xb[2], *x1, *hbuf, *q, *o, *u;
@@ -356,6 +363,11 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
 
     T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
     LAUNCH(XC_K_EMBED, -1, 1, patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
+    // RoPE table of this chunk (absolute frames n*F .. n*F + F - 1)
+    LAUNCH(XC_K_EMBED, -1, 1,
+           rope_table(hd, (double)ctx->cfg.rope_theta, n * ctx->cfg.frames,
+                      make_int4(ctx->V, ctx->cfg.frames, ctx->cfg.grid_h, ctx->cfg.grid_w), ctx->rope_cs,
+                      ctx->rope_n, st));
     CK(cudaMemsetAsync(ctx->flags, 0, B, st));
     CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
 
@@ -433,8 +445,9 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.gw = ctx->cfg.grid_w;
         ep.frames = ctx->cfg.frames;
         ep.frame0 = n * ctx->cfg.frames;
-        ep.rope_freq = ctx->rope_freq;
         ep.rope_axis = ctx->rope_axis;
+        ep.rope_off = ctx->rope_off;
+        ep.rope_cs = ctx->rope_cs;
         if constexpr (sizeof(T) == 2) {
             LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
             LAUNCH(XC_K_ATTN, b, 1, attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L,
@@ -640,13 +653,14 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
             cudaFree(tmp);
         }
         {
-            std::vector<float> fr;
-            std::vector<int> ax;
-            rope_table(ctx->hd, cfg->rope_theta, fr, ax);
-            ctx->rope_freq = dalloc<float>(ctx, fr.size() * sizeof(float));
+            std::vector<int> ax, off;
+            const int npos[4] = {cfg->n_cams, cfg->frames, cfg->grid_h, cfg->grid_w};
+            ctx->rope_n = rope_layout(ctx->hd, npos, ax, off);
             ctx->rope_axis = dalloc<int>(ctx, ax.size() * sizeof(int));
-            CK(cudaMemcpy(ctx->rope_freq, fr.data(), fr.size() * sizeof(float), cudaMemcpyHostToDevice));
+            ctx->rope_off = dalloc<int>(ctx, off.size() * sizeof(int));
+            ctx->rope_cs = dalloc<float2>(ctx, (size_t)ctx->rope_n * sizeof(float2));
             CK(cudaMemcpy(ctx->rope_axis, ax.data(), ax.size() * sizeof(int), cudaMemcpyHostToDevice));
+            CK(cudaMemcpy(ctx->rope_off, off.data(), off.size() * sizeof(int), cudaMemcpyHostToDevice));
         }
 
         // activations
@@ -1038,24 +1052,29 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
         d % head_dim != 0 || A == nullptr || Wt == nullptr || bias == nullptr || q == nullptr || k == nullptr ||
         v == nullptr)
         OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: bad argument");
-    static float *freq = nullptr;
-    static int *axis = nullptr;
-    static int table_hd = -1;
-    static float table_theta = 0.0f;
-    if (table_hd != head_dim || table_theta != rope_theta) {
-        std::vector<float> fr;
-        std::vector<int> ax;
-        rope_table(head_dim, rope_theta, fr, ax);
-        cudaDeviceSynchronize();
-        if (freq) cudaFree(freq);
+    // per-call RoPE layout and table (operator path; the chunk step keeps its own)
+    static int *axis = nullptr, *off = nullptr;
+    static float2 *cs = nullptr;
+    static size_t cap_pairs = 0, cap_entries = 0;
+    std::vector<int> ax, of;
+    const int npos[4] = {n_cams, frames, gh, gw};
+    const int n_entries = rope_layout(head_dim, npos, ax, of);
+    cudaStream_t st0 = reinterpret_cast<cudaStream_t>(stream);
+    if (ax.size() > cap_pairs || (size_t)n_entries > cap_entries) {
+        OP_CK(cudaDeviceSynchronize());
         if (axis) cudaFree(axis);
-        OP_CK(cudaMalloc(&freq, fr.size() * sizeof(float)));
-        OP_CK(cudaMalloc(&axis, ax.size() * sizeof(int)));
-        OP_CK(cudaMemcpy(freq, fr.data(), fr.size() * sizeof(float), cudaMemcpyHostToDevice));
-        OP_CK(cudaMemcpy(axis, ax.data(), ax.size() * sizeof(int), cudaMemcpyHostToDevice));
-        table_hd = head_dim;
-        table_theta = rope_theta;
+        if (off) cudaFree(off);
+        if (cs) cudaFree(cs);
+        cap_pairs = ax.size();
+        cap_entries = (size_t)n_entries;
+        OP_CK(cudaMalloc(&axis, cap_pairs * sizeof(int)));
+        OP_CK(cudaMalloc(&off, cap_pairs * sizeof(int)));
+        OP_CK(cudaMalloc(&cs, cap_entries * sizeof(float2)));
     }
+    OP_CK(cudaMemcpyAsync(axis, ax.data(), ax.size() * sizeof(int), cudaMemcpyHostToDevice, st0));
+    OP_CK(cudaMemcpyAsync(off, of.data(), of.size() * sizeof(int), cudaMemcpyHostToDevice, st0));
+    OP_CK(rope_table(head_dim, (double)rope_theta, chunk * frames, make_int4(n_cams, frames, gh, gw), cs, n_entries,
+                     st0));
     const int npc = frames * gh * gw, M = n_cams * npc;
     EpiParams ep;
     memset(&ep, 0, sizeof ep);
@@ -1072,9 +1091,10 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
     ep.gw = gw;
     ep.frames = frames;
     ep.frame0 = chunk * frames;
-    ep.rope_freq = freq;
     ep.rope_axis = axis;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    ep.rope_off = off;
+    ep.rope_cs = cs;
+    cudaStream_t st = st0;
     if (dtype == XC_BF16) {
         if ((3 * d) % 256 != 0 || d % 64 != 0) OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: bf16 needs 3d %% 256, d %% 64");
         CUtensorMap ta, tb;

@@ -86,6 +86,14 @@ __device__ __forceinline__ float gelu_tanh(float x) {
     const float k0 = 0.7978845608028654f;   // sqrt(2/pi)
     return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
 }
+__device__ __forceinline__ float gelu_tanh_approx(float x) {
+    const float k0 = 0.7978845608028654f;
+    const float u = k0 * fmaf(0.044715f * x, x * x, x);
+    float t;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(u));
+    const float hx = 0.5f * x;
+    return fmaf(hx, t, hx);
+}
 __device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
 
 // ------------------------------------------------------------ GEMM epilogue
@@ -103,8 +111,9 @@ struct EpiParams {
     void *rhat;                // [M][N]  residual cache slot or nullptr
     // RoPE geometry (QKV kind)
     int d, head_dim, npc, gh, gw, frames, frame0;
-    const float *rope_freq;    // [head_dim/2] rotation frequency of each pair
     const int *rope_axis;      // [head_dim/2] 0 camera, 1 frame, 2 h, 3 w
+    const int *rope_off;       // [head_dim/2] table entry of position 0 of each pair
+    const float2 *rope_cs;     // (cos, sin) table of this chunk (rope_table_kernel)
 };
 
 enum { EPI_BIAS = XC_EPI_BIAS, EPI_GELU = XC_EPI_GELU, EPI_RESID_GATE = XC_EPI_RESID_GATE,
@@ -119,8 +128,15 @@ __device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col,
     if constexpr (EPI == EPI_BIAS) {
         store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
     } else if constexpr (EPI == EPI_GELU) {
+        if constexpr (sizeof(T) == 2) {
+            // bf16 output: the hardware tanh (rel. error ~2^-11) is below the
+            // output rounding (2^-9)
 #pragma unroll
-        for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh(acc[i]);
+            for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh_approx(acc[i]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh(acc[i]);
+        }
         store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
     } else if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
         float r[16];
@@ -147,17 +163,15 @@ __device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col,
             const int f = rem / (p.gh * p.gw);
             const int hh = (rem / p.gw) % p.gh;
             const int ww = rem % p.gw;
-            const float pos[4] = {(float)cam, (float)(p.frame0 + f), (float)hh, (float)ww};
+            const int pos[4] = {cam, f, hh, ww};      // frame: index within the chunk
             const int pair0 = (c % p.head_dim) >> 1;
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int pr = pair0 + j;
-                const float ang = pos[p.rope_axis[pr]] * p.rope_freq[pr];
-                float sn, cs;
-                sincosf(ang, &sn, &cs);
+                const float2 t = p.rope_cs[p.rope_off[pr] + pos[p.rope_axis[pr]]];
                 const float x0 = acc[2 * j], x1 = acc[2 * j + 1];
-                acc[2 * j] = x0 * cs - x1 * sn;
-                acc[2 * j + 1] = x0 * sn + x1 * cs;
+                acc[2 * j] = x0 * t.x - x1 * t.y;
+                acc[2 * j + 1] = x0 * t.y + x1 * t.x;
             }
         }
         T *dst = reinterpret_cast<T *>(part == 0 ? p.out : (part == 1 ? p.out_k : p.out_v));
