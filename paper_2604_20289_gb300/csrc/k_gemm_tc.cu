@@ -2,16 +2,22 @@
 //
 //   C[M][N] = epilogue(A[M][K] @ Wt[N][K]^T), fp32 accumulation in TMEM.
 //
-// One CTA computes a 128 x BN tile.  Warp roles (320 threads):
+// Persistent: one CTA per SM walks the 128 x BN output tiles round-robin
+// (n fastest, so the CTAs running at the same time share A tiles in L2).
+// Warp roles (320 threads):
 //   warp 0, lane 0 : TMA producer, STAGES-deep ring of (A 128x64, B BNx64)
-//                    tiles in 128B-swizzled shared memory;
-//   warp 1         : allocates TMEM; lane 0 issues tcgen05.mma (M=128, N=BN,
-//                    K=16 per instruction, 4 per 64-wide k-tile) and commits
-//                    each stage back to the producer;
+//                    tiles in 128B-swizzled shared memory, continuous across
+//                    output tiles;
+//   warp 1         : allocates TMEM (two BN-column accumulators); lane 0
+//                    issues tcgen05.mma (M=128, N=BN, K=16; 4 per 64-wide
+//                    k-tile) into the free accumulator and commits each stage
+//                    back to the producer;
 //   warps 2..9     : epilogue -- tcgen05.ld of their 32-lane TMEM quadrant
 //                    (two warps per quadrant, half of the columns each),
 //                    fused bias / GELU / gated residual / residual-cache /
-//                    RoPE, vectorised stores.
+//                    RoPE, vectorised stores; then they release the
+//                    accumulator, so the epilogue of tile i overlaps the
+//                    main loop of tile i + 1.
 // The skip flag of the block lets the whole recompute path early-exit when
 // the gate chose reuse (Eq. 4), so decisions never return to the host.
 #include "xc_ptx.cuh"
@@ -29,7 +35,8 @@ struct GemmTile {
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int BAR_OFFSET = STAGES * STAGE_BYTES;
     static constexpr int SMEM_BYTES = BAR_OFFSET + 256 + 1024;   // barriers + alignment slack
-    static constexpr int TMEM_COLS = BN;
+    static constexpr int TMEM_COLS = 2 * BN;                      // double-buffered accumulator
+    static constexpr int EPI_THREADS = 256;
 };
 
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
@@ -47,19 +54,24 @@ __global__ void __launch_bounds__(320, 1)
     uint8_t *smem = align1024(smem_raw);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + G::BAR_OFFSET);
     uint64_t *empty = full + G::STAGES;
-    uint64_t *done = empty + G::STAGES;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    uint64_t *acc_full = empty + G::STAGES;    // [2]
+    uint64_t *acc_empty = acc_full + 2;        // [2]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * GEMM_BM;
     const int KT = K / GEMM_BK;
+    const int tiles_n = ep.N / BN;
+    const int n_tiles = ((ep.M + GEMM_BM - 1) / GEMM_BM) * tiles_n;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < G::STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(done, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], G::EPI_THREADS);
+        }
         mbar_fence_init();
     }
     if (warp == 1) tmem_alloc(tmem_slot, G::TMEM_COLS);
@@ -70,55 +82,79 @@ __global__ void __launch_bounds__(320, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            int issued = 0;
-            for (int kt = 0; kt < KT; ++kt) {
-                const int s = kt % G::STAGES;
-                const uint32_t ph = (kt / G::STAGES) & 1;
-                if (!mbar_wait(&empty[s], ph ^ 1, err, ERR_WAIT_PRODUCER)) break;
-                uint8_t *sa = smem + s * G::STAGE_BYTES;
-                mbar_expect_tx(&full[s], G::STAGE_BYTES);
-                tma_load_2d(sa, &tmA, &full[s], kt * GEMM_BK, m0);
-                tma_load_2d(sa + G::A_BYTES, &tmB, &full[s], kt * GEMM_BK, n0);
-                issued = kt + 1;
+            int it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x) {
+                const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
+                for (int kt = 0; kt < KT; ++kt, ++it) {
+                    const int s = it % G::STAGES;
+                    const uint32_t ph = (it / G::STAGES) & 1;
+                    if (!mbar_wait(&empty[s], ph ^ 1, err, ERR_WAIT_PRODUCER)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t *sa = smem + s * G::STAGE_BYTES;
+                    mbar_expect_tx(&full[s], G::STAGE_BYTES);
+                    tma_load_2d(sa, &tmA, &full[s], kt * GEMM_BK, m0);
+                    tma_load_2d(sa + G::A_BYTES, &tmB, &full[s], kt * GEMM_BK, n0);
+                }
             }
             // Drain: every copy this thread started has landed before exit.
-            for (int kt = issued - G::STAGES < 0 ? 0 : issued - G::STAGES; kt < issued; ++kt)
-                mbar_wait(&full[kt % G::STAGES], (kt / G::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+            for (int j = it - G::STAGES < 0 ? 0 : it - G::STAGES; j < it; ++j)
+                mbar_wait(&full[j % G::STAGES], (j / G::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(GEMM_BM, BN, false, false);
-            for (int kt = 0; kt < KT; ++kt) {
-                const int s = kt % G::STAGES;
-                const uint32_t ph = (kt / G::STAGES) & 1;
-                if (!mbar_wait(&full[s], ph, err, ERR_WAIT_MMA)) break;
+            int it = 0, local = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++local) {
+                const int buf = local & 1;
+                const uint32_t use = (uint32_t)(local >> 1);
+                if (!mbar_wait(&acc_empty[buf], (use & 1) ^ 1, err, ERR_WAIT_MMA)) break;
                 tc_fence_after();
-                const uint32_t a = smem_u32(smem + s * G::STAGE_BYTES);
-                const uint32_t b = a + G::A_BYTES;
+                const uint32_t acc = tmem + buf * BN;
+                for (int kt = 0; kt < KT; ++kt, ++it) {
+                    const int s = it % G::STAGES;
+                    if (!mbar_wait(&full[s], (it / G::STAGES) & 1, err, ERR_WAIT_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a = smem_u32(smem + s * G::STAGE_BYTES);
+                    const uint32_t b = a + G::A_BYTES;
 #pragma unroll
-                for (int k = 0; k < GEMM_BK / 16; ++k) {
-                    tc_mma(tmem, sdesc_sw128(a + 32 * k, 16, 1024), sdesc_sw128(b + 32 * k, 16, 1024), idesc,
-                           (kt | k) != 0 ? 1u : 0u);
+                    for (int k = 0; k < GEMM_BK / 16; ++k)
+                        tc_mma(acc, sdesc_sw128(a + 32 * k, 16, 1024), sdesc_sw128(b + 32 * k, 16, 1024), idesc,
+                               (kt | k) != 0 ? 1u : 0u);
+                    tc_commit(&empty[s]);
                 }
-                tc_commit(&empty[s]);
+                tc_commit(&acc_full[buf]);
             }
-            tc_commit(done);
         }
     } else {
         // warps 2..9: two warps per TMEM lane quadrant, each half of the columns
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
         const int half = (warp - 2) >> 2;
-        const bool ok = mbar_wait(done, 0, err, ERR_WAIT_EPI);
-        tc_fence_after();
-        if (ok) {
+        const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
+        int local = 0;
+        for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++local) {
+            const int buf = local & 1;
+            const uint32_t use = (uint32_t)(local >> 1);
+            const bool ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
+            __syncwarp();
+            if (!__all_sync(0xffffffffu, ok)) break;
+            tc_fence_after();
+            const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
             const int row = m0 + q * 32 + lane;
-            const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
             for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
                 float v[16];
-                tmem_ld16_sync(tq + c, v);
+                tmem_ld16_sync(tq + buf * BN + c, v);
                 epilogue16<EPI, T>(ep, row, n0 + c, v);
             }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
         }
     }
     tc_fence_before();
@@ -170,12 +206,18 @@ static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const
     using G = GemmTile<BN>;
     auto kern = gemm_tc_kernel<BN, EPI, bf16>;
     static bool attr_set = false;
+    static int n_sm = 0;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM_BYTES);
         if (e != cudaSuccess) return e;
+        int dev = 0;
+        e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    dim3 grid(ep.N / BN, (ep.M + GEMM_BM - 1) / GEMM_BM);
+    const int n_tiles = (ep.N / BN) * ((ep.M + GEMM_BM - 1) / GEMM_BM);
+    const int grid = n_tiles < n_sm ? n_tiles : n_sm;
     kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
     return cudaGetLastError();
 }

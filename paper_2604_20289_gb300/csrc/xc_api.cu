@@ -138,10 +138,9 @@ struct xc_ctx {
     int *d_err;
 
     // gate scratch
-    int g_ns, g_R;
-    float *g_colsum;
-    double *g_sp, *g_gl;
-    unsigned *g_cnt;
+    int g_ns;
+    size_t g_ticket_off;
+    char *g_scratch;
 
     // tensor maps (bf16)
     CUtensorMap tm_h, tm_o, tm_u, tm_q;
@@ -278,7 +277,7 @@ void clear_state(xc_ctx *ctx) {
     CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
     if (ctx->phi != nullptr)
         CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * ctx->phi_n_all * sizeof(float), ctx->st));
-    CK(cudaMemsetAsync(ctx->g_cnt, 0, (size_t)(ctx->V * ctx->g_ns + 1) * sizeof(unsigned), ctx->st));
+    CK(cudaMemsetAsync(ctx->g_scratch + ctx->g_ticket_off, 0, sizeof(unsigned), ctx->st));
     CK(cudaStreamSynchronize(ctx->st));
     ctx->n = 0;
     ctx->next_step = 0;
@@ -398,7 +397,6 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.fp_rows = ctx->fp_rows;
             g.kfp = ctx->kfp;
             g.n_slices = ctx->g_ns;
-            g.R = ctx->g_R;
             const size_t cell = (size_t)t * B + b;
             g.phi = ctx->phi + cell * 2 * ctx->phi_n_all;
             g.phi_act = ctx->phi_act + cell * 16;
@@ -420,11 +418,8 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.s_cos = ctx->s_cos + b;
             g.d_max = ctx->d_max + b;
             g.tau_out = ctx->tau + b;
-            g.colsum = ctx->g_colsum;
-            g.sp_part = ctx->g_sp;
-            g.gl_part = ctx->g_gl;
-            g.cnt_cs = ctx->g_cnt;
-            g.cnt_all = ctx->g_cnt + ctx->V * ctx->g_ns;
+            g.part = reinterpret_cast<double *>(ctx->g_scratch);
+            g.ticket = reinterpret_cast<unsigned *>(ctx->g_scratch + ctx->g_ticket_off);
             LAUNCH(XC_K_GATE, b, 1, gate_launch<T>(g, st));
         }
 
@@ -705,11 +700,7 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         CK(cudaMallocHost(reinterpret_cast<void **>(&ctx->h_stats), 3 * XC_MAX_BLOCKS * sizeof(float)));
 
         // gate scratch
-        gate_geometry(ctx->V, ctx->npc, d, ctx->n_sm, &ctx->g_ns, &ctx->g_R);
-        ctx->g_colsum = dalloc<float>(ctx, (size_t)ctx->V * ctx->g_R * d * sizeof(float));
-        ctx->g_sp = dalloc<double>(ctx, (size_t)ctx->V * ctx->g_ns * ctx->g_R * 5 * sizeof(double));
-        ctx->g_gl = dalloc<double>(ctx, (size_t)ctx->V * ctx->g_ns * 3 * sizeof(double));
-        ctx->g_cnt = dalloc<unsigned>(ctx, (size_t)(ctx->V * ctx->g_ns + 1) * sizeof(unsigned));
+        ctx->g_scratch = dalloc<char>(ctx, gate_scratch(ctx->V, d, &ctx->g_ns, &ctx->g_ticket_off));
 
         // tensor maps of the bf16 path
         if (ctx->bf) {
@@ -1150,30 +1141,15 @@ xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x, const 
     return XC_OK;
 }
 
-// Workspace of one gate launch: column sums [V][R][d] f32, spatial partials
-// [V*ns*R][5] f64, global partials [V*ns][3] f64, tickets [V*ns + 1] u32.
+// Workspace of one gate launch: fp64 partials per CTA, then the ticket.
 struct GateWorkspace {
-    int ns, R;
-    size_t colsum, sp, gl, cnt, cnt_bytes, total;
+    int ns;
+    size_t ticket, total;
 };
 static GateWorkspace gate_workspace(int V, int npc, int d) {
-    int dev = 0, n_sm = 152;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    (void)npc;
     GateWorkspace w;
-    gate_geometry(V, npc, d, n_sm, &w.ns, &w.R);
-    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
-    size_t off = 0;
-    w.colsum = off;
-    off = al(off + (size_t)V * w.R * d * sizeof(float));
-    w.sp = off;
-    off = al(off + (size_t)V * w.ns * w.R * 5 * sizeof(double));
-    w.gl = off;
-    off = al(off + (size_t)V * w.ns * 3 * sizeof(double));
-    w.cnt = off;
-    w.cnt_bytes = (size_t)(V * w.ns + 1) * sizeof(unsigned);
-    off = al(off + w.cnt_bytes);
-    w.total = off;
+    w.total = gate_scratch(V, d, &w.ns, &w.ticket);
     return w;
 }
 
@@ -1210,7 +1186,7 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
         OP_FAIL(XC_EINVAL, "xc_op_gate: workspace %zu bytes < %zu needed", workspace_bytes, ws.total);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     char *w = reinterpret_cast<char *>(workspace);
-    OP_CK(cudaMemsetAsync(w + ws.cnt, 0, ws.cnt_bytes, st));
+    OP_CK(cudaMemsetAsync(w + ws.ticket, 0, sizeof(unsigned), st));
     GateArgs g;
     memset(&g, 0, sizeof g);
     g.x = x;
@@ -1220,7 +1196,6 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
     g.fp_rows = fp_rows;
     g.kfp = kfp;
     g.n_slices = ws.ns;
-    g.R = ws.R;
     g.phi = phi;
     g.phi_act = phi_act;
     for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
@@ -1241,11 +1216,8 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
     g.s_cos = s_cos;
     g.d_max = d_max;
     g.tau_out = tau;
-    g.colsum = reinterpret_cast<float *>(w + ws.colsum);
-    g.sp_part = reinterpret_cast<double *>(w + ws.sp);
-    g.gl_part = reinterpret_cast<double *>(w + ws.gl);
-    g.cnt_cs = reinterpret_cast<unsigned *>(w + ws.cnt);
-    g.cnt_all = g.cnt_cs + n_cams * ws.ns;
+    g.part = reinterpret_cast<double *>(w);
+    g.ticket = reinterpret_cast<unsigned *>(w + ws.ticket);
     if (dtype == XC_BF16)
         OP_CK(gate_launch<bf16>(g, st));
     else

@@ -17,7 +17,7 @@ struct GateArgs {
     int d, V, npc;
     const int *fp_rows;
     int kfp;
-    int n_slices, R;
+    int n_slices;            // 64-column slices: one CTA per (camera, slice)
     float *phi;
     float *phi_act;
     float action[8];
@@ -29,13 +29,11 @@ struct GateArgs {
     int max_skips, fp_refresh, replay;
     uint8_t *flag;
     float *s_cos, *d_max, *tau_out;
-    float *colsum;
-    double *sp_part;
-    double *gl_part;
-    unsigned *cnt_cs;
-    unsigned *cnt_all;
+    double *part;            // scratch [V * n_slices][8]
+    unsigned *ticket;        // scratch, zero before the launch (left zero)
 };
-void gate_geometry(int V, int npc, int d, int n_sm, int *n_slices, int *R);
+// Bytes of scratch of one gate launch (partials, then the ticket at *ticket_off).
+size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off);
 template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);
 bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,

@@ -103,8 +103,8 @@ def test_static_scratch_gate_rejects_geometry_beyond_its_maximum():
     buf = torch.zeros(1024, dtype=torch.uint8, device=DEV)
     p = buf.data_ptr()
     act = np.zeros(2, np.float32)
-    # 64 cameras x d 8192 needs 64 * 8192 * 4 bytes = 2 MiB of column sums alone
-    st = xb.LIB.xc_op_gate_static(xb.XC_BF16, 64, 8, 8192, p, p, 1, p, p, p, act.ctypes.data, 2, 1, 1,
+    # 64 cameras x d 32768 = 64 x 512 column-slice CTAs x 64 bytes of partials = 2 MiB
+    st = xb.LIB.xc_op_gate_static(xb.XC_BF16, 64, 8, 32768, p, p, 1, p, p, p, act.ctypes.data, 2, 1, 1,
                                   None, p, p, p, p, None)
     assert st == xb.XC_EINVAL
     assert "static maximum" in xb.last_error(None)
