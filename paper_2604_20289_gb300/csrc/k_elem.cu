@@ -295,14 +295,18 @@ cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, i
 
 // ------------------------------------------------------------------- head
 // One warp per row, row in registers: hf = round(LN(x) (1 + scale) + shift);
-// v = hf W_out + b_out (16 output channels, float32 out).  Each lane forms the
-// 16 partial dot products of its runs (float4 reads of W_out), then the warp
-// reduces them.
+// v = hf W_out + b_out (16 output channels, float32 out).  The normalised row
+// goes through shared memory in 512-element pieces; lane l then owns outputs
+// 4 (l % 4) .. +3 for rows i = l / 4 (mod 8) of the piece, so one float4 load
+// instruction of the warp reads 8 consecutive rows of W_out (512 contiguous
+// bytes); three shuffle levels fold the 8 row groups.
 template <typename T, int NCH>
 __global__ void __launch_bounds__(256)
     head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
                 const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
-    const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    __shared__ float hrow[8][512];
+    const int wib = threadIdx.x >> 5;
+    const int row = blockIdx.x * 8 + wib;
     const int lane = threadIdx.x & 31;
     if (row >= L) return;
     const T *xr = x + (size_t)row * d;
@@ -315,38 +319,46 @@ __global__ void __launch_bounds__(256)
     const Moments mo = warp_moments(lane_moments<NCH>(val, mine));
     const float rstd = rsqrtf(mo.m2 / (float)d + eps);
     const float *shift = hm, *scale = hm + d;
-    float acc[16];
-#pragma unroll
-    for (int o = 0; o < 16; ++o) acc[o] = 0.0f;
+    const int grp = lane >> 2, oq = lane & 3;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int k = 0; k < NCH; ++k) {
+        if (32 * k * 16 >= d) break;                       // warp-uniform
         if (k < mine) {
             const int c = 16 * (lane + 32 * k);
             float sc[16], sh[16];
             load16<float>(scale + c, sc);
             load16<float>(shift + c, sh);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const float hv = round_to<T>((val[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i]);
-                float wr[16];
-                load16<float>(w + (size_t)(c + i) * 16, wr);
-#pragma unroll
-                for (int o = 0; o < 16; ++o) acc[o] = fmaf(hv, wr[o], acc[o]);
-            }
+            for (int i = 0; i < 16; ++i)
+                hrow[wib][16 * lane + i] = round_to<T>((val[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i]);
         }
+        __syncwarp();
+        const int c0 = 512 * k;
+        const int n_here = d - c0 < 512 ? d - c0 : 512;
+        const float4 *w4 = reinterpret_cast<const float4 *>(w + (size_t)c0 * 16) + oq;
+#pragma unroll 4
+        for (int i = grp; i < n_here; i += 8) {
+            const float hv = hrow[wib][i];
+            const float4 t = w4[(size_t)i * 4];
+            acc.x = fmaf(hv, t.x, acc.x);
+            acc.y = fmaf(hv, t.y, acc.y);
+            acc.z = fmaf(hv, t.z, acc.z);
+            acc.w = fmaf(hv, t.w, acc.w);
+        }
+        __syncwarp();
     }
 #pragma unroll
-    for (int o = 0; o < 16; ++o) {
-#pragma unroll
-        for (int s = 16; s > 0; s >>= 1) acc[o] += __shfl_xor_sync(0xffffffffu, acc[o], s);
+    for (int s = 4; s < 32; s <<= 1) {
+        acc.x += __shfl_xor_sync(0xffffffffu, acc.x, s);
+        acc.y += __shfl_xor_sync(0xffffffffu, acc.y, s);
+        acc.z += __shfl_xor_sync(0xffffffffu, acc.z, s);
+        acc.w += __shfl_xor_sync(0xffffffffu, acc.w, s);
     }
     if (lane < 4) {
-        float4 r;
-        r.x = acc[4 * lane] + b[4 * lane];
-        r.y = acc[4 * lane + 1] + b[4 * lane + 1];
-        r.z = acc[4 * lane + 2] + b[4 * lane + 2];
-        r.w = acc[4 * lane + 3] + b[4 * lane + 3];
-        reinterpret_cast<float4 *>(v + (size_t)row * 16)[lane] = r;
+        const float4 bb = reinterpret_cast<const float4 *>(b)[lane];
+        reinterpret_cast<float4 *>(v + (size_t)row * 16)[lane] =
+            make_float4(acc.x + bb.x, acc.y + bb.y, acc.z + bb.z, acc.w + bb.w);
     }
 }
 
