@@ -14,10 +14,10 @@
 // Grid: one CTA (512 threads) per (camera c, 64-column slice s).  The CTA
 // streams all of camera c's rows of its slice once (16-byte loads, 8 rows in
 // flight per thread), so it completes that slice's per-camera means by
-// itself; it also takes the slice of the spatial sample.  Per-thread and
-// per-warp reductions run in fp32; each CTA writes 8 partials (fp64) and takes
-// an atomic ticket; the last CTA combines all partials in a fixed order (fp64)
-// and makes the decision.  No spin-wait anywhere; deterministic.  The cached
+// itself; it also takes the slice of the spatial sample.  All reductions run
+// in fp32; each CTA writes 8 partials and takes an atomic ticket; the last
+// CTA combines all partials in a fixed order and makes the decision (the EMA
+// state is kept in fp64).  No spin-wait anywhere; deterministic.  The cached
 // fingerprint is double-buffered per (t, b): the current fingerprint goes to
 // the inactive half, which becomes active when the block recomputes.
 #include <cmath>
@@ -36,11 +36,11 @@ constexpr int GATE_PARTS = 8;        // dot, |cur|^2, |prev|^2, max|diff|, sum|p
 
 // Cosine of one entry from its dot product and squared norms (Eq. 5):
 // both norms < 1e-12 -> 1, exactly one -> 0, NaN -> 0.
-__device__ __forceinline__ double cos_rule(double dot, double n1sq, double n2sq) {
-    const double a = sqrt(n1sq), b = sqrt(n2sq);
-    if (isnan(a) || isnan(b) || isnan(dot)) return 0.0;
-    if (a < 1e-12 && b < 1e-12) return 1.0;
-    if (a < 1e-12 || b < 1e-12) return 0.0;
+__device__ __forceinline__ float cos_rule_f(float dot, float n1sq, float n2sq) {
+    const float a = sqrtf(n1sq), b = sqrtf(n2sq);
+    if (isnan(a) || isnan(b) || isnan(dot)) return 0.0f;
+    if (a < 1e-12f && b < 1e-12f) return 1.0f;
+    if (a < 1e-12f || b < 1e-12f) return 0.0f;
     return dot / (a * b);
 }
 
@@ -70,7 +70,6 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     constexpr int NW = GATE_THREADS / 32;
     __shared__ float red[RPAR * GATE_CW];
     __shared__ float wpart[NW][GATE_PARTS];
-    __shared__ double dpart[NW][GATE_PARTS];
     __shared__ int s_last;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -92,16 +91,16 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     {
         const int ty = tid / TPR, tx = tid % TPR;
         const T *base = x + (size_t)c * npc * d + col0 + tx * VEC;
-        int r = ty;
-        for (; r + (GATE_UNROLL - 1) * RPAR < npc; r += GATE_UNROLL * RPAR) {
+        // GATE_UNROLL guarded loads in flight per step, the ragged end included
+        for (int r = ty; r < npc; r += GATE_UNROLL * RPAR) {
             uint4 u[GATE_UNROLL];
 #pragma unroll
             for (int k = 0; k < GATE_UNROLL; ++k)
-                u[k] = *reinterpret_cast<const uint4 *>(base + (size_t)(r + k * RPAR) * d);
+                u[k] = r + k * RPAR < npc ? *reinterpret_cast<const uint4 *>(base + (size_t)(r + k * RPAR) * d)
+                                          : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
             for (int k = 0; k < GATE_UNROLL; ++k) add_vec16<T>(acc, u[k]);
         }
-        for (; r < npc; r += RPAR) add_vec16<T>(acc, *reinterpret_cast<const uint4 *>(base + (size_t)r * d));
 #pragma unroll
         for (int i = 0; i < VEC; ++i) red[ty * GATE_CW + tx * VEC + i] = acc[i];
     }
@@ -134,7 +133,7 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         p[3] = fmaxf(p[3], fabsf(cur - prev));
         p[4] += fabsf(prev);
     }
-    // CTA reduction: fp32 within warps, fp64 across warps in a fixed order
+    // CTA reduction: within warps, then across warps in a fixed order
 #pragma unroll
     for (int k = 0; k < GATE_PARTS; ++k) {
         float v = p[k];
@@ -147,8 +146,8 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     }
     __syncthreads();
     if (tid < GATE_PARTS) {
-        double v = 0.0;
-        for (int w = 0; w < NW; ++w) v = tid == 3 ? fmax(v, (double)wpart[w][tid]) : v + (double)wpart[w][tid];
+        float v = 0.0f;
+        for (int w = 0; w < NW; ++w) v = tid == 3 ? fmaxf(v, wpart[w][tid]) : v + wpart[w][tid];
         g.part[(size_t)blk * GATE_PARTS + tid] = v;
     }
 
@@ -159,46 +158,49 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    double v[GATE_PARTS] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+    float v[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     for (int b = tid; b < (int)gridDim.x; b += GATE_THREADS) {
 #pragma unroll
         for (int k = 0; k < GATE_PARTS; ++k) {
-            const double q = __ldcg(&g.part[(size_t)b * GATE_PARTS + k]);
-            v[k] = k == 3 ? fmax(v[k], q) : v[k] + q;
+            const float q = __ldcg(&g.part[(size_t)b * GATE_PARTS + k]);
+            v[k] = k == 3 ? fmaxf(v[k], q) : v[k] + q;
         }
     }
 #pragma unroll
     for (int k = 0; k < GATE_PARTS; ++k) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
-            const double w = __shfl_xor_sync(0xffffffffu, v[k], o);
-            v[k] = k == 3 ? fmax(v[k], w) : v[k] + w;
+            const float w = __shfl_xor_sync(0xffffffffu, v[k], o);
+            v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
         }
-        if (lane == 0) dpart[warp][k] = v[k];
+        if (lane == 0) wpart[warp][k] = v[k];
     }
     __syncthreads();
     if (tid != 0) return;
     for (int k = 0; k < GATE_PARTS; ++k) {
-        double a = dpart[0][k];
-        for (int w = 1; w < NW; ++w) a = k == 3 ? fmax(a, dpart[w][k]) : a + dpart[w][k];
+        float a = wpart[0][k];
+        for (int w = 1; w < NW; ++w) a = k == 3 ? fmaxf(a, wpart[w][k]) : a + wpart[w][k];
         v[k] = a;
     }
     *g.ticket = 0;
 
-    double da = 0.0, na = 0.0, nb = 0.0;
+    // All sums and metrics are fp32 (relative error ~1e-7, far inside the
+    // 1e-3 band around a threshold): FP64 arithmetic, square roots and divides
+    // are slow on this part; only the EMA state stays fp64.
+    float da = 0.0f, na = 0.0f, nb = 0.0f;
     for (int i = 0; i < g.A; ++i) {
-        const double a = (double)g.action[i];
-        const double b = (double)g.phi_act[active * 8 + i];
-        da += a * b;
-        na += a * a;
-        nb += b * b;
+        const float a = g.action[i];
+        const float b = g.phi_act[active * 8 + i];
+        da = fmaf(a, b, da);
+        na = fmaf(a, a, na);
+        nb = fmaf(b, b, nb);
         g.phi_act[(active ^ 1) * 8 + i] = g.action[i];
     }
-    const double cos_sp = cos_rule(v[0], v[1], v[2]);
-    const double cos_gl = cos_rule(v[5], v[6], v[7]);
-    const double cos_a = cos_rule(da, na, nb);
-    const double s_min = fmin(fmin(cos_sp, cos_gl), cos_a);
-    double dmax = v[3] / (v[4] / (double)n_sp + (double)g.eps_dev);
+    const float cos_sp = cos_rule_f(v[0], v[1], v[2]);
+    const float cos_gl = cos_rule_f(v[5], v[6], v[7]);
+    const float cos_a = cos_rule_f(da, na, nb);
+    const double s_min = (double)fminf(fminf(cos_sp, cos_gl), cos_a);
+    float dmax = v[3] / (v[4] / (float)n_sp + g.eps_dev);
     if (isnan(dmax)) dmax = INFINITY;
 
     GateCell cell = *g.cell;
@@ -207,7 +209,7 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     if (g.mode == 1 && cell.valid) {
         double tau = cell.has_hist ? fmax((double)g.tau_floor, cell.ema - (double)g.margin) : (double)g.tau_floor;
         if (g.strict_tau > 0.0f && g.step == 0) tau = fmax(tau, (double)g.strict_tau);
-        bool skip = (s_min >= tau) && (dmax < (double)g.tau_dev);
+        bool skip = (s_min >= tau) && (dmax < g.tau_dev);
         if (g.max_skips > 0 && cell.stale >= g.max_skips) skip = false;
         if (g.replay >= 0) skip = g.replay != 0;
         cell.ema = cell.has_hist ? (double)g.alpha * s_min + (1.0 - (double)g.alpha) * cell.ema : s_min;
@@ -228,12 +230,12 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     *g.flag = dec;
 }
 
-// Scratch of one gate launch: GATE_PARTS fp64 partials per CTA, then one
+// Scratch of one gate launch: GATE_PARTS fp32 partials per CTA, then one
 // 32-bit ticket (which must be zero before the launch; the kernel leaves it
 // zero).  Returns the total bytes; *ticket_off receives the ticket's offset.
 size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off) {
     *n_slices = d / GATE_CW;
-    const size_t part = (size_t)V * *n_slices * GATE_PARTS * sizeof(double);
+    const size_t part = (size_t)V * *n_slices * GATE_PARTS * sizeof(float);
     *ticket_off = (part + 255) & ~(size_t)255;
     return *ticket_off + 256;
 }
@@ -360,7 +362,7 @@ extern "C" xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam
     g.s_cos = s_cos;
     g.d_max = d_max;
     g.tau_out = tau;
-    g.part = reinterpret_cast<double *>(w);
+    g.part = reinterpret_cast<float *>(w);
     g.ticket = reinterpret_cast<unsigned *>(w + ticket_off);
     const cudaError_t e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, st) : xc::gate_launch<float>(g, st);
     if (e != cudaSuccess) return fail(XC_ECUDA, cudaGetErrorString(e));

@@ -418,7 +418,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.s_cos = ctx->s_cos + b;
             g.d_max = ctx->d_max + b;
             g.tau_out = ctx->tau + b;
-            g.part = reinterpret_cast<double *>(ctx->g_scratch);
+            g.part = reinterpret_cast<float *>(ctx->g_scratch);
             g.ticket = reinterpret_cast<unsigned *>(ctx->g_scratch + ctx->g_ticket_off);
             LAUNCH(XC_K_GATE, b, 1, gate_launch<T>(g, st));
         }
@@ -1141,7 +1141,7 @@ xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x, const 
     return XC_OK;
 }
 
-// Workspace of one gate launch: fp64 partials per CTA, then the ticket.
+// Workspace of one gate launch: fp32 partials per CTA, then the ticket.
 struct GateWorkspace {
     int ns;
     size_t ticket, total;
@@ -1216,7 +1216,7 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
     g.s_cos = s_cos;
     g.d_max = d_max;
     g.tau_out = tau;
-    g.part = reinterpret_cast<double *>(w);
+    g.part = reinterpret_cast<float *>(w);
     g.ticket = reinterpret_cast<unsigned *>(w + ws.ticket);
     if (dtype == XC_BF16)
         OP_CK(gate_launch<bf16>(g, st));

@@ -29,7 +29,7 @@ struct GateArgs {
     int max_skips, fp_refresh, replay;
     uint8_t *flag;
     float *s_cos, *d_max, *tau_out;
-    double *part;            // scratch [V * n_slices][8]
+    float *part;             // scratch [V * n_slices][8]
     unsigned *ticket;        // scratch, zero before the launch (left zero)
 };
 // Bytes of scratch of one gate launch (partials, then the ticket at *ticket_off).
