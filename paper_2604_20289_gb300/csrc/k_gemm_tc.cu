@@ -33,7 +33,9 @@ struct GemmTile {
     static constexpr int A_BYTES = GEMM_BM * GEMM_BK * 2;
     static constexpr int B_BYTES = BN * GEMM_BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int BAR_OFFSET = STAGES * STAGE_BYTES;
+    static constexpr int STAGE_EPI = STAGES * STAGE_BYTES;       // 8 warps x [32 rows][32 fp32]
+    static constexpr int EPI_BYTES = 8 * 32 * 32 * 4;
+    static constexpr int BAR_OFFSET = STAGE_EPI + EPI_BYTES;
     static constexpr int SMEM_BYTES = BAR_OFFSET + 256 + 1024;   // barriers + alignment slack
     static constexpr int TMEM_COLS = 2 * BN;                      // double-buffered accumulator
     static constexpr int EPI_THREADS = 256;
@@ -133,10 +135,14 @@ __global__ void __launch_bounds__(320, 1)
             }
         }
     } else {
-        // warps 2..9: two warps per TMEM lane quadrant, each half of the columns
+        // warps 2..9: two warps per TMEM lane quadrant, each half of the columns.
+        // Each 32-row x 32-column block goes TMEM -> registers (thread = row) ->
+        // XOR-swizzled shared memory -> registers (4 lanes per row, 8 columns
+        // each), so the epilogue's global loads and stores are row-contiguous.
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
         const int half = (warp - 2) >> 2;
         const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
+        float *stg = reinterpret_cast<float *>(smem + G::STAGE_EPI) + (warp - 2) * 32 * 32;
         int local = 0;
         for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++local) {
             const int buf = local & 1;
@@ -146,12 +152,26 @@ __global__ void __launch_bounds__(320, 1)
             if (!__all_sync(0xffffffffu, ok)) break;
             tc_fence_after();
             const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
-            const int row = m0 + q * 32 + lane;
 #pragma unroll 1
-            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
+            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
                 float v[16];
                 tmem_ld16_sync(tq + buf * BN + c, v);
-                epilogue16<EPI, T>(ep, row, n0 + c, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) stg[lane * 32 + (i ^ lane)] = v[i];
+                tmem_ld16_sync(tq + buf * BN + c + 16, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) stg[lane * 32 + ((16 + i) ^ lane)] = v[i];
+                __syncwarp();
+                const int c8 = (lane & 3) * 8;
+#pragma unroll
+                for (int it = 0; it < 4; ++it) {
+                    const int r = it * 8 + (lane >> 2);
+                    float a[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) a[k] = stg[r * 32 + ((c8 + k) ^ r)];
+                    epilogue_run<EPI, T, 8>(ep, m0 + q * 32 + r, n0 + c + c8, a);
+                }
+                __syncwarp();
             }
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);

@@ -119,43 +119,88 @@ struct EpiParams {
 enum { EPI_BIAS = XC_EPI_BIAS, EPI_GELU = XC_EPI_GELU, EPI_RESID_GATE = XC_EPI_RESID_GATE,
        EPI_RESID_CACHE = XC_EPI_RESID_CACHE, EPI_QKV_ROPE = 16 };
 
-template <int EPI, typename T>
-__device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col, float (&acc)[16]) {
-    if (row >= p.M) return;
+// Runs of W = 8 or 16 consecutive elements (16-byte aligned).
+template <typename T, int W>
+__device__ __forceinline__ void loadW(const T *p, float (&v)[W]) {
+    if constexpr (W == 16) {
+        load16<T>(p, v);
+    } else if constexpr (sizeof(T) == 2) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(p);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-    for (int i = 0; i < 16; ++i) acc[i] += p.bias[col + i];
+        for (int j = 0; j < 4; ++j) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
+            v[2 * j] = f.x;
+            v[2 * j + 1] = f.y;
+        }
+    } else {
+        const float4 a = reinterpret_cast<const float4 *>(p)[0], b = reinterpret_cast<const float4 *>(p)[1];
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+}
+template <typename T, int W>
+__device__ __forceinline__ void storeW(T *p, const float (&v)[W]) {
+    if constexpr (W == 16) {
+        store16<T>(p, v);
+    } else if constexpr (sizeof(T) == 2) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+            w[j] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+    } else {
+        reinterpret_cast<float4 *>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4 *>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
+// Fused GEMM epilogue on one run of W consecutive output columns
+// [col, col + W) of one row (W = 8 or 16, col a multiple of W).
+template <int EPI, typename T, int W>
+__device__ __forceinline__ void epilogue_run(const EpiParams &p, int row, int col, float (&acc)[W]) {
+    if (row >= p.M) return;
+    {
+        float b[W];
+        loadW<float, W>(p.bias + col, b);
+#pragma unroll
+        for (int i = 0; i < W; ++i) acc[i] += b[i];
+    }
     const size_t off = (size_t)row * p.N + col;
     if constexpr (EPI == EPI_BIAS) {
-        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+        storeW<T, W>(reinterpret_cast<T *>(p.out) + off, acc);
     } else if constexpr (EPI == EPI_GELU) {
         if constexpr (sizeof(T) == 2) {
             // bf16 output: the hardware tanh (rel. error ~2^-11) is below the
             // output rounding (2^-9)
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh_approx(acc[i]);
+            for (int i = 0; i < W; ++i) acc[i] = gelu_tanh_approx(acc[i]);
         } else {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = gelu_tanh(acc[i]);
+            for (int i = 0; i < W; ++i) acc[i] = gelu_tanh(acc[i]);
         }
-        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+        storeW<T, W>(reinterpret_cast<T *>(p.out) + off, acc);
     } else if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
-        float r[16];
-        load16<T>(reinterpret_cast<const T *>(p.resid) + off, r);
+        float r[W], g[W];
+        loadW<T, W>(reinterpret_cast<const T *>(p.resid) + off, r);
+        loadW<float, W>(p.gate + col, g);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) acc[i] = r[i] + p.gate[col + i] * acc[i];
-        store16<T>(reinterpret_cast<T *>(p.out) + off, acc);
+        for (int i = 0; i < W; ++i) acc[i] = r[i] + g[i] * acc[i];
+        storeW<T, W>(reinterpret_cast<T *>(p.out) + off, acc);
         if constexpr (EPI == EPI_RESID_CACHE) {
             if (p.rhat != nullptr) {
-                float xi[16];
-                load16<T>(reinterpret_cast<const T *>(p.xin) + off, xi);
+                float xi[W];
+                loadW<T, W>(reinterpret_cast<const T *>(p.xin) + off, xi);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = round_to<T>(acc[i]) - xi[i];
-                store16<T>(reinterpret_cast<T *>(p.rhat) + off, acc);
+                for (int i = 0; i < W; ++i) acc[i] = round_to<T>(acc[i]) - xi[i];
+                storeW<T, W>(reinterpret_cast<T *>(p.rhat) + off, acc);
             }
         }
     } else if constexpr (EPI == EPI_QKV_ROPE) {
         const int d = p.d;
-        const int part = col / d;          // 0 q, 1 k, 2 v (16-runs never straddle: d % 16 == 0)
+        const int part = col / d;          // 0 q, 1 k, 2 v (runs never straddle: d % 16 == 0)
         const int c = col - part * d;
         if (part < 2) {
             const int cam = row / p.npc;
@@ -166,7 +211,7 @@ __device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col,
             const int pos[4] = {cam, f, hh, ww};      // frame: index within the chunk
             const int pair0 = (c % p.head_dim) >> 1;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int j = 0; j < W / 2; ++j) {
                 const int pr = pair0 + j;
                 const float2 t = p.rope_cs[p.rope_off[pr] + pos[p.rope_axis[pr]]];
                 const float x0 = acc[2 * j], x1 = acc[2 * j + 1];
@@ -175,8 +220,12 @@ __device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col,
             }
         }
         T *dst = reinterpret_cast<T *>(part == 0 ? p.out : (part == 1 ? p.out_k : p.out_v));
-        store16<T>(dst + (size_t)row * d + c, acc);
+        storeW<T, W>(dst + (size_t)row * d + c, acc);
     }
+}
+template <int EPI, typename T>
+__device__ __forceinline__ void epilogue16(const EpiParams &p, int row, int col, float (&acc)[16]) {
+    epilogue_run<EPI, T, 16>(p, row, col, acc);
 }
 
 }  // namespace xc
