@@ -4,12 +4,14 @@
 //   the current chunk's queries see every resident key of the rolling KV
 //   cache (past chunks' clean K/V plus the current chunk's own K/V).
 //
-// One CTA = two 128-query tiles (Q0, Q1) of one head, 320 threads:
+// One CTA = two 128-query tiles (Q0, Q1) of one head, 352 threads:
 //   warps 0..3  softmax WG 0 (tile Q0), thread = query row = TMEM lane;
 //   warps 4..7  softmax WG 1 (tile Q1);
 //   warp 8      TMA producer: Q0/Q1 once, then 128-key K and V tiles through
 //               a STAGES-deep ring (separate K and V barriers);
-//   warp 9      TMEM allocation; lane 0 issues every MMA.
+//   warp 9      TMEM allocation; lane 0 issues the MMAs of tile Q0;
+//   warp 10     lane 0 issues the MMAs of tile Q1 (each tile advances on
+//               its own softmax's signals; K/V stages are freed by both).
 // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after it.  P (bf16)
 // goes back into TMEM and feeds tcgen05.mma as the A operand straight from
 // tensor memory (no shared-memory round trip); V is read MN-major from its
@@ -42,7 +44,7 @@ struct AttnTile {
     static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
     static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
     static constexpr int TMEM_COLS = 512;
-    static constexpr int THREADS = 320;
+    static constexpr int THREADS = 352;            // 8 softmax, 1 TMA, 2 MMA warps
     static constexpr bool SEP_P = HD == 64;            // P has its own TMEM columns
     __host__ __device__ static constexpr int S_COL(int i) { return 128 * i; }
     __host__ __device__ static constexpr int O_COL(int i) { return 256 + HD * i; }
@@ -55,6 +57,12 @@ __device__ __forceinline__ uint8_t *align1024_a(uint8_t *p) {
     return p + ((1024u - (s & 1023u)) & 1023u);
 }
 
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float y;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+    return y;
+}
+
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -62,7 +70,7 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 
 template <int HD>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(352, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
                    const int n_keys, const int d, const uint8_t *__restrict__ skip_flag, int *err) {
@@ -83,7 +91,8 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t *s_cons = s_full + 2;             // [2] S_i read by its softmax WG (hd 64)
     uint64_t *p_full = s_cons + 2;             // [2] P_i written, O_i corrected
     uint64_t *pv_done = p_full + 2;            // [2] P_i V done (hd 64: every tile; hd 128: last)
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(pv_done + 2);
+    uint64_t *turn = pv_done + 2;              // [2] exponential phase hand-off between the WGs
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * (A::QT * A::BQ);
@@ -94,15 +103,16 @@ __global__ void __launch_bounds__(320, 1)
         mbar_init(q_full, 1);
         for (int s = 0; s < A::STAGES; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 1);
+            mbar_init(&k_empty[s], 2);        // released by both MMA issuers
             mbar_init(&v_full[s], 1);
-            mbar_init(&v_empty[s], 1);
+            mbar_init(&v_empty[s], 2);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
             mbar_init(&s_cons[i], 128);
             mbar_init(&p_full[i], 128);
             mbar_init(&pv_done[i], 1);
+            mbar_init(&turn[i], 4);           // one arrive per warp of the other WG
         }
         mbar_fence_init();
     }
@@ -143,8 +153,8 @@ __global__ void __launch_bounds__(320, 1)
             for (int j = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; j < v_issued; ++j)
                 mbar_wait(&v_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
-    } else if (warp == 9) {
-        // ---------------------------------------------------------- MMA issue
+    } else if (warp >= 9) {
+        // ------------------------------------------ MMA issue (one warp per Q tile)
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);
             constexpr uint32_t idesc_o = idesc_bf16(128, HD, false, true);
@@ -167,11 +177,16 @@ __global__ void __launch_bounds__(320, 1)
                                   sdesc_sw128(aV + st * A::KV_BYTES + ks * 16 * 128, A::REGION, 1024), idesc_o,
                                   (j > 0 || ks > 0) ? 1u : 0u);
             };
+            // One issuing warp per Q tile, so that neither tile's MMAs wait
+            // on the other's softmax.  hd 64: S_i(j+1) goes as soon as the
+            // softmax has read S_i(j), ahead of P_i V_j.  hd 128: P_i aliases
+            // S_i, so S_i(j+1) follows P_i V_j.  K and V stages are released
+            // by both issuers (barrier count 2).
+            const int i = warp - 9;
             bool ok = mbar_wait(q_full, 0, err, ERR_WAIT_MMA) && mbar_wait(&k_full[0], 0, err, ERR_WAIT_MMA);
             if (ok) {
                 tc_fence_after();
-                issue_s(0, 0);
-                issue_s(1, 0);
+                issue_s(i, 0);
                 tc_commit(&k_empty[0]);
             }
             for (int j = 0; ok && j < nkt; ++j) {
@@ -179,45 +194,30 @@ __global__ void __launch_bounds__(320, 1)
                 const int st1 = (j + 1) % A::STAGES;
                 const bool more = j + 1 < nkt;
                 if constexpr (A::SEP_P) {
-                    // next scores as soon as the current ones have been read
                     if (more) {
+                        if (!mbar_wait(&s_cons[i], j & 1, err, ERR_WAIT_MMA)) break;
                         if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                        if (!mbar_wait(&s_cons[0], j & 1, err, ERR_WAIT_MMA)) break;
                         tc_fence_after();
-                        issue_s(0, j + 1);
-                        if (!mbar_wait(&s_cons[1], j & 1, err, ERR_WAIT_MMA)) break;
-                        tc_fence_after();
-                        issue_s(1, j + 1);
+                        issue_s(i, j + 1);
                         tc_commit(&k_empty[st1]);
                     }
+                    if (!mbar_wait(&p_full[i], j & 1, err, ERR_WAIT_MMA)) break;
                     if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                    if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
                     tc_fence_after();
-                    issue_pv(0, j);
-                    tc_commit(&pv_done[0]);
-                    if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
-                    issue_pv(1, j);
-                    tc_commit(&pv_done[1]);
+                    issue_pv(i, j);
+                    tc_commit(&pv_done[i]);
                     tc_commit(&v_empty[st]);
                 } else {
+                    if (!mbar_wait(&p_full[i], j & 1, err, ERR_WAIT_MMA)) break;
                     if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                    if (!mbar_wait(&p_full[0], j & 1, err, ERR_WAIT_MMA)) break;
                     tc_fence_after();
-                    issue_pv(0, j);
-                    if (!more) tc_commit(&pv_done[0]);
+                    issue_pv(i, j);
+                    tc_commit(&v_empty[st]);
+                    if (!more) tc_commit(&pv_done[i]);
                     if (more) {
                         if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
                         tc_fence_after();
-                        issue_s(0, j + 1);
-                    }
-                    if (!mbar_wait(&p_full[1], j & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
-                    issue_pv(1, j);
-                    tc_commit(&v_empty[st]);
-                    if (!more) tc_commit(&pv_done[1]);
-                    if (more) {
-                        issue_s(1, j + 1);
+                        issue_s(i, j + 1);
                         tc_commit(&k_empty[st1]);
                     }
                 }
@@ -252,15 +252,18 @@ __global__ void __launch_bounds__(320, 1)
                 for (int c = 0; c < 128; ++c)
                     if (c >= tail) s[c] = -INFINITY;
             }
-            float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+            // row max: 16 independent chains of three-input max, then a tree
+            float mx[16];
 #pragma unroll
-            for (int c = 4; c < 128; c += 4) {
-                mx0 = fmaxf(mx0, s[c]);
-                mx1 = fmaxf(mx1, s[c + 1]);
-                mx2 = fmaxf(mx2, s[c + 2]);
-                mx3 = fmaxf(mx3, s[c + 3]);
+            for (int k = 0; k < 16; ++k) mx[k] = s[k];
+#pragma unroll
+            for (int c = 16; c < 128; c += 32) {
+#pragma unroll
+                for (int k = 0; k < 16; ++k) mx[k] = fmax3(mx[k], s[c + k], s[c + 16 + k]);
             }
-            const float m_new = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+#pragma unroll
+            for (int k = 0; k < 5; ++k) mx[k] = fmax3(mx[k], mx[k + 5], mx[k + 10]);
+            const float m_new = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[15]), mx[0]) * sl2;
             const bool grow = j > 0 && m_new > m + A::LAZY;
             const float alpha = grow ? ex2_approx(m - m_new) : 1.0f;
             if (j == 0 || grow) m = m_new;
@@ -283,6 +286,15 @@ __global__ void __launch_bounds__(320, 1)
                     for (int i = 0; i < 16; ++i) t[i] *= alpha;
                     tmem_st16_sync(tO + 16 * c, t);
                 }
+            }
+            // The two WGs take turns on the exponential phase (MUFU bound):
+            // WG 0 does tile j, then WG 1 tile j, then WG 0 tile j + 1 ...
+            // so that one WG's exponentials overlap the other's loads, max
+            // and MMA waits instead of competing for the same units.
+            if (wg == 1 || j > 0) {
+                ok = mbar_wait(&turn[wg], (wg == 1 ? j : j - 1) & 1, err, ERR_WAIT_SOFTMAX);
+                __syncwarp();
+                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             }
             // probabilities p = 2^(s * sl2 - m), packed bf16 pairs + row sum,
             // stored to TMEM in two 64-key halves
@@ -311,6 +323,8 @@ __global__ void __launch_bounds__(320, 1)
             l = l * alpha + (rs.x + rs.y);
             tc_fence_before();
             mbar_arrive(&p_full[wg]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&turn[wg ^ 1]);
         }
         if (ok) ok = mbar_wait(&pv_done[wg], A::SEP_P ? ((nkt - 1) & 1) : 0, err, ERR_WAIT_SOFTMAX);
         __syncwarp();
