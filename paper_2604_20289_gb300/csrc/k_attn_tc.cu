@@ -4,14 +4,12 @@
 //   the current chunk's queries see every resident key of the rolling KV
 //   cache (past chunks' clean K/V plus the current chunk's own K/V).
 //
-// One CTA = two 128-query tiles (Q0, Q1) of one head, 352 threads:
+// One CTA = two 128-query tiles (Q0, Q1) of one head, 320 threads:
 //   warps 0..3  softmax WG 0 (tile Q0), thread = query row = TMEM lane;
 //   warps 4..7  softmax WG 1 (tile Q1);
 //   warp 8      TMA producer: Q0/Q1 once, then 128-key K and V tiles through
 //               a STAGES-deep ring (separate K and V barriers);
-//   warp 9      TMEM allocation; lane 0 issues the MMAs of tile Q0;
-//   warp 10     lane 0 issues the MMAs of tile Q1 (each tile advances on
-//               its own softmax's signals; K/V stages are freed by both).
+//   warp 9      TMEM allocation and MMA issue (converged warp, elected lane).
 // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after it.  P (bf16)
 // goes back into TMEM and feeds tcgen05.mma as the A operand straight from
 // tensor memory (no shared-memory round trip); V is read MN-major from its
@@ -44,7 +42,7 @@ struct AttnTile {
     static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
     static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
     static constexpr int TMEM_COLS = 512;
-    static constexpr int THREADS = 352;            // 8 softmax, 1 TMA, 2 MMA warps
+    static constexpr int THREADS = 320;            // 8 softmax, 1 TMA, 1 MMA warp
     static constexpr bool SEP_P = HD == 64;            // P has its own TMEM columns
     __host__ __device__ static constexpr int S_COL(int i) { return 128 * i; }
     __host__ __device__ static constexpr int O_COL(int i) { return 256 + HD * i; }
@@ -70,7 +68,7 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 
 template <int HD>
-__global__ void __launch_bounds__(352, 1)
+__global__ void __launch_bounds__(320, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
                    const int n_keys, const int d, const uint8_t *__restrict__ skip_flag, int *err) {
@@ -103,9 +101,9 @@ __global__ void __launch_bounds__(352, 1)
         mbar_init(q_full, 1);
         for (int s = 0; s < A::STAGES; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 2);        // released by both MMA issuers
+            mbar_init(&k_empty[s], 1);
             mbar_init(&v_full[s], 1);
-            mbar_init(&v_empty[s], 2);
+            mbar_init(&v_empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
@@ -153,41 +151,55 @@ __global__ void __launch_bounds__(352, 1)
             for (int j = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; j < v_issued; ++j)
                 mbar_wait(&v_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
-    } else if (warp >= 9) {
-        // ------------------------------------------ MMA issue (one warp per Q tile)
-        if (lane == 0) {
+    } else if (warp == 9) {
+        // ------------------------------------------------------ MMA issue
+        // The whole warp runs this loop (converged); one elected lane issues
+        // each tcgen05 instruction.
+        {
             constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);
             constexpr uint32_t idesc_o = idesc_bf16(128, HD, false, true);
-            const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV);
+            // Descriptors are built once; each MMA adds a constant to the
+            // start-address field (addresses stay below 256 KB, so the
+            // 14-bit field never carries).
+            const uint64_t dQ0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
+            const uint64_t dK0 = sdesc_sw128(smem_u32(sK), 16, 1024);
+            const uint64_t dV0 = sdesc_sw128(smem_u32(sV), A::REGION, 1024);
             auto issue_s = [&](int i, int j) {        // S_i = Q_i K_j^T
-                const int st = j % A::STAGES;
+                const uint64_t dq = dQ0 + (uint64_t)((i * A::Q_BYTES) >> 4);
+                const uint64_t dk = dK0 + (uint64_t)(((j % A::STAGES) * A::KV_BYTES) >> 4);
 #pragma unroll
                 for (int ks = 0; ks < HD / 16; ++ks) {
-                    const uint32_t off = (ks >> 2) * A::REGION + (ks & 3) * 32;
-                    tc_mma(tmem + A::S_COL(i), sdesc_sw128(aQ + i * A::Q_BYTES + off, 16, 1024),
-                           sdesc_sw128(aK + st * A::KV_BYTES + off, 16, 1024), idesc_s, ks > 0 ? 1u : 0u);
+                    const uint32_t off = ((ks >> 2) * A::REGION + (ks & 3) * 32) >> 4;
+                    tc_mma_warp(tmem + A::S_COL(i), dq + off, dk + off, idesc_s, ks > 0 ? 1u : 0u);
                 }
-                tc_commit(&s_full[i]);
+                tc_commit_warp(&s_full[i]);
             };
             auto issue_pv = [&](int i, int j) {       // O_i += P_i V_j, P_i in TMEM
-                const int st = j % A::STAGES;
+                const uint64_t dv = dV0 + (uint64_t)(((j % A::STAGES) * A::KV_BYTES) >> 4);
 #pragma unroll
                 for (int ks = 0; ks < A::BKV / 16; ++ks)
-                    tc_mma_tmem_a(tmem + A::O_COL(i), tmem + A::P_COL(i) + 8 * ks,
-                                  sdesc_sw128(aV + st * A::KV_BYTES + ks * 16 * 128, A::REGION, 1024), idesc_o,
-                                  (j > 0 || ks > 0) ? 1u : 0u);
+                    tc_mma_tmem_a_warp(tmem + A::O_COL(i), tmem + A::P_COL(i) + 8 * ks, dv + ((ks * 16 * 128) >> 4),
+                                       idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
             };
-            // One issuing warp per Q tile, so that neither tile's MMAs wait
-            // on the other's softmax.  hd 64: S_i(j+1) goes as soon as the
-            // softmax has read S_i(j), ahead of P_i V_j.  hd 128: P_i aliases
-            // S_i, so S_i(j+1) follows P_i V_j.  K and V stages are released
-            // by both issuers (barrier count 2).
-            const int i = warp - 9;
-            bool ok = mbar_wait(q_full, 0, err, ERR_WAIT_MMA) && mbar_wait(&k_full[0], 0, err, ERR_WAIT_MMA);
+            // One issuing thread, in the order the two softmax warpgroups
+            // produce their signals when they take turns on the exponential
+            // phase (WG 0 then WG 1 on every key tile):
+            //   hd 64 : S0(j+1), P1V(j-1), S1(j+1), P0V(j)  -- S_{j+1} is issued
+            //           once the softmax has read S_j (P has its own columns);
+            //   hd 128: P0V(j), S0(j+1), P1V(j), S1(j+1)    -- P overwrites S, so
+            //           S_{j+1} follows P V of the same tile.
+            // Each P V is then issued as soon as its P is ready and the
+            // tensor core has no other tile's work queued in front of it.
+            auto wait = [&](uint64_t *b, int parity) {
+                const bool r = mbar_wait(b, parity & 1, err, ERR_WAIT_MMA);
+                return __all_sync(0xffffffffu, r);
+            };
+            bool ok = wait(q_full, 0) && wait(&k_full[0], 0);
             if (ok) {
                 tc_fence_after();
-                issue_s(i, 0);
-                tc_commit(&k_empty[0]);
+                issue_s(0, 0);
+                issue_s(1, 0);
+                tc_commit_warp(&k_empty[0]);
             }
             for (int j = 0; ok && j < nkt; ++j) {
                 const int st = j % A::STAGES;
@@ -195,30 +207,53 @@ __global__ void __launch_bounds__(352, 1)
                 const bool more = j + 1 < nkt;
                 if constexpr (A::SEP_P) {
                     if (more) {
-                        if (!mbar_wait(&s_cons[i], j & 1, err, ERR_WAIT_MMA)) break;
-                        if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                        if (!(wait(&s_cons[0], j) && wait(&k_full[st1], (j + 1) / A::STAGES))) break;
                         tc_fence_after();
-                        issue_s(i, j + 1);
-                        tc_commit(&k_empty[st1]);
+                        issue_s(0, j + 1);
                     }
-                    if (!mbar_wait(&p_full[i], j & 1, err, ERR_WAIT_MMA)) break;
-                    if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
-                    issue_pv(i, j);
-                    tc_commit(&pv_done[i]);
-                    tc_commit(&v_empty[st]);
-                } else {
-                    if (!mbar_wait(&p_full[i], j & 1, err, ERR_WAIT_MMA)) break;
-                    if (!mbar_wait(&v_full[st], (j / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
-                    tc_fence_after();
-                    issue_pv(i, j);
-                    tc_commit(&v_empty[st]);
-                    if (!more) tc_commit(&pv_done[i]);
-                    if (more) {
-                        if (!mbar_wait(&k_full[st1], ((j + 1) / A::STAGES) & 1, err, ERR_WAIT_MMA)) break;
+                    if (j >= 1) {
+                        const int sp = (j - 1) % A::STAGES;
+                        if (!wait(&p_full[1], j - 1)) break;
                         tc_fence_after();
-                        issue_s(i, j + 1);
-                        tc_commit(&k_empty[st1]);
+                        issue_pv(1, j - 1);
+                        tc_commit_warp(&pv_done[1]);
+                        tc_commit_warp(&v_empty[sp]);
+                    }
+                    if (more) {
+                        if (!wait(&s_cons[1], j)) break;
+                        tc_fence_after();
+                        issue_s(1, j + 1);
+                        tc_commit_warp(&k_empty[st1]);
+                    }
+                    if (!(wait(&p_full[0], j) && wait(&v_full[st], j / A::STAGES))) break;
+                    tc_fence_after();
+                    issue_pv(0, j);
+                    tc_commit_warp(&pv_done[0]);
+                    if (!more) {
+                        if (!wait(&p_full[1], j)) break;
+                        tc_fence_after();
+                        issue_pv(1, j);
+                        tc_commit_warp(&pv_done[1]);
+                        tc_commit_warp(&v_empty[st]);
+                    }
+                } else {
+                    if (!(wait(&p_full[0], j) && wait(&v_full[st], j / A::STAGES))) break;
+                    tc_fence_after();
+                    issue_pv(0, j);
+                    if (!more) tc_commit_warp(&pv_done[0]);
+                    if (more) {
+                        if (!wait(&k_full[st1], (j + 1) / A::STAGES)) break;
+                        tc_fence_after();
+                        issue_s(0, j + 1);
+                    }
+                    if (!wait(&p_full[1], j)) break;
+                    tc_fence_after();
+                    issue_pv(1, j);
+                    tc_commit_warp(&v_empty[st]);
+                    if (!more) tc_commit_warp(&pv_done[1]);
+                    if (more) {
+                        issue_s(1, j + 1);
+                        tc_commit_warp(&k_empty[st1]);
                     }
                 }
             }
