@@ -4,12 +4,14 @@
 //   the current chunk's queries see every resident key of the rolling KV
 //   cache (past chunks' clean K/V plus the current chunk's own K/V).
 //
-// One CTA = two 128-query tiles (Q0, Q1) of one head, 320 threads:
+// One CTA = two 128-query tiles (Q0, Q1) of one head, 352 threads:
 //   warps 0..3  softmax WG 0 (tile Q0), thread = query row = TMEM lane;
 //   warps 4..7  softmax WG 1 (tile Q1);
 //   warp 8      TMA producer: Q0/Q1 once, then 128-key K and V tiles through
 //               a STAGES-deep ring (separate K and V barriers);
-//   warp 9      TMEM allocation and MMA issue (converged warp, elected lane).
+//   warp 9      TMEM allocation; MMA issue (hd 64: tile Q0; hd 128: both);
+//   warp 10     hd 64: MMA issue for tile Q1 (MMA warps run converged, one
+//               elected lane issuing each instruction).
 // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 after it.  P (bf16)
 // goes back into TMEM and feeds tcgen05.mma as the A operand straight from
 // tensor memory (no shared-memory round trip); V is read MN-major from its
@@ -20,6 +22,8 @@
 //   hd = 128: TMEM is full (S0 S1 O0 O1 = 512 columns); P_i overwrites S_i and
 //             S_{j+1} waits until P_j V has been issued; the two tiles
 //             ping-pong so the tensor core still has the other tile's work.
+// The two softmax warps of each SM sub-partition (one per tile) take turns
+// on the MUFU-bound exponential phase.
 // Online softmax in the exp2 domain with lazy rescaling: a row's O and sum
 // are rescaled only when its running max grows by more than 8 (2^8 headroom
 // in fp32 / bf16).  Score scaling and row sums use packed fp32 pairs
@@ -40,10 +44,11 @@ struct AttnTile {
     static constexpr int OFF_K = QT * Q_BYTES;
     static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
     static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
-    static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+    static constexpr int SMEM_BYTES = OFF_BAR + 512 + 1024;
     static constexpr int TMEM_COLS = 512;
-    static constexpr int THREADS = 320;            // 8 softmax, 1 TMA, 1 MMA warp
+    static constexpr int THREADS = 352;            // 8 softmax, 1 TMA, 2 MMA warps
     static constexpr bool SEP_P = HD == 64;            // P has its own TMEM columns
+    static constexpr int ISSUERS = SEP_P ? 2 : 1;      // MMA-issuing warps (9, 10)
     __host__ __device__ static constexpr int S_COL(int i) { return 128 * i; }
     __host__ __device__ static constexpr int O_COL(int i) { return 256 + HD * i; }
     __host__ __device__ static constexpr int P_COL(int i) { return SEP_P ? 256 + 2 * HD + 64 * i : 128 * i; }
@@ -68,7 +73,7 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 
 template <int HD>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(352, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
                    const int n_keys, const int d, const uint8_t *__restrict__ skip_flag, int *err) {
@@ -89,8 +94,8 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t *s_cons = s_full + 2;             // [2] S_i read by its softmax WG (hd 64)
     uint64_t *p_full = s_cons + 2;             // [2] P_i written, O_i corrected
     uint64_t *pv_done = p_full + 2;            // [2] P_i V done (hd 64: every tile; hd 128: last)
-    uint64_t *turn = pv_done + 2;              // [2] exponential phase hand-off between the WGs
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 2);
+    uint64_t *turn = pv_done + 2;              // [2][4] exponential-phase hand-off per (WG, quadrant)
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 8);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * (A::QT * A::BQ);
@@ -101,16 +106,16 @@ __global__ void __launch_bounds__(320, 1)
         mbar_init(q_full, 1);
         for (int s = 0; s < A::STAGES; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 1);
+            mbar_init(&k_empty[s], A::ISSUERS);   // freed by every MMA warp
             mbar_init(&v_full[s], 1);
-            mbar_init(&v_empty[s], 1);
+            mbar_init(&v_empty[s], A::ISSUERS);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
             mbar_init(&s_cons[i], 128);
             mbar_init(&p_full[i], 128);
             mbar_init(&pv_done[i], 1);
-            mbar_init(&turn[i], 4);           // one arrive per warp of the other WG
+            for (int qd = 0; qd < 4; ++qd) mbar_init(&turn[4 * i + qd], 1);
         }
         mbar_fence_init();
     }
@@ -151,11 +156,14 @@ __global__ void __launch_bounds__(320, 1)
             for (int j = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; j < v_issued; ++j)
                 mbar_wait(&v_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
-    } else if (warp == 9) {
+    } else if (warp >= 9) {
         // ------------------------------------------------------ MMA issue
-        // The whole warp runs this loop (converged); one elected lane issues
-        // each tcgen05 instruction.
-        {
+        // Warp 9 issues every MMA of Q tile 0, warp 10 those of tile 1, so
+        // the issue work is spread over two SM sub-partitions and neither
+        // tile waits on the other's softmax.  The whole warp runs the loop
+        // (converged); one elected lane issues each tcgen05 instruction.
+        // (hd 128 uses warp 9 alone; warp 10 has no work.)
+        if (warp == 9 || A::ISSUERS == 2) {
             constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);
             constexpr uint32_t idesc_o = idesc_bf16(128, HD, false, true);
             // Descriptors are built once; each MMA adds a constant to the
@@ -181,62 +189,51 @@ __global__ void __launch_bounds__(320, 1)
                     tc_mma_tmem_a_warp(tmem + A::O_COL(i), tmem + A::P_COL(i) + 8 * ks, dv + ((ks * 16 * 128) >> 4),
                                        idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
             };
-            // One issuing thread, in the order the two softmax warpgroups
-            // produce their signals when they take turns on the exponential
-            // phase (WG 0 then WG 1 on every key tile):
-            //   hd 64 : S0(j+1), P1V(j-1), S1(j+1), P0V(j)  -- S_{j+1} is issued
-            //           once the softmax has read S_j (P has its own columns);
-            //   hd 128: P0V(j), S0(j+1), P1V(j), S1(j+1)    -- P overwrites S, so
-            //           S_{j+1} follows P V of the same tile.
-            // Each P V is then issued as soon as its P is ready and the
-            // tensor core has no other tile's work queued in front of it.
             auto wait = [&](uint64_t *b, int parity) {
                 const bool r = mbar_wait(b, parity & 1, err, ERR_WAIT_MMA);
                 return __all_sync(0xffffffffu, r);
             };
             bool ok = wait(q_full, 0) && wait(&k_full[0], 0);
-            if (ok) {
-                tc_fence_after();
-                issue_s(0, 0);
-                issue_s(1, 0);
-                tc_commit_warp(&k_empty[0]);
-            }
-            for (int j = 0; ok && j < nkt; ++j) {
-                const int st = j % A::STAGES;
-                const int st1 = (j + 1) % A::STAGES;
-                const bool more = j + 1 < nkt;
-                if constexpr (A::SEP_P) {
-                    if (more) {
-                        if (!(wait(&s_cons[0], j) && wait(&k_full[st1], (j + 1) / A::STAGES))) break;
+            if constexpr (A::SEP_P) {
+                // hd 64: warp 9 drives tile 0 and warp 10 tile 1.  S_i(j+1) is
+                // issued once the softmax has read S_i(j) (P has its own
+                // columns), then P_i V_j once P_i is ready.  A K (V) stage is
+                // released when both warps' MMAs that read it are done.
+                const int i = warp - 9;
+                if (ok) {
+                    tc_fence_after();
+                    issue_s(i, 0);
+                    tc_commit_warp(&k_empty[0]);
+                }
+                for (int j = 0; ok && j < nkt; ++j) {
+                    const int st = j % A::STAGES;
+                    const int st1 = (j + 1) % A::STAGES;
+                    if (j + 1 < nkt) {
+                        if (!(wait(&s_cons[i], j) && wait(&k_full[st1], (j + 1) / A::STAGES))) break;
                         tc_fence_after();
-                        issue_s(0, j + 1);
-                    }
-                    if (j >= 1) {
-                        const int sp = (j - 1) % A::STAGES;
-                        if (!wait(&p_full[1], j - 1)) break;
-                        tc_fence_after();
-                        issue_pv(1, j - 1);
-                        tc_commit_warp(&pv_done[1]);
-                        tc_commit_warp(&v_empty[sp]);
-                    }
-                    if (more) {
-                        if (!wait(&s_cons[1], j)) break;
-                        tc_fence_after();
-                        issue_s(1, j + 1);
+                        issue_s(i, j + 1);
                         tc_commit_warp(&k_empty[st1]);
                     }
-                    if (!(wait(&p_full[0], j) && wait(&v_full[st], j / A::STAGES))) break;
+                    if (!(wait(&p_full[i], j) && wait(&v_full[st], j / A::STAGES))) break;
                     tc_fence_after();
-                    issue_pv(0, j);
-                    tc_commit_warp(&pv_done[0]);
-                    if (!more) {
-                        if (!wait(&p_full[1], j)) break;
-                        tc_fence_after();
-                        issue_pv(1, j);
-                        tc_commit_warp(&pv_done[1]);
-                        tc_commit_warp(&v_empty[st]);
-                    }
-                } else {
+                    issue_pv(i, j);
+                    tc_commit_warp(&pv_done[i]);
+                    tc_commit_warp(&v_empty[st]);
+                }
+            } else {
+                // hd 128: one warp issues P0V(j), S0(j+1), P1V(j), S1(j+1) -- the
+                // order in which the warpgroups finish their turns; P_i
+                // overwrites S_i, so S_i(j+1) follows P_i V_j.
+                if (ok) {
+                    tc_fence_after();
+                    issue_s(0, 0);
+                    issue_s(1, 0);
+                    tc_commit_warp(&k_empty[0]);
+                }
+                for (int j = 0; ok && j < nkt; ++j) {
+                    const int st = j % A::STAGES;
+                    const int st1 = (j + 1) % A::STAGES;
+                    const bool more = j + 1 < nkt;
                     if (!(wait(&p_full[0], j) && wait(&v_full[st], j / A::STAGES))) break;
                     tc_fence_after();
                     issue_pv(0, j);
@@ -322,12 +319,15 @@ __global__ void __launch_bounds__(320, 1)
                     tmem_st16_sync(tO + 16 * c, t);
                 }
             }
-            // The two WGs take turns on the exponential phase (MUFU bound):
-            // WG 0 does tile j, then WG 1 tile j, then WG 0 tile j + 1 ...
-            // so that one WG's exponentials overlap the other's loads, max
-            // and MMA waits instead of competing for the same units.
+            // The two warps of each SM sub-partition (quadrant q of WG 0 and
+            // of WG 1) take turns on the exponential phase, which is bound
+            // by the sub-partition's MUFU: WG 0 does tile j, then WG 1 tile
+            // j, then WG 0 tile j + 1 ... so that one warp's exponentials
+            // overlap the other's loads, max and MMA waits.  The hand-off is
+            // per quadrant, so a slower sub-partition does not hold up the
+            // others.
             if (wg == 1 || j > 0) {
-                ok = mbar_wait(&turn[wg], (wg == 1 ? j : j - 1) & 1, err, ERR_WAIT_SOFTMAX);
+                ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? j : j - 1) & 1, err, ERR_WAIT_SOFTMAX);
                 __syncwarp();
                 if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             }
@@ -359,7 +359,7 @@ __global__ void __launch_bounds__(320, 1)
             tc_fence_before();
             mbar_arrive(&p_full[wg]);
             __syncwarp();
-            if (lane == 0) mbar_arrive(&turn[wg ^ 1]);
+            if (lane == 0) mbar_arrive(&turn[4 * (wg ^ 1) + q]);
         }
         if (ok) ok = mbar_wait(&pv_done[wg], A::SEP_P ? ((nkt - 1) & 1) : 0, err, ERR_WAIT_SOFTMAX);
         __syncwarp();

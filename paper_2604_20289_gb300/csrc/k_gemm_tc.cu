@@ -106,32 +106,40 @@ __global__ void __launch_bounds__(320, 1)
                 mbar_wait(&full[j % G::STAGES], (j / G::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
     } else if (warp == 1) {
-        if (lane == 0) {
+        // MMA issue: the whole warp runs the loop (converged) and one elected
+        // lane issues each tcgen05 instruction, so issue keeps pace while the
+        // epilogue warps of the same sub-partitions are busy.
+        {
             constexpr uint32_t idesc = idesc_bf16(GEMM_BM, BN, false, false);
+            auto wait = [&](uint64_t *b, uint32_t parity) {
+                const bool r = mbar_wait(b, parity, err, ERR_WAIT_MMA);
+                return __all_sync(0xffffffffu, r);
+            };
+            // start-address field += offset >> 4 (shared addresses < 256 KB: no carry)
+            const uint64_t d0 = sdesc_sw128(smem_u32(smem), 16, 1024);
             int it = 0, local = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++local) {
                 const int buf = local & 1;
                 const uint32_t use = (uint32_t)(local >> 1);
-                if (!mbar_wait(&acc_empty[buf], (use & 1) ^ 1, err, ERR_WAIT_MMA)) break;
+                if (!wait(&acc_empty[buf], (use & 1) ^ 1)) break;
                 tc_fence_after();
                 const uint32_t acc = tmem + buf * BN;
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % G::STAGES;
-                    if (!mbar_wait(&full[s], (it / G::STAGES) & 1, err, ERR_WAIT_MMA)) {
+                    if (!wait(&full[s], (it / G::STAGES) & 1)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a = smem_u32(smem + s * G::STAGE_BYTES);
-                    const uint32_t b = a + G::A_BYTES;
+                    const uint64_t da = d0 + (uint64_t)((s * G::STAGE_BYTES) >> 4);
+                    const uint64_t db = da + (uint64_t)(G::A_BYTES >> 4);
 #pragma unroll
                     for (int k = 0; k < GEMM_BK / 16; ++k)
-                        tc_mma(acc, sdesc_sw128(a + 32 * k, 16, 1024), sdesc_sw128(b + 32 * k, 16, 1024), idesc,
-                               (kt | k) != 0 ? 1u : 0u);
-                    tc_commit(&empty[s]);
+                        tc_mma_warp(acc, da + 2 * k, db + 2 * k, idesc, (kt | k) != 0 ? 1u : 0u);
+                    tc_commit_warp(&empty[s]);
                 }
-                tc_commit(&acc_full[buf]);
+                tc_commit_warp(&acc_full[buf]);
             }
         }
     } else {
