@@ -112,6 +112,13 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
     for (int k = 0; k < NCH; ++k)
         if (k < mine) load16<T>(xr + 16 * (lane + 32 * k), v[k]);
+    // the modulation vectors do not depend on the moments: fetch them while
+    // the row reduction runs (one chunk ahead for wide rows)
+    float sc[16], sh[16];
+    if (mine > 0) {
+        load16<float>(scale + 16 * lane, sc);
+        load16<float>(shift + 16 * lane, sh);
+    }
     const Moments mo = warp_moments(lane_moments<NCH>(v, mine));
     const float rstd = rsqrtf(mo.m2 / (float)d + eps);
     T *orow = out + (size_t)row * d;
@@ -119,9 +126,10 @@ __global__ void __launch_bounds__(256)
     for (int k = 0; k < NCH; ++k) {
         if (k < mine) {
             const int c = 16 * (lane + 32 * k);
-            float sc[16], sh[16];
-            load16<float>(scale + c, sc);
-            load16<float>(shift + c, sh);
+            if (k > 0) {
+                load16<float>(scale + c, sc);
+                load16<float>(shift + c, sh);
+            }
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[k][i] = (v[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i];
             store16<T>(orow + c, v[k]);
@@ -217,27 +225,42 @@ cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st) 
 
 // y[j] = act_out( sum_i in(i) W[i][j] + b[j] + add[j] ), W [n_in][n_out].
 // in_silu: in = SiLU(x) instead of x.  act_out 0: none, 1: SiLU.
-// CTA = 32 output columns x 8 warps; warp w sums rows i = w (mod 8) with
-// coalesced 128-byte row segments, then the warps reduce in shared memory.
-__global__ void __launch_bounds__(256)
+// CTA = 32 output columns x 16 warps; the input vector (after SiLU) is
+// staged in shared memory once; warp w sums rows i = w (mod 16), four
+// independent rows per step so that several coalesced 128-byte row segments
+// are in flight per warp; the warps then reduce in shared memory.
+constexpr int GEMV_WARPS = 16;
+__global__ void __launch_bounds__(GEMV_WARPS * 32)
     gemv_kernel(const float *__restrict__ x, int in_silu, const float *__restrict__ W, const float *__restrict__ b,
                 const float *__restrict__ add, float *__restrict__ y, int n_in, int n_out, int act_out) {
-    __shared__ float part[8][33];
+    extern __shared__ float xs[];                       // [n_in]
+    __shared__ float part[GEMV_WARPS][33];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < n_in; i += blockDim.x) xs[i] = in_silu ? silu(x[i]) : x[i];
+    __syncthreads();
     const int j = blockIdx.x * 32 + lane;
-    float acc = 0.0f;
+    float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
     if (j < n_out) {
-        for (int i = warp; i < n_in; i += 8) {
-            const float xi = in_silu ? silu(x[i]) : x[i];
-            acc = fmaf(xi, W[(size_t)i * n_out + j], acc);
+        const float *wj = W + j;
+        int i = warp;
+        for (; i + 3 * GEMV_WARPS < n_in; i += 4 * GEMV_WARPS) {
+            const float w0 = wj[(size_t)i * n_out];
+            const float w1 = wj[(size_t)(i + GEMV_WARPS) * n_out];
+            const float w2 = wj[(size_t)(i + 2 * GEMV_WARPS) * n_out];
+            const float w3 = wj[(size_t)(i + 3 * GEMV_WARPS) * n_out];
+            a0 = fmaf(xs[i], w0, a0);
+            a1 = fmaf(xs[i + GEMV_WARPS], w1, a1);
+            a2 = fmaf(xs[i + 2 * GEMV_WARPS], w2, a2);
+            a3 = fmaf(xs[i + 3 * GEMV_WARPS], w3, a3);
         }
+        for (; i < n_in; i += GEMV_WARPS) a0 = fmaf(xs[i], wj[(size_t)i * n_out], a0);
     }
-    part[warp][lane] = acc;
+    part[warp][lane] = (a0 + a1) + (a2 + a3);
     __syncthreads();
     if (warp == 0 && j < n_out) {
         float s = 0.0f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) s += part[w][lane];
+        for (int w = 0; w < GEMV_WARPS; ++w) s += part[w][lane];
         s += b[j];
         if (add != nullptr) s += add[j];
         y[j] = act_out == 1 ? silu(s) : s;
@@ -246,7 +269,9 @@ __global__ void __launch_bounds__(256)
 
 cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
                  int n_out, int act_out, cudaStream_t st) {
-    gemv_kernel<<<(n_out + 31) / 32, 256, 0, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
+    const size_t smem = (size_t)n_in * sizeof(float);
+    if (smem > 48 * 1024) return cudaErrorInvalidValue;
+    gemv_kernel<<<(n_out + 31) / 32, GEMV_WARPS * 32, smem, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
     return cudaGetLastError();
 }
 
