@@ -50,10 +50,19 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
 
 /* o = softmax(q k^T / sqrt(head_dim)) v per head, no mask (every query sees
  * every key: full attention within the chunk and over all resident cached
- * keys).  q, o [Lq][H*hd]; k, v [n_keys][H*hd]. */
+ * keys).  q, o [Lq][H*hd]; k, v [n_keys][H*hd] (bf16: 16-byte aligned rows).
+ *   workspace  device, optional.  With at least
+ *              xc_op_attention_workspace_bytes() bytes and more (head,
+ *              256-query) units than SMs, the key range is split evenly over
+ *              the SMs and units cut between two SMs are merged by a second
+ *              kernel; with NULL (or too small) every unit runs whole on one
+ *              SM.  Contents on entry are ignored; it must not be shared by
+ *              calls that overlap in time.
+ * bf16 needs head_dim 64 or 128; fp32 head_dim 16, 32 or 64. */
+size_t xc_op_attention_workspace_bytes(int dtype, int head_dim);
 xc_status xc_op_attention(int dtype, int Lq, int n_keys, int n_heads, int head_dim,
                           const void *q, const void *k, const void *v, void *o,
-                          void *stream);
+                          void *workspace, size_t workspace_bytes, void *stream);
 
 /* out = LayerNorm(x) * (1 + scale) + shift over rows of length d (no affine,
  * population variance, eps), adaLN-Zero modulation.  x, out [M][d]. */

@@ -72,11 +72,35 @@ __device__ __forceinline__ float ex2_approx(float x) {
     return y;
 }
 
+// Work split.  A unit is (head, pair of 128-query tiles); its n_kt key tiles
+// form a row of the (unit, key tile) iteration space, T = n_units * n_kt.
+// CTA c of a G-CTA grid takes the contiguous iterations
+// [c T / G, (c + 1) T / G) -- whole units when G = n_units, a balanced
+// "stream-K" share when G = number of SMs < n_units.  A unit cut by the
+// boundary between CTAs c - 1 and c is finished by both: each writes its
+// unnormalised O with its running max m and sum l (a flash-decoding partial)
+// to slot (boundary c, part 0 = head / 1 = tail), and attn_combine_kernel
+// merges the two.  Every CTA's share is at least one unit, so a unit is cut
+// at most once.
+struct TileCursor {
+    int g, u, k;                                   // tile of this CTA, unit, key tile of the unit
+    __device__ __forceinline__ void next(int n_kt) {
+        ++g;
+        if (++k == n_kt) { k = 0; ++u; }
+    }
+};
+struct AttnSplit {
+    long long T;          // total iterations
+    int n_kt, n_qblk, G;
+    __host__ __device__ long long begin(int c) const { return T * c / G; }
+};
+
 template <int HD>
 __global__ void __launch_bounds__(352, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
-                   const int n_keys, const int d, const uint8_t *__restrict__ skip_flag, int *err) {
+                   const int n_keys, const int d, const AttnSplit sp, float *__restrict__ ws_o,
+                   float2 *__restrict__ ws_ml, const uint8_t *__restrict__ skip_flag, int *err) {
     using A = AttnTile<HD>;
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     extern __shared__ uint8_t smem_raw[];
@@ -85,25 +109,34 @@ __global__ void __launch_bounds__(352, 1)
     uint8_t *sK = smem + A::OFF_K;
     uint8_t *sV = smem + A::OFF_V;
     uint64_t *bar = reinterpret_cast<uint64_t *>(smem + A::OFF_BAR);
-    uint64_t *q_full = bar;
-    uint64_t *k_full = bar + 1;
+    uint64_t *q_full = bar;                    // Q of piece p landed (phase p)
+    uint64_t *q_empty = bar + 1;               // every S MMA of piece p done (phase p)
+    uint64_t *k_full = bar + 2;
     uint64_t *k_empty = k_full + A::STAGES;
     uint64_t *v_full = k_empty + A::STAGES;
     uint64_t *v_empty = v_full + A::STAGES;
     uint64_t *s_full = v_empty + A::STAGES;    // [2] S_i computed
     uint64_t *s_cons = s_full + 2;             // [2] S_i read by its softmax WG (hd 64)
     uint64_t *p_full = s_cons + 2;             // [2] P_i written, O_i corrected
-    uint64_t *pv_done = p_full + 2;            // [2] P_i V done (hd 64: every tile; hd 128: last)
-    uint64_t *turn = pv_done + 2;              // [2][4] exponential-phase hand-off per (WG, quadrant)
+    uint64_t *pv_done = p_full + 2;            // [2] P_i V done (hd 64: every tile; hd 128: last of a piece)
+    uint64_t *o_free = pv_done + 2;            // [2] O_i of piece p read out (phase p)
+    uint64_t *turn = o_free + 2;               // [2][4] exponential-phase hand-off per (WG, quadrant)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(turn + 8);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int q0 = blockIdx.x * (A::QT * A::BQ);
-    const int h = blockIdx.y;
-    const int nkt = (n_keys + A::BKV - 1) / A::BKV;
+    const int nkt = sp.n_kt;
+    const long long it0 = sp.begin(blockIdx.x);
+    const int n_t = (int)(sp.begin(blockIdx.x + 1) - it0);    // key tiles of this CTA (>= 1)
+    const int u0 = (int)(it0 / nkt);
+    // Each role walks this CTA's tiles with a cursor (tile g, unit u, key
+    // tile k) instead of dividing per tile.
+    const TileCursor c0{0, u0, (int)(it0 % nkt)};
+    auto first_of = [&](const TileCursor &c) { return c.g == 0 || c.k == 0; };
+    auto last_of = [&](const TileCursor &c) { return c.g == n_t - 1 || c.k == nkt - 1; };
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
+        mbar_init(q_empty, A::ISSUERS);
         for (int s = 0; s < A::STAGES; ++s) {
             mbar_init(&k_full[s], 1);
             mbar_init(&k_empty[s], A::ISSUERS);   // freed by every MMA warp
@@ -115,6 +148,7 @@ __global__ void __launch_bounds__(352, 1)
             mbar_init(&s_cons[i], 128);
             mbar_init(&p_full[i], 128);
             mbar_init(&pv_done[i], 1);
+            mbar_init(&o_free[i], 128);
             for (int qd = 0; qd < 4; ++qd) mbar_init(&turn[4 * i + qd], 1);
         }
         mbar_fence_init();
@@ -128,41 +162,51 @@ __global__ void __launch_bounds__(352, 1)
     if (warp == 8) {
         // ------------------------------------------------------ TMA producer
         if (lane == 0) {
-            mbar_expect_tx(q_full, A::QT * A::Q_BYTES);
-            for (int i = 0; i < A::QT; ++i)
-                for (int r = 0; r < A::NR; ++r)
-                    tma_load_2d(sQ + i * A::Q_BYTES + r * A::REGION, &tmQ, q_full, h * HD + 64 * r, q0 + i * A::BQ);
-            int k_issued = 0, v_issued = 0;
-            for (int j = 0; j < nkt; ++j) {
-                const int st = j % A::STAGES;
-                const uint32_t ph = ((j / A::STAGES) & 1) ^ 1;
+            int q_loads = 0, k_issued = 0, v_issued = 0;
+            int h = 0;
+            for (TileCursor c = c0; c.g < n_t; c.next(nkt)) {
+                const int g = c.g;
+                if (first_of(c)) {
+                    h = c.u / sp.n_qblk;
+                    const int q0 = (c.u % sp.n_qblk) * (A::QT * A::BQ);
+                    // the previous piece's Q stays until its last S MMA is done
+                    if (q_loads > 0 && !mbar_wait(q_empty, (q_loads - 1) & 1, err, ERR_WAIT_PRODUCER)) break;
+                    mbar_expect_tx(q_full, A::QT * A::Q_BYTES);
+                    for (int i = 0; i < A::QT; ++i)
+                        for (int r = 0; r < A::NR; ++r)
+                            tma_load_2d(sQ + i * A::Q_BYTES + r * A::REGION, &tmQ, q_full, h * HD + 64 * r,
+                                        q0 + i * A::BQ);
+                    ++q_loads;
+                }
+                const int st = g % A::STAGES, kt = c.k;
+                const uint32_t ph = ((g / A::STAGES) & 1) ^ 1;
                 if (!mbar_wait(&k_empty[st], ph, err, ERR_WAIT_PRODUCER)) break;
                 mbar_expect_tx(&k_full[st], A::KV_BYTES);
                 for (int r = 0; r < A::NR; ++r)
                     tma_load_2d(sK + st * A::KV_BYTES + r * A::REGION, &tmK, &k_full[st], h * HD + 64 * r,
-                                j * A::BKV);
-                k_issued = j + 1;
+                                kt * A::BKV);
+                k_issued = g + 1;
                 if (!mbar_wait(&v_empty[st], ph, err, ERR_WAIT_PRODUCER)) break;
                 mbar_expect_tx(&v_full[st], A::KV_BYTES);
                 for (int r = 0; r < A::NR; ++r)
                     tma_load_2d(sV + st * A::KV_BYTES + r * A::REGION, &tmV, &v_full[st], h * HD + 64 * r,
-                                j * A::BKV);
-                v_issued = j + 1;
+                                kt * A::BKV);
+                v_issued = g + 1;
             }
             // Drain: every copy this thread started has landed before exit.
-            mbar_wait(q_full, 0, err, ERR_WAIT_PRODUCER);
-            for (int j = k_issued - A::STAGES < 0 ? 0 : k_issued - A::STAGES; j < k_issued; ++j)
-                mbar_wait(&k_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
-            for (int j = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; j < v_issued; ++j)
-                mbar_wait(&v_full[j % A::STAGES], (j / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+            if (q_loads > 0) mbar_wait(q_full, (q_loads - 1) & 1, err, ERR_WAIT_PRODUCER);
+            for (int g = k_issued - A::STAGES < 0 ? 0 : k_issued - A::STAGES; g < k_issued; ++g)
+                mbar_wait(&k_full[g % A::STAGES], (g / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
+            for (int g = v_issued - A::STAGES < 0 ? 0 : v_issued - A::STAGES; g < v_issued; ++g)
+                mbar_wait(&v_full[g % A::STAGES], (g / A::STAGES) & 1, err, ERR_WAIT_PRODUCER);
         }
     } else if (warp >= 9) {
         // ------------------------------------------------------ MMA issue
-        // Warp 9 issues every MMA of Q tile 0, warp 10 those of tile 1, so
-        // the issue work is spread over two SM sub-partitions and neither
-        // tile waits on the other's softmax.  The whole warp runs the loop
-        // (converged); one elected lane issues each tcgen05 instruction.
-        // (hd 128 uses warp 9 alone; warp 10 has no work.)
+        // hd 64: warp 9 issues every MMA of Q tile 0, warp 10 those of tile 1,
+        // so the issue work is spread over two SM sub-partitions and neither
+        // tile waits on the other's softmax.  hd 128: warp 9 alone.  The
+        // whole warp runs the loop (converged); one elected lane issues each
+        // tcgen05 instruction.
         if (warp == 9 || A::ISSUERS == 2) {
             constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);
             constexpr uint32_t idesc_o = idesc_bf16(128, HD, false, true);
@@ -172,9 +216,9 @@ __global__ void __launch_bounds__(352, 1)
             const uint64_t dQ0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
             const uint64_t dK0 = sdesc_sw128(smem_u32(sK), 16, 1024);
             const uint64_t dV0 = sdesc_sw128(smem_u32(sV), A::REGION, 1024);
-            auto issue_s = [&](int i, int j) {        // S_i = Q_i K_j^T
+            auto issue_s = [&](int i, int g) {        // S_i = Q_i K_g^T
                 const uint64_t dq = dQ0 + (uint64_t)((i * A::Q_BYTES) >> 4);
-                const uint64_t dk = dK0 + (uint64_t)(((j % A::STAGES) * A::KV_BYTES) >> 4);
+                const uint64_t dk = dK0 + (uint64_t)(((g % A::STAGES) * A::KV_BYTES) >> 4);
 #pragma unroll
                 for (int ks = 0; ks < HD / 16; ++ks) {
                     const uint32_t off = ((ks >> 2) * A::REGION + (ks & 3) * 32) >> 4;
@@ -182,75 +226,92 @@ __global__ void __launch_bounds__(352, 1)
                 }
                 tc_commit_warp(&s_full[i]);
             };
-            auto issue_pv = [&](int i, int j) {       // O_i += P_i V_j, P_i in TMEM
-                const uint64_t dv = dV0 + (uint64_t)(((j % A::STAGES) * A::KV_BYTES) >> 4);
+            auto issue_pv = [&](int i, const TileCursor &c) {   // O_i (+)= P_i V_g, P_i in TMEM
+                const uint64_t dv = dV0 + (uint64_t)(((c.g % A::STAGES) * A::KV_BYTES) >> 4);
+                const bool fresh = first_of(c);        // first tile of a piece: O_i = P_i V_g
 #pragma unroll
                 for (int ks = 0; ks < A::BKV / 16; ++ks)
                     tc_mma_tmem_a_warp(tmem + A::O_COL(i), tmem + A::P_COL(i) + 8 * ks, dv + ((ks * 16 * 128) >> 4),
-                                       idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+                                       idesc_o, (!fresh || ks > 0) ? 1u : 0u);
             };
-            auto wait = [&](uint64_t *b, int parity) {
+            auto wait = [&](uint64_t *b, int parity) -> bool {
                 const bool r = mbar_wait(b, parity & 1, err, ERR_WAIT_MMA);
-                return __all_sync(0xffffffffu, r);
+                return __all_sync(0xffffffffu, r) != 0;
             };
-            bool ok = wait(q_full, 0) && wait(&k_full[0], 0);
+            // S of tile g needs its piece's Q (and, after a piece's last S,
+            // the producer may replace Q); P V of the first tile of a piece
+            // overwrites O, so it waits until the softmax has read O out.
+            auto s_ready = [&](const TileCursor &c) -> bool {
+                if (first_of(c) && !wait(q_full, c.u - u0)) return false;
+                return wait(&k_full[c.g % A::STAGES], c.g / A::STAGES);
+            };
+            auto pv_ready = [&](int i, const TileCursor &c) -> bool {
+                if (first_of(c) && c.u > u0 && !wait(&o_free[i], c.u - u0 - 1)) return false;
+                return wait(&p_full[i], c.g) && wait(&v_full[c.g % A::STAGES], c.g / A::STAGES);
+            };
             if constexpr (A::SEP_P) {
-                // hd 64: warp 9 drives tile 0 and warp 10 tile 1.  S_i(j+1) is
-                // issued once the softmax has read S_i(j) (P has its own
-                // columns), then P_i V_j once P_i is ready.  A K (V) stage is
-                // released when both warps' MMAs that read it are done.
+                // hd 64: S_i(g+1) is issued once the softmax has read S_i(g) (P
+                // has its own columns), then P_i V_g once P_i is ready.
                 const int i = warp - 9;
+                bool ok = s_ready(c0);
                 if (ok) {
                     tc_fence_after();
                     issue_s(i, 0);
                     tc_commit_warp(&k_empty[0]);
+                    if (last_of(c0)) tc_commit_warp(q_empty);
                 }
-                for (int j = 0; ok && j < nkt; ++j) {
-                    const int st = j % A::STAGES;
-                    const int st1 = (j + 1) % A::STAGES;
-                    if (j + 1 < nkt) {
-                        if (!(wait(&s_cons[i], j) && wait(&k_full[st1], (j + 1) / A::STAGES))) break;
+                TileCursor cs = c0;                    // next S tile is cs + 1
+                for (TileCursor c = c0; ok && c.g < n_t; c.next(nkt)) {
+                    const int g = c.g;
+                    if (g + 1 < n_t) {
+                        cs.next(nkt);
+                        if (!(wait(&s_cons[i], g) && s_ready(cs))) break;
                         tc_fence_after();
-                        issue_s(i, j + 1);
-                        tc_commit_warp(&k_empty[st1]);
+                        issue_s(i, g + 1);
+                        tc_commit_warp(&k_empty[(g + 1) % A::STAGES]);
+                        if (last_of(cs)) tc_commit_warp(q_empty);
                     }
-                    if (!(wait(&p_full[i], j) && wait(&v_full[st], j / A::STAGES))) break;
+                    if (!pv_ready(i, c)) break;
                     tc_fence_after();
-                    issue_pv(i, j);
+                    issue_pv(i, c);
                     tc_commit_warp(&pv_done[i]);
-                    tc_commit_warp(&v_empty[st]);
+                    tc_commit_warp(&v_empty[g % A::STAGES]);
                 }
             } else {
-                // hd 128: one warp issues P0V(j), S0(j+1), P1V(j), S1(j+1) -- the
+                // hd 128: one warp issues P0V(g), S0(g+1), P1V(g), S1(g+1) -- the
                 // order in which the warpgroups finish their turns; P_i
-                // overwrites S_i, so S_i(j+1) follows P_i V_j.
+                // overwrites S_i, so S_i(g+1) follows P_i V_g.
+                bool ok = s_ready(c0);
                 if (ok) {
                     tc_fence_after();
                     issue_s(0, 0);
                     issue_s(1, 0);
                     tc_commit_warp(&k_empty[0]);
+                    if (last_of(c0)) tc_commit_warp(q_empty);
                 }
-                for (int j = 0; ok && j < nkt; ++j) {
-                    const int st = j % A::STAGES;
-                    const int st1 = (j + 1) % A::STAGES;
-                    const bool more = j + 1 < nkt;
-                    if (!(wait(&p_full[0], j) && wait(&v_full[st], j / A::STAGES))) break;
+                TileCursor cs = c0;                    // next S tile is cs + 1
+                for (TileCursor c = c0; ok && c.g < n_t; c.next(nkt)) {
+                    const int g = c.g;
+                    const bool more = g + 1 < n_t;
+                    if (more) cs.next(nkt);
+                    if (!pv_ready(0, c)) break;
                     tc_fence_after();
-                    issue_pv(0, j);
-                    if (!more) tc_commit_warp(&pv_done[0]);
+                    issue_pv(0, c);
+                    if (last_of(c)) tc_commit_warp(&pv_done[0]);
                     if (more) {
-                        if (!wait(&k_full[st1], (j + 1) / A::STAGES)) break;
+                        if (!s_ready(cs)) break;
                         tc_fence_after();
-                        issue_s(0, j + 1);
+                        issue_s(0, g + 1);
                     }
-                    if (!wait(&p_full[1], j)) break;
+                    if (!pv_ready(1, c)) break;
                     tc_fence_after();
-                    issue_pv(1, j);
-                    tc_commit_warp(&v_empty[st]);
-                    if (!more) tc_commit_warp(&pv_done[1]);
+                    issue_pv(1, c);
+                    tc_commit_warp(&v_empty[g % A::STAGES]);
+                    if (last_of(c)) tc_commit_warp(&pv_done[1]);
                     if (more) {
-                        issue_s(1, j + 1);
-                        tc_commit_warp(&k_empty[st1]);
+                        issue_s(1, g + 1);
+                        tc_commit_warp(&k_empty[(g + 1) % A::STAGES]);
+                        if (last_of(cs)) tc_commit_warp(q_empty);
                     }
                 }
             }
@@ -259,17 +320,23 @@ __global__ void __launch_bounds__(352, 1)
         // ------------------------------------------------------------ softmax
         const int wg = warp >> 2;                          // tile of this warpgroup
         const int q = warp & 3;                            // TMEM lane quadrant
-        const int row = q0 + wg * A::BQ + q * 32 + lane;
+        const int r_tile = wg * A::BQ + q * 32 + lane;     // row within the unit (0..255)
         const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
         const uint32_t tS = tl + A::S_COL(wg);
         const uint32_t tP = tl + A::P_COL(wg);
         const uint32_t tO = tl + A::O_COL(wg);
         const float sl2 = rsqrtf((float)HD) * 1.4426950408889634f;
         const int tail = n_keys - (nkt - 1) * A::BKV;      // valid keys in the last tile
-        float m = -INFINITY, l = 0.0f;
         bool ok = true;
-        for (int j = 0; j < nkt; ++j) {
-            ok = mbar_wait(&s_full[wg], j & 1, err, ERR_WAIT_SOFTMAX);
+        TileCursor cur = c0;
+        while (ok && cur.g < n_t) {
+          // ---- one piece: key tiles [cur.k, ...] of unit cur.u
+          const bool cut_front = cur.g == 0 && cur.k != 0;       // the unit began in CTA c-1
+          float m = -INFINITY, l = 0.0f;
+          bool fresh = true;
+          for (;;) {
+            const int g = cur.g;
+            ok = mbar_wait(&s_full[wg], g & 1, err, ERR_WAIT_SOFTMAX);
             __syncwarp();
             if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             tc_fence_after();
@@ -279,7 +346,7 @@ __global__ void __launch_bounds__(352, 1)
                 tc_fence_before();
                 mbar_arrive(&s_cons[wg]);
             }
-            if (j == nkt - 1 && tail < A::BKV) {
+            if (cur.k == nkt - 1 && tail < A::BKV) {
 #pragma unroll
                 for (int c = 0; c < 128; ++c)
                     if (c >= tail) s[c] = -INFINITY;
@@ -296,19 +363,20 @@ __global__ void __launch_bounds__(352, 1)
 #pragma unroll
             for (int k = 0; k < 5; ++k) mx[k] = fmax3(mx[k], mx[k + 5], mx[k + 10]);
             const float m_new = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[15]), mx[0]) * sl2;
-            const bool grow = j > 0 && m_new > m + A::LAZY;
+            if (fresh) m = m_new;
+            const bool grow = !fresh && m_new > m + A::LAZY;
             const float alpha = grow ? ex2_approx(m - m_new) : 1.0f;
-            if (j == 0 || grow) m = m_new;
+            if (grow) m = m_new;
             if constexpr (A::SEP_P) {
                 // P_i buffer free and O_i stable once P V of the previous tile is done
-                if (j >= 1) {
-                    ok = mbar_wait(&pv_done[wg], (j - 1) & 1, err, ERR_WAIT_SOFTMAX);
+                if (g >= 1) {
+                    ok = mbar_wait(&pv_done[wg], (g - 1) & 1, err, ERR_WAIT_SOFTMAX);
                     __syncwarp();
                     if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
                     tc_fence_after();
                 }
             }
-            // (hd 128: the commit behind s_full already covers P V of tile j-1)
+            // (hd 128: the commit behind s_full already covers P V of tile g-1)
             if (__any_sync(0xffffffffu, grow)) {
 #pragma unroll 1
                 for (int c = 0; c < HD / 16; ++c) {
@@ -321,26 +389,26 @@ __global__ void __launch_bounds__(352, 1)
             }
             // The two warps of each SM sub-partition (quadrant q of WG 0 and
             // of WG 1) take turns on the exponential phase, which is bound
-            // by the sub-partition's MUFU: WG 0 does tile j, then WG 1 tile
-            // j, then WG 0 tile j + 1 ... so that one warp's exponentials
+            // by the sub-partition's MUFU: WG 0 does tile g, then WG 1 tile
+            // g, then WG 0 tile g + 1 ... so that one warp's exponentials
             // overlap the other's loads, max and MMA waits.  The hand-off is
             // per quadrant, so a slower sub-partition does not hold up the
             // others.
-            if (wg == 1 || j > 0) {
-                ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? j : j - 1) & 1, err, ERR_WAIT_SOFTMAX);
+            if (wg == 1 || g > 0) {
+                ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? g : g - 1) & 1, err, ERR_WAIT_SOFTMAX);
                 __syncwarp();
                 if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             }
             // probabilities p = 2^(s * sl2 - m), packed bf16 pairs + row sum,
-            // stored to TMEM in two 64-key halves
+            // stored to TMEM in four 32-key quarters
             const float2 sc2 = make_float2(sl2, sl2), nm2 = make_float2(-m, -m);
             float2 rs0 = make_float2(0.f, 0.f), rs1 = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t w[32];
+            for (int qt = 0; qt < 4; ++qt) {
+                uint32_t w[16];
 #pragma unroll
-                for (int k = 0; k < 32; k += 2) {
-                    const int c = 64 * half + 2 * k;
+                for (int k = 0; k < 16; k += 2) {
+                    const int c = 32 * qt + 2 * k;
                     const float2 a = __ffma2_rn(make_float2(s[c], s[c + 1]), sc2, nm2);
                     const float2 b = __ffma2_rn(make_float2(s[c + 2], s[c + 3]), sc2, nm2);
                     const float2 pa = make_float2(ex2_approx(a.x), ex2_approx(a.y));
@@ -352,7 +420,7 @@ __global__ void __launch_bounds__(352, 1)
                     w[k] = *reinterpret_cast<uint32_t *>(&h0);
                     w[k + 1] = *reinterpret_cast<uint32_t *>(&h1);
                 }
-                tmem_st32_sync(tP + 32 * half, w);
+                tmem_st16u_sync(tP + 16 * qt, w);
             }
             const float2 rs = __fadd2_rn(rs0, rs1);
             l = l * alpha + (rs.x + rs.y);
@@ -360,20 +428,46 @@ __global__ void __launch_bounds__(352, 1)
             mbar_arrive(&p_full[wg]);
             __syncwarp();
             if (lane == 0) mbar_arrive(&turn[4 * (wg ^ 1) + q]);
-        }
-        if (ok) ok = mbar_wait(&pv_done[wg], A::SEP_P ? ((nkt - 1) & 1) : 0, err, ERR_WAIT_SOFTMAX);
-        __syncwarp();
-        if (__all_sync(0xffffffffu, ok)) {
-            tc_fence_after();
-            const float inv = 1.0f / l;
+            fresh = false;
+            if (last_of(cur)) break;
+            cur.next(nkt);
+          }
+          if (!ok) break;
+          {
+                // end of a piece: O_i complete -> output (whole unit) or partial
+                const int g = cur.g, u = cur.u, p = u - u0;
+                ok = mbar_wait(&pv_done[wg], (A::SEP_P ? g : p) & 1, err, ERR_WAIT_SOFTMAX);
+                __syncwarp();
+                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                tc_fence_after();
+                const int h = u / sp.n_qblk;
+                const int row = (u % sp.n_qblk) * (A::QT * A::BQ) + r_tile;
+                const bool head_part = cur.k != nkt - 1;                       // unit continues in CTA c+1
+                if (!head_part && !cut_front) {
+                    const float inv = 1.0f / l;
 #pragma unroll 1
-            for (int c = 0; c < HD / 16; ++c) {
-                float t[16];
-                tmem_ld16_sync(tO + 16 * c, t);
+                    for (int c = 0; c < HD / 16; ++c) {
+                        float t[16];
+                        tmem_ld16_sync(tO + 16 * c, t);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) t[i] *= inv;
-                if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
-            }
+                        for (int i = 0; i < 16; ++i) t[i] *= inv;
+                        if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
+                    }
+                } else {
+                    const int slot = head_part ? 2 * (blockIdx.x + 1) : 2 * blockIdx.x + 1;
+                    float *wo = ws_o + ((size_t)slot * (A::QT * A::BQ) + r_tile) * HD;
+#pragma unroll 1
+                    for (int c = 0; c < HD / 16; ++c) {
+                        float t[16];
+                        tmem_ld16_sync(tO + 16 * c, t);
+                        store16<float>(wo + 16 * c, t);
+                    }
+                    ws_ml[(size_t)slot * (A::QT * A::BQ) + r_tile] = make_float2(m, l);
+                }
+                tc_fence_before();
+                mbar_arrive(&o_free[wg]);
+          }
+          cur.next(nkt);
         }
     }
     tc_fence_before();
@@ -384,12 +478,61 @@ __global__ void __launch_bounds__(352, 1)
     }
 }
 
+// Merges the two partials of every unit cut by a CTA boundary (see
+// AttnSplit): m = max(m0, m1), O = (O0 2^(m0-m) + O1 2^(m1-m)) /
+// (l0 2^(m0-m) + l1 2^(m1-m)).  One CTA per boundary, one thread per row.
+template <int HD>
+__global__ void __launch_bounds__(256)
+    attn_combine_kernel(bf16 *__restrict__ o, const int Lq, const int d, const AttnSplit sp,
+                        const float *__restrict__ ws_o, const float2 *__restrict__ ws_ml,
+                        const uint8_t *__restrict__ skip_flag) {
+    if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
+    const int b = blockIdx.x + 1;                      // boundary between CTAs b-1 and b
+    const long long it = sp.begin(b);
+    if (it % sp.n_kt == 0) return;                     // the boundary falls between units
+    const int u = (int)(it / sp.n_kt);
+    const int h = u / sp.n_qblk;
+    const int r = threadIdx.x;
+    const int row = (u % sp.n_qblk) * 256 + r;
+    if (row >= Lq) return;
+    const float2 a = ws_ml[(size_t)(2 * b) * 256 + r], c = ws_ml[(size_t)(2 * b + 1) * 256 + r];
+    const float mm = fmaxf(a.x, c.x);
+    const float w0 = exp2f(a.x - mm), w1 = exp2f(c.x - mm);
+    const float inv = 1.0f / (a.y * w0 + c.y * w1);
+    const float *o0 = ws_o + ((size_t)(2 * b) * 256 + r) * HD;
+    const float *o1 = ws_o + ((size_t)(2 * b + 1) * 256 + r) * HD;
+#pragma unroll 1
+    for (int k = 0; k < HD; k += 16) {
+        float x0[16], x1[16];
+        load16<float>(o0 + k, x0);
+        load16<float>(o1 + k, x1);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) x0[i] = (x0[i] * w0 + x1[i] * w1) * inv;
+        store16<bf16>(o + (size_t)row * d + h * HD + k, x0);
+    }
+}
+
 bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+
+static int sm_count() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    }
+    return n;
+}
+
+size_t attn_workspace_bytes(int head_dim) {
+    const size_t slots = 2 * ((size_t)sm_count() + 1);
+    return slots * 256 * ((size_t)head_dim * sizeof(float) + sizeof(float2));
+}
 
 template <int HD>
 static cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, bf16 *o,
-                               int Lq, int n_keys, int n_heads, int d, const uint8_t *skip, int *err,
-                               cudaStream_t st) {
+                               int Lq, int n_keys, int n_heads, int d, void *ws, size_t ws_bytes,
+                               const uint8_t *skip, int *err, int *n_launched, cudaStream_t st) {
     using A = AttnTile<HD>;
     static bool attr_set = false;
     if (!attr_set) {
@@ -398,18 +541,40 @@ static cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, con
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    dim3 grid((Lq + A::QT * A::BQ - 1) / (A::QT * A::BQ), n_heads);
-    attn_tc_kernel<HD><<<grid, A::THREADS, A::SMEM_BYTES, st>>>(tq, tk, tv, o, Lq, n_keys, d, skip, err);
-    return cudaGetLastError();
+    AttnSplit sp;
+    sp.n_kt = (n_keys + A::BKV - 1) / A::BKV;
+    sp.n_qblk = (Lq + A::QT * A::BQ - 1) / (A::QT * A::BQ);
+    const int n_units = sp.n_qblk * n_heads;
+    sp.T = (long long)n_units * sp.n_kt;
+    const int n_sm = sm_count();
+    const bool split = n_units > n_sm && ws != nullptr && ws_bytes >= attn_workspace_bytes(HD);
+    sp.G = split ? n_sm : n_units;
+    float *ws_o = split ? reinterpret_cast<float *>(ws) : nullptr;
+    float2 *ws_ml = split ? reinterpret_cast<float2 *>(ws_o + 2 * ((size_t)n_sm + 1) * 256 * HD) : nullptr;
+    attn_tc_kernel<HD><<<sp.G, A::THREADS, A::SMEM_BYTES, st>>>(tq, tk, tv, o, Lq, n_keys, d, sp, ws_o, ws_ml, skip,
+                                                                 err);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    if (n_launched) *n_launched = 1;
+    if (split && sp.G > 1) {
+        attn_combine_kernel<HD><<<sp.G - 1, 256, 0, st>>>(o, Lq, d, sp, ws_o, ws_ml, skip);
+        e = cudaGetLastError();
+        if (n_launched) *n_launched = 2;
+    }
+    return e;
 }
 
 // q [Lq][d], k / v maps over [>= n_keys][d] (box 128 rows), o [Lq][d]; hd in {64, 128}.
+// ws: attn_workspace_bytes(hd) bytes enable the balanced split over the SMs
+// when there are more units than SMs (nullptr: one CTA per unit).
 cudaError_t attn_tc(int head_dim, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
-                    bf16 *o, int Lq, int n_keys, int n_heads, int d, const uint8_t *skip, int *err,
-                    cudaStream_t st) {
+                    bf16 *o, int Lq, int n_keys, int n_heads, int d, void *ws, size_t ws_bytes,
+                    const uint8_t *skip, int *err, int *n_launched, cudaStream_t st) {
     if (n_keys < 1 || Lq < 1) return cudaErrorInvalidValue;
-    if (head_dim == 64) return launch_attn<64>(tq, tk, tv, o, Lq, n_keys, n_heads, d, skip, err, st);
-    if (head_dim == 128) return launch_attn<128>(tq, tk, tv, o, Lq, n_keys, n_heads, d, skip, err, st);
+    if (head_dim == 64)
+        return launch_attn<64>(tq, tk, tv, o, Lq, n_keys, n_heads, d, ws, ws_bytes, skip, err, n_launched, st);
+    if (head_dim == 128)
+        return launch_attn<128>(tq, tk, tv, o, Lq, n_keys, n_heads, d, ws, ws_bytes, skip, err, n_launched, st);
     return cudaErrorInvalidValue;
 }
 

@@ -142,6 +142,10 @@ struct xc_ctx {
     size_t g_ticket_off;
     char *g_scratch;
 
+    // attention split workspace (partials of units cut between CTAs)
+    void *attn_ws;
+    size_t attn_ws_bytes;
+
     // tensor maps (bf16)
     CUtensorMap tm_h, tm_o, tm_u, tm_q;
     std::vector<CUtensorMap> tm_wqkv, tm_wo, tm_w1, tm_w2, tm_rk, tm_rv;
@@ -445,8 +449,10 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.rope_cs = ctx->rope_cs;
         if constexpr (sizeof(T) == 2) {
             LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
-            LAUNCH(XC_K_ATTN, b, 1, attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L,
-                                            n_keys, ctx->H, d, flag, ctx->d_err, st));
+            int n_attn = 1;
+            LAUNCH(XC_K_ATTN, b, n_attn,
+                   attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L, n_keys,
+                           ctx->H, d, ctx->attn_ws, ctx->attn_ws_bytes, flag, ctx->d_err, &n_attn, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->qkv_wt) + (size_t)b * 3 * d * d;
             LAUNCH(XC_K_QKV, b, 1, gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
@@ -701,6 +707,10 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
 
         // gate scratch
         ctx->g_scratch = dalloc<char>(ctx, gate_scratch(ctx->V, d, &ctx->g_ns, &ctx->g_ticket_off));
+        if (ctx->bf) {
+            ctx->attn_ws_bytes = attn_workspace_bytes(ctx->hd);
+            ctx->attn_ws = dalloc<char>(ctx, ctx->attn_ws_bytes);
+        }
 
         // tensor maps of the bf16 path
         if (ctx->bf) {
@@ -1101,8 +1111,13 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
     return XC_OK;
 }
 
+size_t xc_op_attention_workspace_bytes(int dtype, int head_dim) {
+    if (dtype != XC_BF16 || (head_dim != 64 && head_dim != 128)) return 0;
+    return attn_workspace_bytes(head_dim);
+}
+
 xc_status xc_op_attention(int dtype, int Lq, int n_keys, int n_heads, int head_dim, const void *q, const void *k,
-                          const void *v, void *o, void *stream) {
+                          const void *v, void *o, void *workspace, size_t workspace_bytes, void *stream) {
     if (Lq < 1 || n_keys < 1 || n_heads < 1 || q == nullptr || k == nullptr || v == nullptr || o == nullptr)
         OP_FAIL(XC_EINVAL, "xc_op_attention: bad argument");
     const int d = n_heads * head_dim;
@@ -1113,8 +1128,8 @@ xc_status xc_op_attention(int dtype, int Lq, int n_keys, int n_heads, int head_d
         if (!make_tmap_bf16(&tq, q, Lq, d, 128) || !make_tmap_bf16(&tk, k, n_keys, d, 128) ||
             !make_tmap_bf16(&tv, v, n_keys, d, 128))
             OP_FAIL(XC_EINVAL, "xc_op_attention: tensor map");
-        OP_CK(attn_tc(head_dim, tq, tk, tv, reinterpret_cast<bf16 *>(o), Lq, n_keys, n_heads, d, nullptr,
-                      op_err_word(), st));
+        OP_CK(attn_tc(head_dim, tq, tk, tv, reinterpret_cast<bf16 *>(o), Lq, n_keys, n_heads, d, workspace,
+                      workspace_bytes, nullptr, op_err_word(), nullptr, st));
     } else if (dtype == XC_F32) {
         OP_CK(attn_simt(head_dim, reinterpret_cast<const float *>(q), reinterpret_cast<const float *>(k),
                         reinterpret_cast<const float *>(v), reinterpret_cast<float *>(o), Lq, n_keys, n_heads,

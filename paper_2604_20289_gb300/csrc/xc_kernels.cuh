@@ -39,7 +39,9 @@ bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t co
 cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
                     const uint8_t *skip, int *err, cudaStream_t st);
 cudaError_t attn_tc(int head_dim, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, bf16 *o,
-                    int Lq, int n_keys, int n_heads, int d, const uint8_t *skip, int *err, cudaStream_t st);
+                    int Lq, int n_keys, int n_heads, int d, void *ws, size_t ws_bytes, const uint8_t *skip, int *err,
+                    int *n_launched, cudaStream_t st);
+size_t attn_workspace_bytes(int head_dim);
 cudaError_t gemm_simt(int epi, const EpiParams &ep, const float *A, const float *Wt, int K, const uint8_t *skip,
                       cudaStream_t st);
 cudaError_t attn_simt(int head_dim, const float *q, const float *k, const float *v, float *o, int Lq, int n_keys,

@@ -93,7 +93,8 @@ SIGNATURES = {
     "xc_profile_stop": (_I, [_P, ctypes.POINTER(ProfileRec), _I, ctypes.POINTER(_I)]),
     "xc_op_linear": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
     "xc_op_qkv_rope": (_I, [_I, _I, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P]),
-    "xc_op_attention": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "xc_op_attention_workspace_bytes": (ctypes.c_size_t, [_I, _I]),
+    "xc_op_attention": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "xc_op_ln_mod": (_I, [_I, _I, _I, _F, _P, _P, _P, _P, _P]),
     "xc_op_residual_reuse": (_I, [_I, _L, _P, _P, _P, _P]),
     "xc_op_device_error": (_I, []),
@@ -270,9 +271,22 @@ def op_qkv_rope(dtype, n_cams, frames, gh, gw, chunk, head_dim, theta, A, Wt, bi
                              _stream(stream)))
 
 
-def op_attention(dtype, n_heads, head_dim, q, k, v, o, stream=None):
+def op_attention_workspace_bytes(dtype, head_dim):
+    return LIB.xc_op_attention_workspace_bytes(dtype_code(dtype), head_dim)
+
+
+def op_attention(dtype, n_heads, head_dim, q, k, v, o, workspace=None, stream=None):
+    """workspace: None (one SM per unit), "auto" (a device buffer of
+    op_attention_workspace_bytes is allocated for the call) or a device
+    tensor of at least that many bytes."""
+    if isinstance(workspace, str) and workspace == "auto":
+        import torch
+        nb = op_attention_workspace_bytes(dtype, head_dim)
+        workspace = torch.empty(max(nb, 1), dtype=torch.uint8, device=q.device) if nb else None
+    ws_ptr = _ptr(workspace) if workspace is not None else None
+    ws_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     check(LIB.xc_op_attention(dtype_code(dtype), q.shape[0], k.shape[0], n_heads, head_dim, _ptr(q),
-                              _ptr(k), _ptr(v), _ptr(o), _stream(stream)))
+                              _ptr(k), _ptr(v), _ptr(o), ws_ptr, ws_bytes, _stream(stream)))
 
 
 def op_ln_mod(dtype, x, shift, scale, out, eps=1e-6, stream=None):

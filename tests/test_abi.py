@@ -72,4 +72,4 @@ def test_host_validation_without_gpu(xb):
     # operator argument checks happen before any launch
     assert xb.LIB.xc_op_linear(1, 0, 0, 256, 64, None, None, None, None, None, None, None, None,
                                None) == xb.XC_EINVAL
-    assert xb.LIB.xc_op_attention(1, 0, 1, 1, 64, None, None, None, None, None) == xb.XC_EINVAL
+    assert xb.LIB.xc_op_attention(1, 0, 1, 1, 64, None, None, None, None, None, 0, None) == xb.XC_EINVAL

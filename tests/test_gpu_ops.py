@@ -199,14 +199,17 @@ def test_residual_reuse_exact(dtype, n):
 
 
 # ------------------------------------------- full workload sizes, sampled
+@pytest.mark.parametrize("ws", [None, "auto"])
 @pytest.mark.parametrize("Lq,Lk,H,hd", [(8064, 32256, 8, 64), (12960, 38880, 12, 128)])
-def test_attention_full_size_sampled(Lq, Lk, H, hd):
+def test_attention_full_size_sampled(Lq, Lk, H, hd, ws):
+    """Both launch shapes: one SM per (head, 256-query) unit, and the
+    balanced split over the SMs with cut units merged from two partials."""
     d = H * hd
     q = rt(f"Fq{Lq}{d}", (Lq, d))
     k = rt(f"Fk{Lk}{d}", (Lk, d))
     v = rt(f"Fv{Lk}{d}", (Lk, d))
     o = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
-    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o)
+    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o, workspace=ws)
     torch.cuda.synchronize()
     rows = np.unique(np.r_[0, 127, 128, Lq - 1, np.random.default_rng(3).integers(0, Lq, 60)])
     want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64),
@@ -239,3 +242,34 @@ def test_linear_full_size_sampled(M, N, K, epi):
     else:
         want = O.to_bf16(res[rows] + g * y)
     assert_close(host(out)[rows], want, "bf16")
+
+
+# Split-mode cases: more (head, 256-query) units than SMs, few key tiles, so
+# the CTA boundaries cut units at many different key tiles, including ragged
+# last tiles inside partial pieces; (8064, 100): one key tile, boundaries
+# never cut a unit.
+@pytest.mark.parametrize("Lq,Lk,H,hd", [(8064, 300, 8, 64), (8064, 700, 8, 64), (8064, 100, 8, 64),
+                                        (12960, 1000, 4, 128)])
+def test_attention_split_all_rows(Lq, Lk, H, hd):
+    d = H * hd
+    q = rt(f"Sq{Lq}{d}", (Lq, d))
+    k = rt(f"Sk{Lk}{d}", (Lk, d))
+    v = rt(f"Sv{Lk}{d}", (Lk, d))
+    o_split = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
+    o_whole = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
+    qd, kd, vd = dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16")
+    xb.op_attention("bf16", H, hd, qd, kd, vd, o_split, workspace="auto")
+    xb.op_attention("bf16", H, hd, qd, kd, vd, o_whole)
+    torch.cuda.synchronize()
+    rows = np.arange(Lq) if hd == 64 else np.unique(np.r_[0, 255, 256, Lq - 1,
+                                                          np.random.default_rng(5).integers(0, Lq, 1500)])
+    want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64),
+                                 k.reshape(Lk, H, hd).astype(np.float64),
+                                 v.reshape(Lk, H, hd).astype(np.float64)).reshape(len(rows), d))
+    got = host(o_split)[rows]
+    assert rel_l2(got, want) <= 5e-3
+    # every row, not just on average: the worst row of a cut unit stays close
+    per_row = np.sqrt(((got - want) ** 2).sum(1) / (want ** 2).sum(1))
+    assert per_row.max() <= 2e-2, per_row.max()
+    assert rel_l2(host(o_whole)[rows], want) <= 5e-3
+    assert xb.op_device_error() == 0
