@@ -52,6 +52,13 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--calibrate", action="store_true", help="print gate-metric quantiles and exit")
+    ap.add_argument("--sweep", action="store_true",
+                    help="threshold sweep on the stress rollout (1.3B shape, closed loop); prints one JSON line")
+    ap.add_argument("--sweep-chunks", type=int, default=200)
+    # gate aggressiveness ladder: tau_floor:margin:tau_dev (Eq. 9 floor, EMA
+    # margin m, deviation threshold of Eq. 7); the first point is Table 1
+    ap.add_argument("--sweep-points",
+                    default="0.97:0.02:2.0,0.95:0.05:3.0,0.9:0.1:4.0,0.8:0.2:6.0,0.6:0.4:10.0,0.3:0.7:20.0")
     return ap.parse_args()
 
 
@@ -202,6 +209,9 @@ def main():
     if args.impl == "reference":
         run_reference(args)
         return
+    if args.sweep:
+        sweep(args)
+        return
     import torch
     from paper_2604_20289_gb300 import xcache as xb
 
@@ -245,13 +255,14 @@ def main():
             xc.profile_start(kinds=("attn",), capacity=cfg.n_blocks * (S + 1) * args.steps + 16)
         barrier()
         l0 = xc.launch_count
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for n in range(args.warmup, n_total):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ev[0].record(stream)
+        for i, n in enumerate(range(args.warmup, n_total)):
             chunk(n, gate)
-        e1.record(stream)
+            ev[i + 1].record(stream)
         barrier()
-        ms = e0.elapsed_time(e1)
+        ms = ev[0].elapsed_time(ev[-1])
+        per_chunk = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
         launches = xc.launch_count - l0
         recs = xc.profile_stop() if profile else []
         if world > 1:
@@ -259,7 +270,7 @@ def main():
             t = torch.tensor([ms], device=dev)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             ms = float(t.item())
-        return ms, launches, recs
+        return ms, launches, recs, per_chunk
 
     gate = xb.gate_params(tau_floor=args.tau_floor, tau_dev=args.tau_dev)
     if args.calibrate:
@@ -268,9 +279,9 @@ def main():
 
     sampler = ClockSampler(local)
     sampler.start()
-    ms_x, launches, recs = timed(gate, profile=True)
+    ms_x, launches, recs, pc_x = timed(gate, profile=True)
     clocks = sampler.stop()
-    ms_all, _, recs_all = timed(xb.gate_params(enabled=0), profile=True)
+    ms_all, _, recs_all, pc_all = timed(xb.gate_params(enabled=0), profile=True)
     xc.sync()
 
     # skip rates over the timed chunks (decisions logged per (pass, block))
@@ -301,9 +312,11 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
             "config": config_of(cfg, args),
             "skip_rate": {"all_passes": skip_all, "denoise_passes": skip_den},
-            "all_blocks": {"ms_per_chunk": ms_all / args.steps,
+            "ms_per_chunk_p50": float(np.median(pc_x)),
+            "all_blocks": {"ms_per_chunk": ms_all / args.steps, "ms_per_chunk_p50": float(np.median(pc_all)),
                            "chunks_per_s": n_chunks / (ms_all * 1e-3)},
             "speedup_vs_all_blocks": ms_all / ms_x,
+            "predicted_speedup": predicted_speedup(xc, chunk, gate, args, cfg, ms_all / args.steps),
             "roofline": roofline, "gpu_launches": int(launches), "clocks": clocks}
 
     if not args.no_e2e:
@@ -323,6 +336,128 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
+    """Speedup predicted from kernel times (untimed, profiled re-run of both
+    arms over the same chunks): T_all / (T_all - sum over skipped block-passes
+    of (T_block - T_gate - T_reuse) + sum over gated block-passes of T_gate),
+    per chunk, T_block from the all-blocks arm at the same (chunk, pass, block)."""
+    from paper_2604_20289_gb300 import xcache as xb
+    S = cfg.n_steps
+    n_total = args.warmup + args.steps
+
+    def run(g):
+        xc.reset()
+        for n in range(args.warmup):
+            chunk(n, g)
+        xc.profile_start(kinds=xb.KERNEL_KINDS, capacity=cfg.n_blocks * (S + 1) * args.steps * 12 + 64)
+        for n in range(args.warmup, n_total):
+            chunk(n, g)
+        return xc.profile_stop()
+
+    block_kinds = {"ln", "qkv", "attn", "oproj", "ffn1", "ffn2"}
+    t_block = {}
+    for r in run(xb.gate_params(enabled=0)):
+        if r["kind"] in block_kinds:
+            key = (r["chunk"], r["pass_seq"] % (S + 1), r["block"])
+            t_block[key] = t_block.get(key, 0.0) + r["ms"]
+    saved = gated = 0.0
+    per = {}
+    for r in run(gate):
+        if r["kind"] in ("gate", "reuse") and r["block"] >= 0:
+            key = (r["chunk"], r["pass_seq"] % (S + 1), r["block"])
+            d = per.setdefault(key, {"dec": r["decision"], "gate": 0.0, "reuse": 0.0})
+            d[r["kind"]] += r["ms"]
+    for key, d in per.items():
+        if d["dec"] == xb.XC_DEC_FORCED:
+            continue
+        gated += d["gate"]
+        if d["dec"] == xb.XC_DEC_SKIP:
+            saved += t_block.get(key, 0.0) - d["gate"] - d["reuse"]
+    saved /= args.steps
+    gated /= args.steps
+    return t_all / (t_all - saved + gated)
+
+
+def sweep(args):
+    """Closed-loop stress rollout (each chunk's KV pass takes the chunk's own
+    denoised latent, so caching errors can accumulate through the KV ring):
+    an all-blocks reference, then one X-Cache rollout per tau_floor.  Per
+    point: skip rates (denoise and KV passes), time per chunk and speedup,
+    rel-L2 of every chunk's final latent against the reference rollout, and
+    the per-block skip counts."""
+    import torch
+    from paper_2604_20289_gb300 import xcache as xb
+    cfg = X.STRESS_1P3B
+    N = args.sweep_chunks
+    S, B = cfg.n_steps, cfg.n_blocks
+    traj = X.Trajectory(cfg, X.STRESS_TRAJ, n_chunks=N)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    noise = torch.stack([torch.from_numpy(traj.noise(n)) for n in range(N)]).to(dev)
+    acts = [traj.action(n) for n in range(N)]
+    stream = torch.cuda.current_stream()
+    xc = xb.XCache(cfg, X.make_weights(cfg), stream=stream)
+    x = torch.empty(cfg.tokens, cfg.c_latent, device=dev)
+    v = torch.empty_like(x)
+
+    def chunk(n, gate):
+        x.copy_(noise[n])
+        for t in range(S):
+            xc.chunk_step(x, acts[n], SIGMAS[t], t, False, gate, v_out=v, want_stats=False)
+            xc.euler(x, v, SIGMAS[t + 1] - SIGMAS[t])
+        xc.chunk_step(x, acts[n], 0.0, S, True, gate, want_stats=False)
+
+    def rollout(gate, ref=None):
+        xc.reset()
+        xc.profile_start(kinds=("ln",), capacity=N * (S + 1) * B * 2 + 64)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(N)]
+        finals, rel = [], []
+        for n in range(N):
+            ev[n][0].record(stream)
+            chunk(n, gate)
+            ev[n][1].record(stream)
+            if ref is None:
+                finals.append(x.clone())
+            else:
+                rel.append(torch.linalg.vector_norm(x - ref[n]) / torch.linalg.vector_norm(ref[n]))
+        torch.cuda.synchronize()
+        recs = xc.profile_stop()
+        ms = [a.elapsed_time(b) for a, b in ev]
+        dec = {}
+        for r in recs:
+            if r["block"] >= 0:
+                dec[(r["pass_seq"], r["block"])] = r["decision"]
+        den = [d for (ps, b), d in dec.items() if ps % (S + 1) < S]
+        kv = [d for (ps, b), d in dec.items() if ps % (S + 1) == S]
+        per_block = [0] * B
+        for (ps, b), d in dec.items():
+            if ps % (S + 1) < S and d == xb.XC_DEC_SKIP:
+                per_block[b] += 1
+        out = {"ms_per_chunk": float(np.mean(ms[1:])), "ms_per_chunk_p50": float(np.median(ms[1:])),
+               "skip_denoise": float(np.mean([d == xb.XC_DEC_SKIP for d in den])) if den else 0.0,
+               "skips_on_kv_passes": int(sum(d == xb.XC_DEC_SKIP for d in kv)),
+               "per_block_denoise_skips": per_block}
+        if ref is not None:
+            rl = np.array([float(t) for t in rel])
+            out.update({"rel_l2_mean": float(rl.mean()), "rel_l2_max": float(rl.max()),
+                        "rel_l2_first20": float(rl[:20].mean()), "rel_l2_last20": float(rl[-20:].mean())})
+        return out, finals
+
+    base, ref = rollout(xb.gate_params(enabled=0))
+    points = []
+    for pt in args.sweep_points.split(","):
+        tau, margin, dev_t = (float(t) for t in pt.split(":"))
+        res, _ = rollout(xb.gate_params(tau_floor=tau, margin=margin, tau_dev=dev_t), ref=ref)
+        res.update({"tau_floor": tau, "margin": margin, "tau_dev": dev_t})
+        res["speedup"] = base["ms_per_chunk"] / res["ms_per_chunk"]
+        points.append(res)
+    line = {"sweep": cfg.name, "chunks": N, "trajectory": "rho 0.95 -> 0.5, action jump +-0.8 every 20 chunks",
+            "closed_loop": True, "timing": "mean over chunks 1..N-1, CUDA events",
+            "all_blocks_ms_per_chunk": base["ms_per_chunk"], "points": points}
+    print(json.dumps(line), flush=True)
+    xc.close()
 
 
 def e2e(xc, traj, acts, cfg, args, gate, world, dev):
