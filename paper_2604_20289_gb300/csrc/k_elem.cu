@@ -7,15 +7,18 @@ namespace xc {
 
 // ------------------------------------------------------------ patch embed
 // X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][16].
-// One thread per (row, 16-column run); float4 loads of z and pe_w (L1-resident).
+// Warp = one 16-column run of 32 consecutive rows (lane = row): every lane
+// needs the same 16 x 16 block of pe_w, so its loads are warp-wide
+// broadcasts, and each lane reads its own 64-byte latent row.
 template <typename T>
 __global__ void __launch_bounds__(256)
     patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w, const float *__restrict__ b,
                        T *__restrict__ out, int L, int d) {
-    const int runs = d / 16;
-    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= L * runs) return;
-    const int row = idx / runs, col = (idx % runs) * 16;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int run = blockIdx.y * 8 + warp;
+    const int row = blockIdx.x * 32 + lane;
+    if (run * 16 >= d || row >= L) return;
+    const int col = run * 16;
     float zr[16];
     load16<float>(z + (size_t)row * 16, zr);
     float acc[16];
@@ -32,9 +35,9 @@ __global__ void __launch_bounds__(256)
 
 template <typename T>
 cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st) {
-    if (C != 16) return cudaErrorInvalidValue;
-    const int n = L * (d / 16);
-    patch_embed_kernel<T><<<(n + 255) / 256, 256, 0, st>>>(z, w, b, out, L, d);
+    if (C != 16 || d % 16 != 0) return cudaErrorInvalidValue;
+    const dim3 grid((L + 31) / 32, (d / 16 + 7) / 8);
+    patch_embed_kernel<T><<<grid, 256, 0, st>>>(z, w, b, out, L, d);
     return cudaGetLastError();
 }
 template cudaError_t patch_embed<float>(const float *, const float *, const float *, float *, int, int, int, cudaStream_t);
@@ -319,94 +322,110 @@ cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, i
 }
 
 // ------------------------------------------------------------------- head
-// One warp per row, row in registers: hf = round(LN(x) (1 + scale) + shift);
-// v = hf W_out + b_out (16 output channels, float32 out).  The normalised row
-// goes through shared memory in 512-element pieces; lane l then owns outputs
-// 4 (l % 4) .. +3 for rows i = l / 4 (mod 8) of the piece, so one float4 load
-// instruction of the warp reads 8 consecutive rows of W_out (512 contiguous
-// bytes); three shuffle levels fold the 8 row groups.
-template <typename T, int NCH>
+// Output head (a10): v = round(LN(x) * (1 + scale) + shift) W_out + b,
+// W_out [d][16].  CTA = 32 rows, 256 threads.  Pass 1: warp w reduces the
+// moments of rows 4w..4w+3.  Pass 2 walks the columns in chunks of 256: the
+// CTA writes the modulated chunk h[32][256] (rounded to the storage type) to
+// shared memory, then warp w multiplies its 32-column slice: lane (r4, c4)
+// accumulates rows 4 r4..4 r4+3 x outputs 4 c4..4 c4+3, reading W_out rows
+// as float4 (shared by the 8 lanes with the same c4) and h as broadcasts
+// (row stride 257 words: the 8 row groups fall in distinct banks).  The 8
+// warps' partial sums are then added in shared memory.
+constexpr int HEAD_ROWS = 32, HEAD_CH = 256;
+template <typename T>
 __global__ void __launch_bounds__(256)
     head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
                 const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
-    __shared__ float hrow[8][512];
-    const int wib = threadIdx.x >> 5;
-    const int row = blockIdx.x * 8 + wib;
-    const int lane = threadIdx.x & 31;
-    if (row >= L) return;
-    const T *xr = x + (size_t)row * d;
+    __shared__ float hs[HEAD_ROWS * (HEAD_CH + 1)];
+    __shared__ float2 stats[HEAD_ROWS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int row0 = blockIdx.x * HEAD_ROWS;
     const int runs = d / 16;
-    const int mine = runs > lane ? (runs - lane + 31) / 32 : 0;
-    float val[NCH][16];
+    for (int rr = 0; rr < 4; ++rr) {
+        const int r = warp * 4 + rr, row = row0 + r;
+        Moments mo{0.0f, 0.0f, 0.0f};
+        if (row < L) {
+            for (int run = lane; run < runs; run += 32) {
+                float t[16];
+                load16<T>(x + (size_t)row * d + 16 * run, t);
+                float sum = 0.0f;
 #pragma unroll
-    for (int k = 0; k < NCH; ++k)
-        if (k < mine) load16<T>(xr + 16 * (lane + 32 * k), val[k]);
-    const Moments mo = warp_moments(lane_moments<NCH>(val, mine));
-    const float rstd = rsqrtf(mo.m2 / (float)d + eps);
+                for (int i = 0; i < 16; ++i) sum += t[i];
+                Moments m1{16.0f, sum * (1.0f / 16.0f), 0.0f};
+#pragma unroll
+                for (int i = 0; i < 16; ++i) m1.m2 += (t[i] - m1.mean) * (t[i] - m1.mean);
+                mo = merge(mo, m1);
+            }
+        }
+        mo = warp_moments(mo);
+        if (lane == 0) stats[r] = make_float2(mo.mean, rsqrtf(mo.m2 / (float)d + eps));
+    }
+    __syncthreads();
     const float *shift = hm, *scale = hm + d;
-    const int grp = lane >> 2, oq = lane & 3;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    const int r4 = lane >> 2, c4 = lane & 3;
+    float acc[4][4];
 #pragma unroll
-    for (int k = 0; k < NCH; ++k) {
-        if (32 * k * 16 >= d) break;                       // warp-uniform
-        if (k < mine) {
-            const int c = 16 * (lane + 32 * k);
-            float sc[16], sh[16];
-            load16<float>(scale + c, sc);
-            load16<float>(shift + c, sh);
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-                hrow[wib][16 * lane + i] = round_to<T>((val[k][i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i]);
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+    for (int c0 = 0; c0 < d; c0 += HEAD_CH) {
+        const int n = d - c0 < HEAD_CH ? d - c0 : HEAD_CH;      // multiple of 16
+        const int nr = n / 16;
+        for (int idx = threadIdx.x; idx < HEAD_ROWS * nr; idx += blockDim.x) {
+            const int r = idx / nr, cr = (idx - r * nr) * 16, row = row0 + r;
+            float t[16];
+            if (row < L) {
+                float sc[16], sh[16];
+                load16<T>(x + (size_t)row * d + c0 + cr, t);
+                load16<float>(scale + c0 + cr, sc);
+                load16<float>(shift + c0 + cr, sh);
+                const float2 st = stats[r];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) t[i] = round_to<T>((t[i] - st.x) * st.y * (1.0f + sc[i]) + sh[i]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) t[i] = 0.0f;
+            }
+#pragma unroll
+            for (int i = 0; i < 16; ++i) hs[r * (HEAD_CH + 1) + cr + i] = t[i];
         }
-        __syncwarp();
-        const int c0 = 512 * k;
-        const int n_here = d - c0 < 512 ? d - c0 : 512;
-        const float4 *w4 = reinterpret_cast<const float4 *>(w + (size_t)c0 * 16) + oq;
-#pragma unroll 4
-        for (int i = grp; i < n_here; i += 8) {
-            const float hv = hrow[wib][i];
-            const float4 t = w4[(size_t)i * 4];
-            acc.x = fmaf(hv, t.x, acc.x);
-            acc.y = fmaf(hv, t.y, acc.y);
-            acc.z = fmaf(hv, t.z, acc.z);
-            acc.w = fmaf(hv, t.w, acc.w);
-        }
-        __syncwarp();
-    }
+        __syncthreads();
+        const int k_end = 32 * warp + 32 < n ? 32 * warp + 32 : n;
+        for (int k = 32 * warp; k < k_end; ++k) {
+            const float4 wv = *reinterpret_cast<const float4 *>(w + (size_t)(c0 + k) * 16 + 4 * c4);
 #pragma unroll
-    for (int s = 4; s < 32; s <<= 1) {
-        acc.x += __shfl_xor_sync(0xffffffffu, acc.x, s);
-        acc.y += __shfl_xor_sync(0xffffffffu, acc.y, s);
-        acc.z += __shfl_xor_sync(0xffffffffu, acc.z, s);
-        acc.w += __shfl_xor_sync(0xffffffffu, acc.w, s);
+            for (int i = 0; i < 4; ++i) {
+                const float hv = hs[(4 * r4 + i) * (HEAD_CH + 1) + k];
+                acc[i][0] = fmaf(hv, wv.x, acc[i][0]);
+                acc[i][1] = fmaf(hv, wv.y, acc[i][1]);
+                acc[i][2] = fmaf(hv, wv.z, acc[i][2]);
+                acc[i][3] = fmaf(hv, wv.w, acc[i][3]);
+            }
+        }
+        __syncthreads();
     }
-    if (lane < 4) {
-        const float4 bb = reinterpret_cast<const float4 *>(b)[lane];
-        reinterpret_cast<float4 *>(v + (size_t)row * 16)[lane] =
-            make_float4(acc.x + bb.x, acc.y + bb.y, acc.z + bb.z, acc.w + bb.w);
+    // partial sums of the 8 warps -> shared memory (reuses hs), then add
+    float *red = hs;                                          // [8][32][16] = 4096 floats
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) red[(warp * HEAD_ROWS + 4 * r4 + i) * 16 + 4 * c4 + j] = acc[i][j];
+    __syncthreads();
+    for (int o = threadIdx.x; o < HEAD_ROWS * 16; o += blockDim.x) {
+        const int r = o >> 4, c = o & 15;
+        float sum = b[c];
+#pragma unroll
+        for (int ww = 0; ww < 8; ++ww) sum += red[(ww * HEAD_ROWS + r) * 16 + c];
+        if (row0 + r < L) v[(size_t)(row0 + r) * 16 + c] = sum;
     }
-}
-
-template <typename T, int NCH>
-static cudaError_t head_n(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d,
-                          float eps, cudaStream_t st) {
-    head_kernel<T, NCH><<<(L + 7) / 8, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
-    return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
                  cudaStream_t st) {
     if (d % 16 != 0) return cudaErrorInvalidValue;
-    switch ((d + 511) / 512) {
-        case 1: return head_n<T, 1>(x, hm, w, b, v, L, d, eps, st);
-        case 2: return head_n<T, 2>(x, hm, w, b, v, L, d, eps, st);
-        case 3: return head_n<T, 3>(x, hm, w, b, v, L, d, eps, st);
-        case 4: return head_n<T, 4>(x, hm, w, b, v, L, d, eps, st);
-        case 5: case 6: case 7: case 8: return head_n<T, 8>(x, hm, w, b, v, L, d, eps, st);
-        case 9: case 10: case 11: case 12: return head_n<T, 12>(x, hm, w, b, v, L, d, eps, st);
-        default: return cudaErrorInvalidValue;
-    }
+    head_kernel<T><<<(L + HEAD_ROWS - 1) / HEAD_ROWS, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
+    return cudaGetLastError();
 }
 template cudaError_t head<float>(const float *, const float *, const float *, const float *, float *, int, int, float,
                                  cudaStream_t);

@@ -46,6 +46,117 @@ __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
     return p + ((1024u - (s & 1023u)) & 1023u);
 }
 
+// Epilogue operands of one 32-column block of a warp: the thread owns rows
+// r = it * 8 + lane / 4 (it = 0..3) of its 32-row quadrant and the 8 columns
+// [col, col + 8).  They are loaded into registers ahead of use (bf16 path).
+template <int EPI>
+struct EpiPrefetch {
+    float bias[8];
+    float gate[8];
+    uint4 resid[4];
+    uint4 xin[4];
+    float2 cs[4][4];      // RoPE (cos, sin) of the 4 pairs, per row
+};
+
+__device__ __forceinline__ uint4 ld_u4(const void *p) { return *reinterpret_cast<const uint4 *>(p); }
+
+template <int EPI>
+__device__ __forceinline__ void epi_prefetch(const EpiParams &p, int row0, int col, int lane, EpiPrefetch<EPI> &f) {
+    loadW<float, 8>(p.bias + col, f.bias);
+    if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
+        loadW<float, 8>(p.gate + col, f.gate);
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+            const int row = row0 + it * 8 + (lane >> 2);
+            if (row < p.M) {
+                f.resid[it] = ld_u4(reinterpret_cast<const bf16 *>(p.resid) + (size_t)row * p.N + col);
+                if constexpr (EPI == EPI_RESID_CACHE)
+                    if (p.rhat != nullptr) f.xin[it] = ld_u4(reinterpret_cast<const bf16 *>(p.xin) + (size_t)row * p.N + col);
+            }
+        }
+    }
+    if constexpr (EPI == EPI_QKV_ROPE) {
+        const int part = col / p.d;
+        const int c = col - part * p.d;
+        if (part < 2) {
+            const int pair0 = (c % p.head_dim) >> 1;
+            int off[4], axis[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                off[j] = p.rope_off[pair0 + j];
+                axis[j] = p.rope_axis[pair0 + j];
+            }
+#pragma unroll
+            for (int it = 0; it < 4; ++it) {
+                const int row = row0 + it * 8 + (lane >> 2);
+                if (row < p.M) {
+                    const int cam = row / p.npc;
+                    const int rem = row - cam * p.npc;
+                    const int pos[4] = {cam, rem / (p.gh * p.gw), (rem / p.gw) % p.gh, rem % p.gw};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) f.cs[it][j] = p.rope_cs[off[j] + pos[axis[j]]];
+                }
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void unpack8(uint4 u, float (&v)[8]) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float2 t = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
+        v[2 * j] = t.x;
+        v[2 * j + 1] = t.y;
+    }
+}
+
+// Same arithmetic as epilogue_run<EPI, bf16, 8> on prefetched operands.
+template <int EPI>
+__device__ __forceinline__ void epi_apply(const EpiParams &p, int row, int col, float (&acc)[8],
+                                          const EpiPrefetch<EPI> &f, int it) {
+    if (row >= p.M) return;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] += f.bias[i];
+    const size_t off = (size_t)row * p.N + col;
+    if constexpr (EPI == EPI_BIAS) {
+        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
+    } else if constexpr (EPI == EPI_GELU) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = gelu_tanh_approx(acc[i]);
+        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
+    } else if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
+        float r[8];
+        unpack8(f.resid[it], r);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = r[i] + f.gate[i] * acc[i];
+        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
+        if constexpr (EPI == EPI_RESID_CACHE) {
+            if (p.rhat != nullptr) {
+                float xi[8];
+                unpack8(f.xin[it], xi);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] = round_to<bf16>(acc[i]) - xi[i];
+                storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.rhat) + off, acc);
+            }
+        }
+    } else if constexpr (EPI == EPI_QKV_ROPE) {
+        const int part = col / p.d;
+        const int c = col - part * p.d;
+        if (part < 2) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 t = f.cs[it][j];
+                const float x0 = acc[2 * j], x1 = acc[2 * j + 1];
+                acc[2 * j] = x0 * t.x - x1 * t.y;
+                acc[2 * j + 1] = x0 * t.y + x1 * t.x;
+            }
+        }
+        bf16 *dst = reinterpret_cast<bf16 *>(part == 0 ? p.out : (part == 1 ? p.out_k : p.out_v));
+        storeW<bf16, 8>(dst + (size_t)row * p.d + c, acc);
+    }
+}
+
 template <int BN, int EPI, typename T>
 __global__ void __launch_bounds__(320, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -155,13 +266,21 @@ __global__ void __launch_bounds__(320, 1)
         for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++local) {
             const int buf = local & 1;
             const uint32_t use = (uint32_t)(local >> 1);
+            const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
+            const int c8 = (lane & 3) * 8;
+            // The global operands of this warp's first column block are
+            // requested before the accumulator is ready; those of block
+            // j + 1 right after block j is stored, so they are in flight
+            // while block j + 1 comes out of TMEM.
+            EpiPrefetch<EPI> pf;
+            epi_prefetch<EPI>(ep, m0 + q * 32, n0 + half * (BN / 2) + c8, lane, pf);
             const bool ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
             __syncwarp();
             if (!__all_sync(0xffffffffu, ok)) break;
             tc_fence_after();
-            const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
-#pragma unroll 1
-            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) {
+                const int c = half * (BN / 2) + 32 * j;
                 float v[16];
                 tmem_ld16_sync(tq + buf * BN + c, v);
 #pragma unroll
@@ -170,15 +289,15 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                 for (int i = 0; i < 16; ++i) stg[lane * 32 + ((16 + i) ^ lane)] = v[i];
                 __syncwarp();
-                const int c8 = (lane & 3) * 8;
 #pragma unroll
                 for (int it = 0; it < 4; ++it) {
                     const int r = it * 8 + (lane >> 2);
                     float a[8];
 #pragma unroll
                     for (int k = 0; k < 8; ++k) a[k] = stg[r * 32 + ((c8 + k) ^ r)];
-                    epilogue_run<EPI, T, 8>(ep, m0 + q * 32 + r, n0 + c + c8, a);
+                    epi_apply<EPI>(ep, m0 + q * 32 + r, n0 + c + c8, a, pf, it);
                 }
+                if (j + 1 < BN / 64) epi_prefetch<EPI>(ep, m0 + q * 32, n0 + c + 32 + c8, lane, pf);
                 __syncwarp();
             }
             tc_fence_before();
