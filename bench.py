@@ -316,8 +316,13 @@ def main():
             "all_blocks": {"ms_per_chunk": ms_all / args.steps, "ms_per_chunk_p50": float(np.median(pc_all)),
                            "chunks_per_s": n_chunks / (ms_all * 1e-3)},
             "speedup_vs_all_blocks": ms_all / ms_x,
-            "predicted_speedup": predicted_speedup(xc, chunk, gate, args, cfg, ms_all / args.steps),
+            "predicted_speedup": None,
             "roofline": roofline, "gpu_launches": int(launches), "clocks": clocks}
+    pred, kernel_us = predicted_speedup(xc, chunk, gate, args, cfg, ms_all / args.steps)
+    line["predicted_speedup"] = pred
+    # warm mean per launch of each kernel kind in the all-blocks arm (us; CUDA events
+    # around each launch of the profiled re-run; "attn" includes the partial merge)
+    line["kernel_us"] = kernel_us
 
     if not args.no_e2e:
         line["e2e"] = e2e(xc, traj, acts, cfg, args, gate, world, dev)
@@ -358,7 +363,13 @@ def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
 
     block_kinds = {"ln", "qkv", "attn", "oproj", "ffn1", "ffn2"}
     t_block = {}
-    for r in run(xb.gate_params(enabled=0)):
+    recs_all = run(xb.gate_params(enabled=0))
+    kernel_us = {}
+    for kind in xb.KERNEL_KINDS:
+        ms = [r["ms"] for r in recs_all if r["kind"] == kind]
+        if ms:
+            kernel_us[kind] = round(1e3 * float(np.mean(ms)), 2)
+    for r in recs_all:
         if r["kind"] in block_kinds:
             key = (r["chunk"], r["pass_seq"] % (S + 1), r["block"])
             t_block[key] = t_block.get(key, 0.0) + r["ms"]
@@ -377,7 +388,7 @@ def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
             saved += t_block.get(key, 0.0) - d["gate"] - d["reuse"]
     saved /= args.steps
     gated /= args.steps
-    return t_all / (t_all - saved + gated)
+    return t_all / (t_all - saved + gated), kernel_us
 
 
 def sweep(args):
