@@ -63,7 +63,7 @@ typedef enum {
  * order.  kv_window_chunks counts ring slots INCLUDING the current chunk.
  * Constraints: d_model = n_heads*head_dim; head_dim % 16 == 0; for XC_BF16
  * head_dim in {64, 128}, d_model % 256 == 0 and d_ffn % 256 == 0;
- * n_blocks <= XC_MAX_BLOCKS; t_freq_dim even. */
+ * n_blocks <= XC_MAX_BLOCKS; t_freq_dim even and <= 512. */
 typedef struct {
     int n_blocks, d_model, n_heads, head_dim, d_ffn, c_latent, action_dim;
     int n_cams, frames, grid_h, grid_w;

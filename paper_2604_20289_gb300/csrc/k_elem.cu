@@ -1,7 +1,7 @@
 // Bandwidth-bound and small kernels of the chunk step: patch embedding,
 // adaLN-Zero LayerNorm modulation, the reuse path (Eq. 4), the conditioning
 // GEMVs, the output head, the Euler update and weight layout conversion.
-#include "xc_common.cuh"
+#include "xc_kernels.cuh"
 
 namespace xc {
 
@@ -140,6 +140,59 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// d <= 512 (one 16-element run per lane): persistent warps walk rows
+// row, row + n_warps, ... with the next row's load in flight while the
+// current one is reduced; the modulation vectors stay in registers.
+template <typename T>
+__global__ void __launch_bounds__(256)
+    ln_mod_row_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
+                      T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
+    if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
+    const int lane = threadIdx.x & 31;
+    const int nw = (gridDim.x * blockDim.x) >> 5;
+    const bool act = lane < d / 16;
+    float sc[16], sh[16], cur[16], nxt[16];
+    if (act) {
+        load16<float>(scale + 16 * lane, sc);
+        load16<float>(shift + 16 * lane, sh);
+    }
+    int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (row < M && act) load16<T>(x + (size_t)row * d + 16 * lane, cur);
+    for (; row < M; row += nw) {
+        const int nrow = row + nw;
+        if (nrow < M && act) load16<T>(x + (size_t)nrow * d + 16 * lane, nxt);
+        Moments mo{0.0f, 0.0f, 0.0f};
+        if (act) {
+            float sum = 0.0f;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) sum += cur[i];
+            mo.n = 16.0f;
+            mo.mean = sum * (1.0f / 16.0f);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) mo.m2 += (cur[i] - mo.mean) * (cur[i] - mo.mean);
+        }
+        mo = warp_moments(mo);
+        const float rstd = rsqrtf(mo.m2 / (float)d + eps);
+        if (act) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) cur[i] = (cur[i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i];
+            store16<T>(out + (size_t)row * d + 16 * lane, cur);
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
+    }
+}
+
+static int n_sm_elem() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    }
+    return n;
+}
+
 template <typename T, int NCH>
 static cudaError_t ln_mod_n(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
                             const uint8_t *skip, cudaStream_t st) {
@@ -151,6 +204,11 @@ template <typename T>
 cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
                    const uint8_t *skip, cudaStream_t st) {
     if (d % 16 != 0) return cudaErrorInvalidValue;
+    if (d <= 512) {
+        const int want = (M + 7) / 8, cap = 2 * n_sm_elem();
+        ln_mod_row_kernel<T><<<want < cap ? want : cap, 256, 0, st>>>(x, shift, scale, out, M, d, eps, skip);
+        return cudaGetLastError();
+    }
     switch ((d + 511) / 512) {
         case 1: return ln_mod_n<T, 1>(x, shift, scale, out, M, d, eps, skip, st);
         case 2: return ln_mod_n<T, 2>(x, shift, scale, out, M, d, eps, skip, st);
@@ -209,72 +267,116 @@ cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_
 }
 
 // ----------------------------------------------------------- conditioning
-// Sinusoidal embedding of the flow time 1000*sigma, computed in double
-// precision (angles reach 1000 rad): e[i] = cos(s f_i), e[half + i] = sin(s f_i),
-// f_i = 10000^(-i/half).
-__global__ void temb_kernel(float sigma, float *__restrict__ e, int dim) {
-    const int half = dim / 2;
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= half) return;
-    const double f = exp(-9.210340371976184 * (double)i / (double)half);   // ln(10000)
-    const double a = 1000.0 * (double)sigma * f;
-    e[i] = (float)cos(a);
-    e[half + i] = (float)sin(a);
-}
-cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st) {
-    temb_kernel<<<(dim / 2 + 127) / 128, 128, 0, st>>>(sigma, e, dim);
-    return cudaGetLastError();
+constexpr int GEMV_WARPS = 16;
+
+// Fused conditioning (a2), three launches per pass:
+//   stage 1: ht = SiLU(W_t1 temb + b_t1), ha = SiLU(W_a1 a + b_a1)
+//   stage 2: e  = (W_t2 ht + b_t2) + (W_a2 ha + b_a2)
+//   stage 3: mods[b] = W_m SiLU(e) + b_m + table_b (every block b),
+//            hmod    = W_h SiLU(e) + b_h + table_head
+// The action and the sinusoidal timestep embedding (computed on the host in
+// double precision, see xc_api.cu) ride in the kernel arguments.  Each CTA
+// owns 32 output columns: the input is staged in shared memory and each of
+// 16 warps keeps eight independent weight rows in flight.
+__device__ __forceinline__ float gemv_col(const float *xs, const float *__restrict__ W, int n_in, int n_out, int j,
+                                          int warp) {
+    float a[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a[k] = 0.0f;
+    const float *wj = W + j;
+    int i = warp;
+    for (; i + 7 * GEMV_WARPS < n_in; i += 8 * GEMV_WARPS) {
+        float w[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[k] = wj[(size_t)(i + k * GEMV_WARPS) * n_out];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) a[k] = fmaf(xs[i + k * GEMV_WARPS], w[k], a[k]);
+    }
+    for (; i < n_in; i += GEMV_WARPS) a[0] = fmaf(xs[i], wj[(size_t)i * n_out], a[0]);
+    return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
 }
 
-// y[j] = act_out( sum_i in(i) W[i][j] + b[j] + add[j] ), W [n_in][n_out].
-// in_silu: in = SiLU(x) instead of x.  act_out 0: none, 1: SiLU.
-// CTA = 32 output columns x 16 warps; the input vector (after SiLU) is
-// staged in shared memory once; warp w sums rows i = w (mod 16), four
-// independent rows per step so that several coalesced 128-byte row segments
-// are in flight per warp; the warps then reduce in shared memory.
-constexpr int GEMV_WARPS = 16;
-__global__ void __launch_bounds__(GEMV_WARPS * 32)
-    gemv_kernel(const float *__restrict__ x, int in_silu, const float *__restrict__ W, const float *__restrict__ b,
-                const float *__restrict__ add, float *__restrict__ y, int n_in, int n_out, int act_out) {
-    extern __shared__ float xs[];                       // [n_in]
+template <int STAGE>
+__global__ void __launch_bounds__(GEMV_WARPS * 32) cond_kernel(const CondArgs c) {
+    extern __shared__ float xs[];
     __shared__ float part[GEMV_WARPS][33];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int i = threadIdx.x; i < n_in; i += blockDim.x) xs[i] = in_silu ? silu(x[i]) : x[i];
-    __syncthreads();
-    const int j = blockIdx.x * 32 + lane;
-    float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
-    if (j < n_out) {
-        const float *wj = W + j;
-        int i = warp;
-        for (; i + 3 * GEMV_WARPS < n_in; i += 4 * GEMV_WARPS) {
-            const float w0 = wj[(size_t)i * n_out];
-            const float w1 = wj[(size_t)(i + GEMV_WARPS) * n_out];
-            const float w2 = wj[(size_t)(i + 2 * GEMV_WARPS) * n_out];
-            const float w3 = wj[(size_t)(i + 3 * GEMV_WARPS) * n_out];
-            a0 = fmaf(xs[i], w0, a0);
-            a1 = fmaf(xs[i + GEMV_WARPS], w1, a1);
-            a2 = fmaf(xs[i + 2 * GEMV_WARPS], w2, a2);
-            a3 = fmaf(xs[i + 3 * GEMV_WARPS], w3, a3);
+    const int d = c.d;
+    const int nb_d = (d + 31) / 32;
+    int j = 0, n_out = d;
+    float acc = 0.0f;
+    if constexpr (STAGE == 1) {
+        const bool tpath = (int)blockIdx.x < nb_d;
+        j = (tpath ? blockIdx.x : blockIdx.x - nb_d) * 32 + lane;
+        const int n_in = tpath ? c.tf : c.A;
+        if (tpath) {
+            for (int i = threadIdx.x; i < c.tf; i += blockDim.x) xs[i] = c.temb[i];
+        } else {
+            for (int i = threadIdx.x; i < c.A; i += blockDim.x) xs[i] = c.act[i];
         }
-        for (; i < n_in; i += GEMV_WARPS) a0 = fmaf(xs[i], wj[(size_t)i * n_out], a0);
-    }
-    part[warp][lane] = (a0 + a1) + (a2 + a3);
-    __syncthreads();
-    if (warp == 0 && j < n_out) {
-        float s = 0.0f;
+        __syncthreads();
+        if (j < d) acc = gemv_col(xs, tpath ? c.t_w1 : c.a_w1, n_in, d, j, warp);
+        part[warp][lane] = acc;
+        __syncthreads();
+        if (warp == 0 && j < d) {
+            float s = 0.0f;
 #pragma unroll
-        for (int w = 0; w < GEMV_WARPS; ++w) s += part[w][lane];
-        s += b[j];
-        if (add != nullptr) s += add[j];
-        y[j] = act_out == 1 ? silu(s) : s;
+            for (int w = 0; w < GEMV_WARPS; ++w) s += part[w][lane];
+            s += (tpath ? c.t_b1 : c.a_b1)[j];
+            (tpath ? c.ht : c.ha)[j] = silu(s);
+        }
+    } else if constexpr (STAGE == 2) {
+        j = blockIdx.x * 32 + lane;
+        for (int i = threadIdx.x; i < d; i += blockDim.x) {
+            xs[i] = c.ht[i];
+            xs[d + i] = c.ha[i];
+        }
+        __syncthreads();
+        if (j < d) acc = gemv_col(xs, c.t_w2, d, d, j, warp) + gemv_col(xs + d, c.a_w2, d, d, j, warp);
+        part[warp][lane] = acc;
+        __syncthreads();
+        if (warp == 0 && j < d) {
+            float s = 0.0f;
+#pragma unroll
+            for (int w = 0; w < GEMV_WARPS; ++w) s += part[w][lane];
+            c.e[j] = s + c.t_b2[j] + c.a_b2[j];
+        }
+    } else {
+        const int nb_m = (6 * d + 31) / 32;
+        const bool mpath = (int)blockIdx.x < nb_m;
+        n_out = mpath ? 6 * d : 2 * d;
+        j = (mpath ? blockIdx.x : blockIdx.x - nb_m) * 32 + lane;
+        for (int i = threadIdx.x; i < d; i += blockDim.x) xs[i] = silu(c.e[i]);
+        __syncthreads();
+        if (j < n_out) acc = gemv_col(xs, mpath ? c.mod_w : c.head_w, d, n_out, j, warp);
+        part[warp][lane] = acc;
+        __syncthreads();
+        if (warp == 0 && j < n_out) {
+            float s = 0.0f;
+#pragma unroll
+            for (int w = 0; w < GEMV_WARPS; ++w) s += part[w][lane];
+            if (mpath) {
+                s += c.mod_b[j];
+                for (int b = 0; b < c.B; ++b) c.mods[(size_t)b * 6 * d + j] = s + c.blk_mod[(size_t)b * 6 * d + j];
+            } else {
+                c.hmod[j] = s + c.head_b[j] + c.head_tab[j];
+            }
+        }
     }
 }
 
-cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
-                 int n_out, int act_out, cudaStream_t st) {
-    const size_t smem = (size_t)n_in * sizeof(float);
-    if (smem > 48 * 1024) return cudaErrorInvalidValue;
-    gemv_kernel<<<(n_out + 31) / 32, GEMV_WARPS * 32, smem, st>>>(x, in_silu, W, b, add, y, n_in, n_out, act_out);
+cudaError_t conditioning(const CondArgs &c, cudaStream_t st) {
+    const int d = c.d, nb_d = (d + 31) / 32;
+    if (c.A < 1 || c.A > 8 || c.tf < 2 || c.tf > COND_TEMB_MAX || (size_t)2 * d * sizeof(float) > 48 * 1024)
+        return cudaErrorInvalidValue;
+    const int in1 = c.tf > c.A ? c.tf : c.A;
+    cond_kernel<1><<<2 * nb_d, GEMV_WARPS * 32, in1 * sizeof(float), st>>>(c);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    cond_kernel<2><<<nb_d, GEMV_WARPS * 32, 2 * d * sizeof(float), st>>>(c);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    cond_kernel<3><<<(6 * d + 31) / 32 + (2 * d + 31) / 32, GEMV_WARPS * 32, d * sizeof(float), st>>>(c);
     return cudaGetLastError();
 }
 
@@ -305,19 +407,6 @@ __global__ void rope_table_kernel(int hd, double theta, int frame0, int4 npos, f
 }
 cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out, int n, cudaStream_t st) {
     rope_table_kernel<<<(n + 127) / 128, 128, 0, st>>>(hd, theta, frame0, npos, out, n);
-    return cudaGetLastError();
-}
-
-// mods_all[b][j][c] = m[j*d + c] + blk_mod[b][j][c]   (B x 6 x d)
-__global__ void assemble_mods_kernel(const float *__restrict__ m, const float *__restrict__ tab,
-                                     float *__restrict__ out, int B, int d) {
-    const long i = blockIdx.x * (long)blockDim.x + threadIdx.x;
-    if (i >= (long)B * 6 * d) return;
-    out[i] = m[i % (6 * d)] + tab[i];
-}
-cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, int d, cudaStream_t st) {
-    const long n = (long)B * 6 * d;
-    assemble_mods_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(m, tab, out, B, d);
     return cudaGetLastError();
 }
 

@@ -117,8 +117,8 @@ struct xc_ctx {
 
     // activations / conditioning
     void *xb[2], *x1, *hbuf, *q, *o, *u;
-    float *lat, *vout, *act_dev;
-    float *temb, *ht, *ha, *e1, *e, *mshared, *mods, *hmod;
+    float *lat, *vout;
+    float *ht, *ha, *e, *mods, *hmod;
 
     // rolling KV ring [B][Wkv][L][d] and caches
     void *ring_k, *ring_v;
@@ -216,7 +216,8 @@ bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
     if (c->n_cams < 1 || c->frames < 1 || c->grid_h < 1 || c->grid_w < 1) return bad("empty latent grid");
     if ((long long)c->n_cams * c->frames * c->grid_h * c->grid_w > (1LL << 24)) return bad("chunk too large");
     if (c->kv_window_chunks < 1 || c->n_denoise_steps < 1 || c->n_denoise_steps > 64) return bad("window / steps");
-    if (c->t_freq_dim < 2 || c->t_freq_dim % 2 != 0) return bad("t_freq_dim must be even");
+    if (c->t_freq_dim < 2 || c->t_freq_dim % 2 != 0 || c->t_freq_dim > COND_TEMB_MAX)
+        return bad("t_freq_dim must be even and at most 512");
     if (!(c->ln_eps > 0.0f) || !(c->rope_theta > 1.0f)) return bad("ln_eps / rope_theta");
     if (c->dtype == XC_BF16) {
         if (c->head_dim != 64 && c->head_dim != 128) return bad("bf16 needs head_dim 64 or 128");
@@ -349,19 +350,27 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     ctx->cur_keys = n_keys;
 
     // conditioning c_t: timestep + action embeddings -> adaLN-Zero vectors
-    CK(cudaMemcpyAsync(ctx->act_dev, action, ctx->A * sizeof(float), cudaMemcpyHostToDevice, st));
     {
-        const int pi = prof_begin(ctx, XC_K_COND, -1);
-        CK(timestep_embedding(sigma, ctx->temb, ctx->cfg.t_freq_dim, st));
-        CK(gemv(ctx->temb, 0, ctx->t_w1, ctx->t_b1, nullptr, ctx->ht, ctx->cfg.t_freq_dim, d, 1, st));
-        CK(gemv(ctx->act_dev, 0, ctx->a_w1, ctx->a_b1, nullptr, ctx->ha, ctx->A, d, 1, st));
-        CK(gemv(ctx->ht, 0, ctx->t_w2, ctx->t_b2, nullptr, ctx->e1, d, d, 0, st));
-        CK(gemv(ctx->ha, 0, ctx->a_w2, ctx->a_b2, ctx->e1, ctx->e, d, d, 0, st));
-        CK(gemv(ctx->e, 1, ctx->mod_w, ctx->mod_b, nullptr, ctx->mshared, d, 6 * d, 0, st));
-        CK(gemv(ctx->e, 1, ctx->head_w, ctx->head_b, ctx->head_tab, ctx->hmod, d, 2 * d, 0, st));
-        CK(assemble_mods(ctx->mshared, ctx->blk_mod, ctx->mods, B, d, st));
-        prof_end(ctx, pi);
-        ctx->launches += 8;
+        CondArgs ca{};
+        // sinusoid of the flow time 1000 sigma: [cos(s f_i), sin(s f_i)],
+        // f_i = 10000^(-i/half), in double precision (angles reach 1000 rad)
+        const int half = ctx->cfg.t_freq_dim / 2;
+        for (int i = 0; i < half; ++i) {
+            const double a = 1000.0 * (double)sigma * std::exp(-std::log(10000.0) * (double)i / (double)half);
+            ca.temb[i] = (float)std::cos(a);
+            ca.temb[half + i] = (float)std::sin(a);
+        }
+        for (int i = 0; i < ctx->A; ++i) ca.act[i] = action[i];
+        ca.A = ctx->A;
+        ca.tf = ctx->cfg.t_freq_dim;
+        ca.d = d;
+        ca.B = B;
+        ca.t_w1 = ctx->t_w1; ca.t_b1 = ctx->t_b1; ca.a_w1 = ctx->a_w1; ca.a_b1 = ctx->a_b1;
+        ca.t_w2 = ctx->t_w2; ca.t_b2 = ctx->t_b2; ca.a_w2 = ctx->a_w2; ca.a_b2 = ctx->a_b2;
+        ca.mod_w = ctx->mod_w; ca.mod_b = ctx->mod_b; ca.blk_mod = ctx->blk_mod;
+        ca.head_w = ctx->head_w; ca.head_b = ctx->head_b; ca.head_tab = ctx->head_tab;
+        ca.ht = ctx->ht; ca.ha = ctx->ha; ca.e = ctx->e; ca.mods = ctx->mods; ca.hmod = ctx->hmod;
+        LAUNCH(XC_K_COND, -1, 3, conditioning(ca, st));
     }
 
     T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
@@ -674,13 +683,9 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->u = dalloc<void>(ctx, (size_t)L * F * es);
         ctx->lat = dalloc<float>(ctx, (size_t)L * C * sizeof(float));
         ctx->vout = dalloc<float>(ctx, (size_t)L * C * sizeof(float));
-        ctx->act_dev = dalloc<float>(ctx, 8 * sizeof(float));
-        ctx->temb = dalloc<float>(ctx, Tf * sizeof(float));
         ctx->ht = dalloc<float>(ctx, d * sizeof(float));
         ctx->ha = dalloc<float>(ctx, d * sizeof(float));
-        ctx->e1 = dalloc<float>(ctx, d * sizeof(float));
         ctx->e = dalloc<float>(ctx, d * sizeof(float));
-        ctx->mshared = dalloc<float>(ctx, 6 * (size_t)d * sizeof(float));
         ctx->mods = dalloc<float>(ctx, (size_t)B * 6 * d * sizeof(float));
         ctx->hmod = dalloc<float>(ctx, 2 * (size_t)d * sizeof(float));
 

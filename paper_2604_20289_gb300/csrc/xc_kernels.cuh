@@ -54,10 +54,17 @@ cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, i
 template <typename T>
 cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t *skip, int n_sm, cudaStream_t st);
 cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_t st);
-cudaError_t timestep_embedding(float sigma, float *e, int dim, cudaStream_t st);
-cudaError_t gemv(const float *x, int in_silu, const float *W, const float *b, const float *add, float *y, int n_in,
-                 int n_out, int act_out, cudaStream_t st);
-cudaError_t assemble_mods(const float *m, const float *tab, float *out, int B, int d, cudaStream_t st);
+// Fused conditioning (three launches), see k_elem.cu.
+constexpr int COND_TEMB_MAX = 512;
+struct CondArgs {
+    float temb[COND_TEMB_MAX];    // sinusoidal embedding of 1000 sigma (host, double precision)
+    float act[8];
+    int A, tf, d, B;
+    const float *t_w1, *t_b1, *a_w1, *a_b1, *t_w2, *t_b2, *a_w2, *a_b2;
+    const float *mod_w, *mod_b, *blk_mod, *head_w, *head_b, *head_tab;
+    float *ht, *ha, *e, *mods, *hmod;
+};
+cudaError_t conditioning(const CondArgs &c, cudaStream_t st);
 template <typename T>
 cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
                  cudaStream_t st);
