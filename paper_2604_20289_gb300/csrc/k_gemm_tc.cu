@@ -346,41 +346,62 @@ bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t co
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int EPI>
+static int gemm_sm_count() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    }
+    return n;
+}
+
+// Output tile width for an M x N GEMM: 256, unless 128 x 256 tiles would
+// leave SMs idle (fewer tiles than SMs) and N allows 128-wide tiles.
+int gemm_tc_bn(int M, int N) {
+    const long tiles256 = (long)((M + GEMM_BM - 1) / GEMM_BM) * (N / 256);
+    return (N % 256 != 0 || (tiles256 < gemm_sm_count() && N % 128 == 0)) ? 128 : 256;
+}
+
+template <int EPI, int BN>
 static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
                              const uint8_t *skip, int *err, cudaStream_t st) {
-    constexpr int BN = 256;
     using G = GemmTile<BN>;
     auto kern = gemm_tc_kernel<BN, EPI, bf16>;
     static bool attr_set = false;
-    static int n_sm = 0;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM_BYTES);
         if (e != cudaSuccess) return e;
-        int dev = 0;
-        e = cudaGetDevice(&dev);
-        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-        if (e != cudaSuccess) return e;
         attr_set = true;
     }
+    const int n_sm = gemm_sm_count();
     const int n_tiles = (ep.N / BN) * ((ep.M + GEMM_BM - 1) / GEMM_BM);
     const int grid = n_tiles < n_sm ? n_tiles : n_sm;
     kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
     return cudaGetLastError();
 }
 
-// Entry used by the chunk step and xc_op_linear / xc_op_qkv_rope (bf16 only).
-// `ta` covers A [M][K], `tb` covers Wt [N][K]; N % 256 == 0, K % 64 == 0.
-cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
-                    const uint8_t *skip, int *err, cudaStream_t st) {
+template <int BN>
+static cudaError_t gemm_tc_bn_(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+                               const uint8_t *skip, int *err, cudaStream_t st) {
     switch (epi) {
-        case EPI_BIAS: return launch_tc<EPI_BIAS>(ta, tb, ep, K, skip, err, st);
-        case EPI_GELU: return launch_tc<EPI_GELU>(ta, tb, ep, K, skip, err, st);
-        case EPI_RESID_GATE: return launch_tc<EPI_RESID_GATE>(ta, tb, ep, K, skip, err, st);
-        case EPI_RESID_CACHE: return launch_tc<EPI_RESID_CACHE>(ta, tb, ep, K, skip, err, st);
-        case EPI_QKV_ROPE: return launch_tc<EPI_QKV_ROPE>(ta, tb, ep, K, skip, err, st);
+        case EPI_BIAS: return launch_tc<EPI_BIAS, BN>(ta, tb, ep, K, skip, err, st);
+        case EPI_GELU: return launch_tc<EPI_GELU, BN>(ta, tb, ep, K, skip, err, st);
+        case EPI_RESID_GATE: return launch_tc<EPI_RESID_GATE, BN>(ta, tb, ep, K, skip, err, st);
+        case EPI_RESID_CACHE: return launch_tc<EPI_RESID_CACHE, BN>(ta, tb, ep, K, skip, err, st);
+        case EPI_QKV_ROPE: return launch_tc<EPI_QKV_ROPE, BN>(ta, tb, ep, K, skip, err, st);
         default: return cudaErrorInvalidValue;
     }
+}
+
+// Entry used by the chunk step and xc_op_linear / xc_op_qkv_rope (bf16 only).
+// `ta` covers A [M][K] (box 128 rows), `tb` covers Wt [N][K] with box rows
+// = bn (gemm_tc_bn(M, N)); N % bn == 0, K % 64 == 0.
+cudaError_t gemm_tc(int epi, int bn, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+                    const uint8_t *skip, int *err, cudaStream_t st) {
+    if (bn == 256) return gemm_tc_bn_<256>(epi, ta, tb, ep, K, skip, err, st);
+    if (bn == 128) return gemm_tc_bn_<128>(epi, ta, tb, ep, K, skip, err, st);
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace xc

@@ -146,8 +146,9 @@ struct xc_ctx {
     void *attn_ws;
     size_t attn_ws_bytes;
 
-    // tensor maps (bf16)
+    // tensor maps (bf16); output tile width of each GEMM
     CUtensorMap tm_h, tm_o, tm_u, tm_q;
+    int bn_qkv, bn_o, bn_f1, bn_f2;
     std::vector<CUtensorMap> tm_wqkv, tm_wo, tm_w1, tm_w2, tm_rk, tm_rv;
 
     int n, next_step;
@@ -457,7 +458,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.rope_off = ctx->rope_off;
         ep.rope_cs = ctx->rope_cs;
         if constexpr (sizeof(T) == 2) {
-            LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->bn_qkv, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
             int n_attn = 1;
             LAUNCH(XC_K_ATTN, b, n_attn,
                    attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L, n_keys,
@@ -479,7 +480,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.resid = xin;
         ep.out = x1;
         if constexpr (sizeof(T) == 2) {
-            LAUNCH(XC_K_OPROJ, b, 1, gemm_tc(EPI_RESID_GATE, ctx->tm_o, ctx->tm_wo[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_OPROJ, b, 1, gemm_tc(EPI_RESID_GATE, ctx->bn_o, ctx->tm_o, ctx->tm_wo[b], ep, d, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->o_wt) + (size_t)b * d * d;
             LAUNCH(XC_K_OPROJ, b, 1, gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
@@ -492,7 +493,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.bias = ctx->f1_b + (size_t)b * F;
         ep.out = ub;
         if constexpr (sizeof(T) == 2) {
-            LAUNCH(XC_K_FFN1, b, 1, gemm_tc(EPI_GELU, ctx->tm_h, ctx->tm_w1[b], ep, d, flag, ctx->d_err, st));
+            LAUNCH(XC_K_FFN1, b, 1, gemm_tc(EPI_GELU, ctx->bn_f1, ctx->tm_h, ctx->tm_w1[b], ep, d, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->f1_wt) + (size_t)b * F * d;
             LAUNCH(XC_K_FFN1, b, 1, gemm_simt(EPI_GELU, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
@@ -508,7 +509,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.out = xout;
         ep.rhat = rh;
         if constexpr (sizeof(T) == 2) {
-            LAUNCH(XC_K_FFN2, b, 1, gemm_tc(EPI_RESID_CACHE, ctx->tm_u, ctx->tm_w2[b], ep, F, flag, ctx->d_err, st));
+            LAUNCH(XC_K_FFN2, b, 1, gemm_tc(EPI_RESID_CACHE, ctx->bn_f2, ctx->tm_u, ctx->tm_w2[b], ep, F, flag, ctx->d_err, st));
         } else {
             const float *W = reinterpret_cast<const float *>(ctx->f2_wt) + (size_t)b * d * F;
             LAUNCH(XC_K_FFN2, b, 1, gemm_simt(EPI_RESID_CACHE, ep, reinterpret_cast<const float *>(ub), W, F, flag, st));
@@ -719,6 +720,10 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
 
         // tensor maps of the bf16 path
         if (ctx->bf) {
+            ctx->bn_qkv = gemm_tc_bn(L, 3 * d);
+            ctx->bn_o = gemm_tc_bn(L, d);
+            ctx->bn_f1 = gemm_tc_bn(L, F);
+            ctx->bn_f2 = gemm_tc_bn(L, d);
             tmap(ctx, &ctx->tm_h, ctx->hbuf, L, d, 128);
             tmap(ctx, &ctx->tm_o, ctx->o, L, d, 128);
             tmap(ctx, &ctx->tm_u, ctx->u, L, F, 128);
@@ -734,10 +739,10 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
                 const char *wo = reinterpret_cast<const char *>(ctx->o_wt) + (size_t)b * d * d * es;
                 const char *w1 = reinterpret_cast<const char *>(ctx->f1_wt) + (size_t)b * F * d * es;
                 const char *w2 = reinterpret_cast<const char *>(ctx->f2_wt) + (size_t)b * d * F * es;
-                tmap(ctx, &ctx->tm_wqkv[b], wq, 3 * (uint64_t)d, d, 256);
-                tmap(ctx, &ctx->tm_wo[b], wo, d, d, 256);
-                tmap(ctx, &ctx->tm_w1[b], w1, F, d, 256);
-                tmap(ctx, &ctx->tm_w2[b], w2, d, F, 256);
+                tmap(ctx, &ctx->tm_wqkv[b], wq, 3 * (uint64_t)d, d, ctx->bn_qkv);
+                tmap(ctx, &ctx->tm_wo[b], wo, d, d, ctx->bn_o);
+                tmap(ctx, &ctx->tm_w1[b], w1, F, d, ctx->bn_f1);
+                tmap(ctx, &ctx->tm_w2[b], w2, d, F, ctx->bn_f2);
                 const char *rk = reinterpret_cast<const char *>(ctx->ring_k) + (size_t)b * ctx->Wkv * Ld * es;
                 const char *rv = reinterpret_cast<const char *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld * es;
                 tmap(ctx, &ctx->tm_rk[b], rk, (uint64_t)ctx->Wkv * L, d, 128);
@@ -1038,9 +1043,10 @@ xc_status xc_op_linear(int dtype, int epilogue, int M, int N, int K, const void 
     if (dtype == XC_BF16) {
         if (N % 256 != 0 || K % 64 != 0) OP_FAIL(XC_EINVAL, "xc_op_linear: bf16 needs N %% 256 == 0, K %% 64 == 0");
         CUtensorMap ta, tb;
-        if (!make_tmap_bf16(&ta, A, M, K, 128) || !make_tmap_bf16(&tb, Wt, N, K, 256))
+        const int bn = gemm_tc_bn(M, N);
+        if (!make_tmap_bf16(&ta, A, M, K, 128) || !make_tmap_bf16(&tb, Wt, N, K, bn))
             OP_FAIL(XC_EINVAL, "xc_op_linear: tensor map (alignment?)");
-        OP_CK(gemm_tc(epilogue, ta, tb, ep, K, nullptr, op_err_word(), st));
+        OP_CK(gemm_tc(epilogue, bn, ta, tb, ep, K, nullptr, op_err_word(), st));
     } else if (dtype == XC_F32) {
         if (N % 16 != 0) OP_FAIL(XC_EINVAL, "xc_op_linear: f32 needs N %% 16 == 0");
         OP_CK(gemm_simt(epilogue, ep, reinterpret_cast<const float *>(A), reinterpret_cast<const float *>(Wt), K,
@@ -1104,9 +1110,10 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
     if (dtype == XC_BF16) {
         if ((3 * d) % 256 != 0 || d % 64 != 0) OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: bf16 needs 3d %% 256, d %% 64");
         CUtensorMap ta, tb;
-        if (!make_tmap_bf16(&ta, A, M, d, 128) || !make_tmap_bf16(&tb, Wt, 3 * (uint64_t)d, d, 256))
+        const int bn = gemm_tc_bn(M, 3 * d);
+        if (!make_tmap_bf16(&ta, A, M, d, 128) || !make_tmap_bf16(&tb, Wt, 3 * (uint64_t)d, d, bn))
             OP_FAIL(XC_EINVAL, "xc_op_qkv_rope: tensor map");
-        OP_CK(gemm_tc(EPI_QKV_ROPE, ta, tb, ep, d, nullptr, op_err_word(), st));
+        OP_CK(gemm_tc(EPI_QKV_ROPE, bn, ta, tb, ep, d, nullptr, op_err_word(), st));
     } else if (dtype == XC_F32) {
         OP_CK(gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(A), reinterpret_cast<const float *>(Wt), d,
                         nullptr, st));

@@ -36,7 +36,8 @@ struct GateArgs {
 size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off);
 template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);
 bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
-cudaError_t gemm_tc(int epi, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
+int gemm_tc_bn(int M, int N);
+cudaError_t gemm_tc(int epi, int bn, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
                     const uint8_t *skip, int *err, cudaStream_t st);
 cudaError_t attn_tc(int head_dim, const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv, bf16 *o,
                     int Lq, int n_keys, int n_heads, int d, void *ws, size_t ws_bytes, const uint8_t *skip, int *err,
