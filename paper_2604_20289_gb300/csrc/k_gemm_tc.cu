@@ -8,37 +8,63 @@
 //   warp 0, lane 0 : TMA producer, STAGES-deep ring of (A 128x64, B BNx64)
 //                    tiles in 128B-swizzled shared memory, continuous across
 //                    output tiles;
-//   warp 1         : allocates TMEM (two BN-column accumulators); lane 0
-//                    issues tcgen05.mma (M=128, N=BN, K=16; 4 per 64-wide
-//                    k-tile) into the free accumulator and commits each stage
-//                    back to the producer;
-//   warps 2..9     : epilogue -- tcgen05.ld of their 32-lane TMEM quadrant
-//                    (two warps per quadrant, half of the columns each),
-//                    fused bias / GELU / gated residual / residual-cache /
-//                    RoPE, vectorised stores; then they release the
-//                    accumulator, so the epilogue of tile i overlaps the
-//                    main loop of tile i + 1.
+//   warp 1         : allocates TMEM (two BN-column accumulators) and issues
+//                    tcgen05.mma (M=128, N=BN, K=16; 4 per 64-wide k-tile)
+//                    into the free accumulator from a converged warp;
+//   warps 2..9     : epilogue, two warps per TMEM lane quadrant, half of the
+//                    columns each, in 32 x 32 blocks: thread = row, the
+//                    block's residual operands arrive in shared memory by
+//                    TMA, the fused epilogue (bias / GELU / gated residual /
+//                    residual cache / RoPE) runs in registers, and the bf16
+//                    block leaves by a TMA store from a 64B-swizzled staging
+//                    buffer.  The accumulator is released after its last
+//                    TMEM read, so the epilogue of tile i overlaps the main
+//                    loop of tile i + 1.
 // The skip flag of the block lets the whole recompute path early-exit when
 // the gate chose reuse (Eq. 4), so decisions never return to the host.
+#include <cstring>
+#include <mutex>
+#include <unordered_map>
+
 #include "xc_ptx.cuh"
 
 namespace xc {
 
 constexpr int GEMM_BM = 128;
 constexpr int GEMM_BK = 64;
+constexpr int GEMM_SMEM_LIMIT = 232448;        // dynamic shared memory per CTA on this part
+constexpr int EPI_BLOCK_BYTES = 32 * 32 * 2;   // one 32 x 32 bf16 block
 
-template <int BN>
+// Staging blocks per epilogue warp: residual cache: out, r_hat, resid, x_in;
+// gated residual: out, resid; the others: out, double-buffered.
+template <int EPI>
+__host__ __device__ constexpr int epi_blocks() {
+    return EPI == EPI_RESID_CACHE ? 4 : 2;
+}
+
+template <int BN, int EPI>
 struct GemmTile {
-    static constexpr int STAGES = BN == 256 ? 4 : 6;
     static constexpr int A_BYTES = GEMM_BM * GEMM_BK * 2;
     static constexpr int B_BYTES = BN * GEMM_BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGE_EPI = STAGES * STAGE_BYTES;       // 8 warps x [32 rows][32 fp32]
-    static constexpr int EPI_BYTES = 8 * 32 * 32 * 4;
-    static constexpr int BAR_OFFSET = STAGE_EPI + EPI_BYTES;
-    static constexpr int SMEM_BYTES = BAR_OFFSET + 256 + 1024;   // barriers + alignment slack
-    static constexpr int TMEM_COLS = 2 * BN;                      // double-buffered accumulator
+    static constexpr int EPI_BYTES = 8 * epi_blocks<EPI>() * EPI_BLOCK_BYTES;
+    static constexpr int BAR_BYTES = 512;
+    static constexpr int FIT = (GEMM_SMEM_LIMIT - 1024 - BAR_BYTES - EPI_BYTES) / STAGE_BYTES;
+    static constexpr int STAGES = FIT > 6 ? 6 : FIT;
+    static constexpr int OFF_EPI = STAGES * STAGE_BYTES;                // 1024-aligned
+    static constexpr int BAR_OFFSET = OFF_EPI + EPI_BYTES;
+    static constexpr int SMEM_BYTES = BAR_OFFSET + BAR_BYTES + 1024;   // + alignment slack
+    static constexpr int TMEM_COLS = 2 * BN;                             // double-buffered accumulator
     static constexpr int EPI_THREADS = 256;
+    static_assert(STAGES >= 3, "main-loop ring too shallow");
+    static_assert(SMEM_BYTES <= GEMM_SMEM_LIMIT, "shared memory");
+};
+
+// Tensor maps of the epilogue (32 x 32 bf16 boxes, 64-byte swizzle):
+// out[0..2] = q, k, v for the QKV epilogue, out[0] otherwise.
+struct EpiMaps {
+    CUtensorMap out[3];
+    CUtensorMap rhat, resid, xin;
 };
 
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
@@ -46,122 +72,56 @@ __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
     return p + ((1024u - (s & 1023u)) & 1023u);
 }
 
-// Epilogue operands of one 32-column block of a warp: the thread owns rows
-// r = it * 8 + lane / 4 (it = 0..3) of its 32-row quadrant and the 8 columns
-// [col, col + 8).  They are loaded into registers ahead of use (bf16 path).
-template <int EPI>
-struct EpiPrefetch {
-    float bias[8];
-    float gate[8];
-    uint4 resid[4];
-    uint4 xin[4];
-    float2 cs[4][4];      // RoPE (cos, sin) of the 4 pairs, per row
-};
+// Byte offset of 16-byte chunk k (0..3) of row r in a 64B-swizzled 32 x 32
+// bf16 block (the layout TMA reads and writes with CU_TENSOR_MAP_SWIZZLE_64B).
+__device__ __forceinline__ uint32_t sw64(int r, int k) { return (uint32_t)(r * 64 + ((k ^ ((r >> 1) & 3)) << 4)); }
 
-__device__ __forceinline__ uint4 ld_u4(const void *p) { return *reinterpret_cast<const uint4 *>(p); }
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *tm, const void *src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];"
+                 ::"l"(reinterpret_cast<uint64_t>(tm)), "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-template <int EPI>
-__device__ __forceinline__ void epi_prefetch(const EpiParams &p, int row0, int col, int lane, EpiPrefetch<EPI> &f) {
-    loadW<float, 8>(p.bias + col, f.bias);
-    if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
-        loadW<float, 8>(p.gate + col, f.gate);
+// 32 bf16 of row r from a swizzled block -> float
+__device__ __forceinline__ void read_row32(const uint8_t *blk, int r, float (&v)[32]) {
 #pragma unroll
-        for (int it = 0; it < 4; ++it) {
-            const int row = row0 + it * 8 + (lane >> 2);
-            if (row < p.M) {
-                f.resid[it] = ld_u4(reinterpret_cast<const bf16 *>(p.resid) + (size_t)row * p.N + col);
-                if constexpr (EPI == EPI_RESID_CACHE)
-                    if (p.rhat != nullptr) f.xin[it] = ld_u4(reinterpret_cast<const bf16 *>(p.xin) + (size_t)row * p.N + col);
-            }
-        }
-    }
-    if constexpr (EPI == EPI_QKV_ROPE) {
-        const int part = col / p.d;
-        const int c = col - part * p.d;
-        if (part < 2) {
-            const int pair0 = (c % p.head_dim) >> 1;
-            int off[4], axis[4];
+    for (int k = 0; k < 4; ++k) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(blk + sw64(r, k));
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                off[j] = p.rope_off[pair0 + j];
-                axis[j] = p.rope_axis[pair0 + j];
-            }
-#pragma unroll
-            for (int it = 0; it < 4; ++it) {
-                const int row = row0 + it * 8 + (lane >> 2);
-                if (row < p.M) {
-                    const int cam = row / p.npc;
-                    const int rem = row - cam * p.npc;
-                    const int pos[4] = {cam, rem / (p.gh * p.gw), (rem / p.gw) % p.gh, rem % p.gw};
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) f.cs[it][j] = p.rope_cs[off[j] + pos[axis[j]]];
-                }
-            }
+        for (int j = 0; j < 4; ++j) {
+            const float2 t = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
+            v[8 * k + 2 * j] = t.x;
+            v[8 * k + 2 * j + 1] = t.y;
         }
     }
 }
-
-__device__ __forceinline__ void unpack8(uint4 u, float (&v)[8]) {
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+// float -> 32 bf16 (round to nearest) into row r of a swizzled block
+__device__ __forceinline__ void write_row32(uint8_t *blk, int r, const float (&v)[32]) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const float2 t = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
-        v[2 * j] = t.x;
-        v[2 * j + 1] = t.y;
+    for (int k = 0; k < 4; ++k) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(v[8 * k + 2 * j], v[8 * k + 2 * j + 1]);
+            w[j] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(blk + sw64(r, k)) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
-// Same arithmetic as epilogue_run<EPI, bf16, 8> on prefetched operands.
-template <int EPI>
-__device__ __forceinline__ void epi_apply(const EpiParams &p, int row, int col, float (&acc)[8],
-                                          const EpiPrefetch<EPI> &f, int it) {
-    if (row >= p.M) return;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) acc[i] += f.bias[i];
-    const size_t off = (size_t)row * p.N + col;
-    if constexpr (EPI == EPI_BIAS) {
-        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
-    } else if constexpr (EPI == EPI_GELU) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = gelu_tanh_approx(acc[i]);
-        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
-    } else if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) {
-        float r[8];
-        unpack8(f.resid[it], r);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = r[i] + f.gate[i] * acc[i];
-        storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.out) + off, acc);
-        if constexpr (EPI == EPI_RESID_CACHE) {
-            if (p.rhat != nullptr) {
-                float xi[8];
-                unpack8(f.xin[it], xi);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i] = round_to<bf16>(acc[i]) - xi[i];
-                storeW<bf16, 8>(reinterpret_cast<bf16 *>(p.rhat) + off, acc);
-            }
-        }
-    } else if constexpr (EPI == EPI_QKV_ROPE) {
-        const int part = col / p.d;
-        const int c = col - part * p.d;
-        if (part < 2) {
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float2 t = f.cs[it][j];
-                const float x0 = acc[2 * j], x1 = acc[2 * j + 1];
-                acc[2 * j] = x0 * t.x - x1 * t.y;
-                acc[2 * j + 1] = x0 * t.y + x1 * t.x;
-            }
-        }
-        bf16 *dst = reinterpret_cast<bf16 *>(part == 0 ? p.out : (part == 1 ? p.out_k : p.out_v));
-        storeW<bf16, 8>(dst + (size_t)row * p.d + c, acc);
-    }
-}
-
-template <int BN, int EPI, typename T>
+template <int BN, int EPI>
 __global__ void __launch_bounds__(320, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const EpiParams ep, const int K, const uint8_t *__restrict__ skip_flag, int *err) {
-    using G = GemmTile<BN>;
+                   const __grid_constant__ EpiMaps em, const EpiParams ep, const int K,
+                   const uint8_t *__restrict__ skip_flag, int *err) {
+    using G = GemmTile<BN, EPI>;
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = align1024(smem_raw);
@@ -169,7 +129,8 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t *empty = full + G::STAGES;
     uint64_t *acc_full = empty + G::STAGES;    // [2]
     uint64_t *acc_empty = acc_full + 2;        // [2]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
+    uint64_t *ld_bar = acc_empty + 2;          // [8] residual operands of an epilogue warp landed
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(ld_bar + 8);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int KT = K / GEMM_BK;
@@ -185,6 +146,7 @@ __global__ void __launch_bounds__(320, 1)
             mbar_init(&acc_full[b], 1);
             mbar_init(&acc_empty[b], G::EPI_THREADS);
         }
+        for (int w = 0; w < 8; ++w) mbar_init(&ld_bar[w], 1);
         mbar_fence_init();
     }
     if (warp == 1) tmem_alloc(tmem_slot, G::TMEM_COLS);
@@ -254,55 +216,152 @@ __global__ void __launch_bounds__(320, 1)
             }
         }
     } else {
-        // warps 2..9: two warps per TMEM lane quadrant, each half of the columns.
-        // Each 32-row x 32-column block goes TMEM -> registers (thread = row) ->
-        // XOR-swizzled shared memory -> registers (4 lanes per row, 8 columns
-        // each), so the epilogue's global loads and stores are row-contiguous.
-        const int q = warp & 3;   // TMEM lane quadrant this warp may access
-        const int half = (warp - 2) >> 2;
+        // ---------------------------------------------------------- epilogue
+        // Warp ew = warp - 2 owns TMEM lane quadrant q (rows q*32 .. q*32+31 of
+        // the tile; thread = row) and column half `half`, in 32-column blocks.
+        constexpr bool RES = EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE;
+        constexpr bool CACHE = EPI == EPI_RESID_CACHE;
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int half = ew >> 2;
         const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
-        float *stg = reinterpret_cast<float *>(smem + G::STAGE_EPI) + (warp - 2) * 32 * 32;
+        uint8_t *eb = smem + G::OFF_EPI + ew * epi_blocks<EPI>() * EPI_BLOCK_BYTES;
+        uint8_t *s_out0 = eb;
+        uint8_t *s_aux = eb + EPI_BLOCK_BYTES;          // r_hat (cache) / resid (gate) / second out
+        uint8_t *s_res = CACHE ? eb + 2 * EPI_BLOCK_BYTES : s_aux;
+        uint8_t *s_xin = eb + 3 * EPI_BLOCK_BYTES;
+        uint64_t *lb = &ld_bar[ew];
+        const bool has_rhat = CACHE && ep.rhat != nullptr;
+        const uint32_t ld_bytes = (uint32_t)EPI_BLOCK_BYTES * (has_rhat ? 2u : 1u);
+        uint32_t n_ld = 0;                               // TMA loads issued on lb (its phases)
+        int n_st = 0;                                    // staging blocks written (out double-buffering)
+        auto load_res = [&](int m0, int col) {           // resid (+ x_in) block -> shared memory
+            if (lane == 0) {
+                mbar_expect_tx(lb, ld_bytes);
+                tma_load_2d(s_res, &em.resid, lb, col, m0 + q * 32);
+                if (has_rhat) tma_load_2d(s_xin, &em.xin, lb, col, m0 + q * 32);
+            }
+            ++n_ld;
+        };
         int local = 0;
-        for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++local) {
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++local) {
             const int buf = local & 1;
             const uint32_t use = (uint32_t)(local >> 1);
             const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
-            const int c8 = (lane & 3) * 8;
-            // The global operands of this warp's first column block are
-            // requested before the accumulator is ready; those of block
-            // j + 1 right after block j is stored, so they are in flight
-            // while block j + 1 comes out of TMEM.
-            EpiPrefetch<EPI> pf;
-            epi_prefetch<EPI>(ep, m0 + q * 32, n0 + half * (BN / 2) + c8, lane, pf);
-            const bool ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
+            const int row = m0 + q * 32 + lane;
+            if constexpr (RES) load_res(m0, n0 + half * (BN / 2));
+            // RoPE position of this thread's row (camera, frame, h, w), once per tile
+            int pos0 = 0, pos1 = 0, pos2 = 0, pos3 = 0;
+            if constexpr (EPI == EPI_QKV_ROPE) {
+                pos0 = row / ep.npc;
+                const int rem = row - pos0 * ep.npc;
+                pos1 = rem / (ep.gh * ep.gw);
+                pos2 = (rem / ep.gw) % ep.gh;
+                pos3 = rem % ep.gw;
+            }
+            ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
             __syncwarp();
-            if (!__all_sync(0xffffffffu, ok)) break;
+            if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
             tc_fence_after();
-#pragma unroll
+#pragma unroll 1
             for (int j = 0; j < BN / 64; ++j) {
                 const int c = half * (BN / 2) + 32 * j;
-                float v[16];
-                tmem_ld16_sync(tq + buf * BN + c, v);
+                const int col = n0 + c;
+                float v[32];
+                {
+                    float t[16];
+                    tmem_ld16_sync(tq + buf * BN + c, t);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) stg[lane * 32 + (i ^ lane)] = v[i];
-                tmem_ld16_sync(tq + buf * BN + c + 16, v);
+                    for (int i = 0; i < 16; ++i) v[i] = t[i];
+                    tmem_ld16_sync(tq + buf * BN + c + 16, t);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) stg[lane * 32 + ((16 + i) ^ lane)] = v[i];
-                __syncwarp();
-#pragma unroll
-                for (int it = 0; it < 4; ++it) {
-                    const int r = it * 8 + (lane >> 2);
-                    float a[8];
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) a[k] = stg[r * 32 + ((c8 + k) ^ r)];
-                    epi_apply<EPI>(ep, m0 + q * 32 + r, n0 + c + c8, a, pf, it);
+                    for (int i = 0; i < 16; ++i) v[16 + i] = t[i];
                 }
-                if (j + 1 < BN / 64) epi_prefetch<EPI>(ep, m0 + q * 32, n0 + c + 32 + c8, lane, pf);
+                if (j == BN / 64 - 1) {
+                    // last TMEM read of this tile: hand the accumulator back
+                    tc_fence_before();
+                    mbar_arrive(&acc_empty[buf]);
+                }
+#pragma unroll
+                for (int i = 0; i < 32; i += 8) {
+                    float bb[8];
+                    loadW<float, 8>(ep.bias + col + i, bb);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) v[i + k] += bb[k];
+                }
+                float xi[32];
+                if constexpr (RES) {
+                    ok = mbar_wait(lb, (n_ld - 1) & 1, err, ERR_WAIT_EPI);
+                    __syncwarp();
+                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                    float r[32];
+                    read_row32(s_res, lane, r);
+                    if constexpr (CACHE)
+                        if (has_rhat) read_row32(s_xin, lane, xi);
+#pragma unroll
+                    for (int i = 0; i < 32; i += 8) {
+                        float g[8];
+                        loadW<float, 8>(ep.gate + col + i, g);
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) v[i + k] = r[i + k] + g[k] * v[i + k];
+                    }
+                    __syncwarp();                      // every lane has read the block
+                    if (j + 1 < BN / 64) load_res(m0, col + 32);
+                }
+                if constexpr (EPI == EPI_GELU) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = gelu_tanh_approx(v[i]);
+                }
+                int part = 0, cl = col;
+                if constexpr (EPI == EPI_QKV_ROPE) {
+                    part = col / ep.d;
+                    cl = col - part * ep.d;
+                    if (part < 2 && row < ep.M) {
+                        const int pair0 = (cl % ep.head_dim) >> 1;
+#pragma unroll
+                        for (int k = 0; k < 16; ++k) {
+                            const int pr = pair0 + k;
+                            const int ax = ep.rope_axis[pr];
+                            const int pa = ax == 0 ? pos0 : (ax == 1 ? pos1 : (ax == 2 ? pos2 : pos3));
+                            const float2 t = ep.rope_cs[ep.rope_off[pr] + pa];
+                            const float x0 = v[2 * k], x1 = v[2 * k + 1];
+                            v[2 * k] = x0 * t.x - x1 * t.y;
+                            v[2 * k + 1] = x0 * t.y + x1 * t.x;
+                        }
+                    }
+                }
+                // staging: out is double-buffered unless the block also carries
+                // residual operands; a buffer is rewritten once the TMA store
+                // that used it has read it
+                uint8_t *s_out = (RES || (n_st & 1) == 0) ? s_out0 : s_aux;
+                if (lane == 0) {
+                    if constexpr (RES) bulk_wait_read<0>();
+                    else bulk_wait_read<1>();
+                }
                 __syncwarp();
+                write_row32(s_out, lane, v);
+                if constexpr (CACHE) {
+                    if (has_rhat) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = round_to<bf16>(v[i]) - xi[i];
+                        write_row32(s_aux, lane, v);
+                    }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&em.out[part], s_out, cl, m0 + q * 32);
+                    if constexpr (CACHE)
+                        if (has_rhat) tma_store_2d(&em.rhat, s_aux, col, m0 + q * 32);
+                    bulk_commit();
+                }
+                ++n_st;
             }
-            tc_fence_before();
-            mbar_arrive(&acc_empty[buf]);
         }
+        // every TMA store of this warp has completed before the CTA exits
+        if (lane == 0) bulk_wait_all();
+        __syncwarp();
     }
     tc_fence_before();
     __syncthreads();
@@ -346,6 +405,73 @@ bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t co
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2-D bf16 map with a 32 x 32 box and 64-byte swizzle (epilogue blocks).
+static bool make_tmap_epi(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols) {
+    EncodeTiledFn fn = encode_fn();
+    if (fn == nullptr) return false;
+    if ((reinterpret_cast<uintptr_t>(base) & 15) != 0 || (cols * 2) % 16 != 0 || cols % 32 != 0) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Encoded epilogue maps, looked up by (base, rows, cols): the chunk step
+// reuses the same activation buffers on every pass, so encoding happens once
+// per buffer.
+namespace {
+struct MapKey {
+    const void *base;
+    uint64_t rows, cols;
+    bool operator==(const MapKey &o) const { return base == o.base && rows == o.rows && cols == o.cols; }
+};
+struct MapKeyHash {
+    size_t operator()(const MapKey &k) const {
+        return std::hash<const void *>()(k.base) ^ (size_t)(k.rows * 0x9E3779B97F4A7C15ull) ^ (size_t)(k.cols << 17);
+    }
+};
+std::mutex g_map_mu;
+std::unordered_map<MapKey, CUtensorMap, MapKeyHash> g_maps;
+}  // namespace
+
+static bool epi_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols) {
+    if (base == nullptr) {                         // unused slot: any valid map
+        memset(m, 0, sizeof(*m));
+        return true;
+    }
+    std::lock_guard<std::mutex> lk(g_map_mu);
+    const MapKey key{base, rows, cols};
+    auto it = g_maps.find(key);
+    if (it != g_maps.end()) {
+        *m = it->second;
+        return true;
+    }
+    if (g_maps.size() > 4096) g_maps.clear();
+    if (!make_tmap_epi(m, base, rows, cols)) return false;
+    g_maps.emplace(key, *m);
+    return true;
+}
+
+template <int EPI>
+static bool build_epi_maps(EpiMaps &em, const EpiParams &ep) {
+    memset(&em, 0, sizeof(em));
+    if constexpr (EPI == EPI_QKV_ROPE) {
+        return epi_map(&em.out[0], ep.out, ep.M, ep.d) && epi_map(&em.out[1], ep.out_k, ep.M, ep.d) &&
+               epi_map(&em.out[2], ep.out_v, ep.M, ep.d);
+    } else {
+        bool ok = epi_map(&em.out[0], ep.out, ep.M, ep.N);
+        if constexpr (EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE) ok = ok && epi_map(&em.resid, ep.resid, ep.M, ep.N);
+        if constexpr (EPI == EPI_RESID_CACHE) {
+            if (ep.rhat != nullptr)
+                ok = ok && epi_map(&em.rhat, ep.rhat, ep.M, ep.N) && epi_map(&em.xin, ep.xin, ep.M, ep.N);
+        }
+        return ok;
+    }
+}
+
 static int gemm_sm_count() {
     static int n = 0;
     if (n == 0) {
@@ -366,8 +492,10 @@ int gemm_tc_bn(int M, int N) {
 template <int EPI, int BN>
 static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,
                              const uint8_t *skip, int *err, cudaStream_t st) {
-    using G = GemmTile<BN>;
-    auto kern = gemm_tc_kernel<BN, EPI, bf16>;
+    using G = GemmTile<BN, EPI>;
+    auto kern = gemm_tc_kernel<BN, EPI>;
+    EpiMaps em;
+    if (!build_epi_maps<EPI>(em, ep)) return cudaErrorInvalidValue;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM_BYTES);
@@ -377,7 +505,7 @@ static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const
     const int n_sm = gemm_sm_count();
     const int n_tiles = (ep.N / BN) * ((ep.M + GEMM_BM - 1) / GEMM_BM);
     const int grid = n_tiles < n_sm ? n_tiles : n_sm;
-    kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, ep, K, skip, err);
+    kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, em, ep, K, skip, err);
     return cudaGetLastError();
 }
 
