@@ -277,11 +277,16 @@ def main():
         calibrate(xc, chunk, cfg, args)
         return
 
+    # Timed runs without profiling (the per-pass block loop then replays its
+    # CUDA graphs); attention launch times and decisions come from separate
+    # profiled runs of the same chunks (decisions are deterministic).
     sampler = ClockSampler(local)
     sampler.start()
-    ms_x, launches, recs, pc_x = timed(gate, profile=True)
+    ms_x, launches, _, pc_x = timed(gate, profile=False)
     clocks = sampler.stop()
-    ms_all, _, recs_all, pc_all = timed(xb.gate_params(enabled=0), profile=True)
+    ms_all, _, _, pc_all = timed(xb.gate_params(enabled=0), profile=False)
+    _, _, recs, _ = timed(gate, profile=True)
+    _, _, recs_all, _ = timed(xb.gate_params(enabled=0), profile=True)
     xc.sync()
 
     # skip rates over the timed chunks (decisions logged per (pass, block))

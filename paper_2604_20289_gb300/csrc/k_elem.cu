@@ -312,7 +312,10 @@ __global__ void __launch_bounds__(GEMV_WARPS * 32) cond_kernel(const CondArgs c)
         if (tpath) {
             for (int i = threadIdx.x; i < c.tf; i += blockDim.x) xs[i] = c.temb[i];
         } else {
-            for (int i = threadIdx.x; i < c.A; i += blockDim.x) xs[i] = c.act[i];
+            for (int i = threadIdx.x; i < c.A; i += blockDim.x) {
+                xs[i] = c.act[i];
+                if (blockIdx.x == nb_d && c.act_out != nullptr) c.act_out[i] = c.act[i];
+            }
         }
         __syncthreads();
         if (j < d) acc = gemv_col(xs, tpath ? c.t_w1 : c.a_w1, n_in, d, j, warp);

@@ -189,12 +189,12 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     // are slow on this part; only the EMA state stays fp64.
     float da = 0.0f, na = 0.0f, nb = 0.0f;
     for (int i = 0; i < g.A; ++i) {
-        const float a = g.action[i];
+        const float a = g.action_dev != nullptr ? g.action_dev[i] : g.action[i];
         const float b = g.phi_act[active * 8 + i];
         da = fmaf(a, b, da);
         na = fmaf(a, a, na);
         nb = fmaf(b, b, nb);
-        g.phi_act[(active ^ 1) * 8 + i] = g.action[i];
+        g.phi_act[(active ^ 1) * 8 + i] = g.action_dev != nullptr ? g.action_dev[i] : g.action[i];
     }
     const float cos_sp = cos_rule_f(v[0], v[1], v[2]);
     const float cos_gl = cos_rule_f(v[5], v[6], v[7]);

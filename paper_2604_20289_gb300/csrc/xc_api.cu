@@ -97,6 +97,20 @@ bool is_host_ptr(const void *p) {
 
 }  // namespace
 
+// Everything the per-pass block loop takes from the host (besides buffers
+// that stay fixed for the context's lifetime).
+struct PassSig {
+    int t, kv, eval_mode, slot, n_keys, replay;
+    uint64_t replay_bits;
+    xc_gate_params p;                 // replay_skip pointer cleared
+    const void *lat, *v, *trace;
+};
+struct GraphEntry {
+    PassSig sig;
+    cudaGraphExec_t exec;
+    long long launches;
+};
+
 struct xc_ctx {
     xc_model_cfg cfg;
     int L, d, F, B, S, H, hd, Wkv, C, A, V, npc;
@@ -145,6 +159,18 @@ struct xc_ctx {
     // attention split workspace (partials of units cut between CTAs)
     void *attn_ws;
     size_t attn_ws_bytes;
+
+    // device copy of the chunk's action (written by the conditioning kernel)
+    float *act_dev;
+
+    // CUDA graphs of the per-pass block loop, keyed by everything the loop
+    // takes from the host (see PassSig).  The context's first pass runs
+    // directly (one-time kernel set-up such as shared-memory attributes
+    // happens outside any capture); every later new signature is captured.
+    std::vector<struct GraphEntry> graphs;
+    bool graphs_on;
+    bool warm;
+    cudaStream_t cap_st;                       // capture stream (the caller's may be the legacy default)
 
     // tensor maps (bf16); output tile width of each GEMM
     CUtensorMap tm_h, tm_o, tm_u, tm_q;
@@ -247,6 +273,11 @@ bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
 }
 
 // (Re)build the spatial sample for a token budget K; resets every gate cell.
+void drop_graphs(xc_ctx *ctx) {
+    for (GraphEntry &e : ctx->graphs) cudaGraphExecDestroy(e.exec);
+    ctx->graphs.clear();
+}
+
 void ensure_fp(xc_ctx *ctx, int K) {
     if (ctx->fp_K == K) return;
     int kfp = 0;
@@ -254,6 +285,7 @@ void ensure_fp(xc_ctx *ctx, int K) {
     const size_t n_all = (size_t)ctx->V * kfp * ctx->d + (size_t)ctx->V * ctx->d;
     if (ctx->fp_rows != nullptr) {
         CK(cudaStreamSynchronize(ctx->st));
+        drop_graphs(ctx);                        // the captured passes point at the old buffers
         for (auto it = ctx->allocs.begin(); it != ctx->allocs.end();) {
             if (*it == ctx->fp_rows || *it == ctx->phi) {
                 cudaFree(*it);
@@ -338,6 +370,46 @@ void prof_end(xc_ctx *ctx, int i) {
         ctx->launches += (n_launch);               \
     } while (0)
 
+// Replays the graph of `sig`, or captures `body` into a new one and
+// replays it (the context's very first pass runs directly instead).
+template <typename F>
+void run_graph(xc_ctx *ctx, const PassSig &sig, F &&body) {
+    auto same = [&](const PassSig &a) { return memcmp(&a, &sig, sizeof sig) == 0; };
+    for (GraphEntry &e : ctx->graphs)
+        if (same(e.sig)) {
+            CK(cudaGraphLaunch(e.exec, ctx->st));
+            ctx->launches += e.launches;
+            return;
+        }
+    if (!ctx->warm) {
+        body(ctx->st);
+        ctx->warm = true;
+        return;
+    }
+    if (ctx->graphs.size() >= 128) drop_graphs(ctx);
+    const long long l0 = ctx->launches;
+    CK(cudaStreamBeginCapture(ctx->cap_st, cudaStreamCaptureModeThreadLocal));
+    cudaGraph_t g = nullptr;
+    try {
+        body(ctx->cap_st);
+    } catch (...) {
+        cudaStreamEndCapture(ctx->cap_st, &g);
+        if (g != nullptr) cudaGraphDestroy(g);
+        ctx->launches = l0;
+        throw;
+    }
+    CK(cudaStreamEndCapture(ctx->cap_st, &g));
+    cudaGraphExec_t ex = nullptr;
+    const cudaError_t e = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    CK(e);
+    const long long n = ctx->launches - l0;
+    ctx->launches = l0;
+    ctx->graphs.push_back(GraphEntry{sig, ex, n});
+    CK(cudaGraphLaunch(ex, ctx->st));
+    ctx->launches += n;
+}
+
 template <typename T>
 void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigma, int t, bool kv,
               const xc_gate_params &p, float *v_dev) {
@@ -371,16 +443,23 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ca.mod_w = ctx->mod_w; ca.mod_b = ctx->mod_b; ca.blk_mod = ctx->blk_mod;
         ca.head_w = ctx->head_w; ca.head_b = ctx->head_b; ca.head_tab = ctx->head_tab;
         ca.ht = ctx->ht; ca.ha = ctx->ha; ca.e = ctx->e; ca.mods = ctx->mods; ca.hmod = ctx->hmod;
+        ca.act_out = ctx->act_dev;
         LAUNCH(XC_K_COND, -1, 3, conditioning(ca, st));
     }
-
-    T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
-    LAUNCH(XC_K_EMBED, -1, 1, patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
     // RoPE table of this chunk (absolute frames n*F .. n*F + F - 1)
     LAUNCH(XC_K_EMBED, -1, 1,
            rope_table(hd, (double)ctx->cfg.rope_theta, n * ctx->cfg.frames,
                       make_int4(ctx->V, ctx->cfg.frames, ctx->cfg.grid_h, ctx->cfg.grid_w), ctx->rope_cs,
                       ctx->rope_n, st));
+
+    // Everything below takes from the host only what PassSig holds, so it is
+    // captured into a CUDA graph and replayed for passes with the same
+    // signature (the gate decisions are device-side, so a graph serves every
+    // decision pattern).
+    auto body = [&](cudaStream_t st) {
+
+    T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
+    LAUNCH(XC_K_EMBED, -1, 1, patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
     CK(cudaMemsetAsync(ctx->flags, 0, B, st));
     CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
 
@@ -414,7 +493,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             const size_t cell = (size_t)t * B + b;
             g.phi = ctx->phi + cell * 2 * ctx->phi_n_all;
             g.phi_act = ctx->phi_act + cell * 16;
-            for (int i = 0; i < ctx->A; ++i) g.action[i] = action[i];
+            g.action_dev = ctx->act_dev;
             g.A = ctx->A;
             g.cell = ctx->cells + cell;
             g.mode = eval_mode ? 1 : 0;
@@ -521,6 +600,29 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
                                Ld * sizeof(T), cudaMemcpyDeviceToDevice, st));
     }
     LAUNCH(XC_K_HEAD, -1, 1, head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
+    };   // body
+
+    if (ctx->prof_on || !ctx->graphs_on) {
+        body(st);                                    // profiling records events per launch
+    } else {
+        PassSig sig;
+        memset(&sig, 0, sizeof sig);
+        sig.t = t;
+        sig.kv = kv ? 1 : 0;
+        sig.eval_mode = (n >= p.warmup_chunks && !(p.protect_step0 && t == 0)) ? 1 : 0;
+        sig.slot = slot;
+        sig.n_keys = n_keys;
+        sig.p = p;
+        sig.p.replay_skip = nullptr;
+        sig.replay = p.replay_skip != nullptr ? 1 : 0;
+        if (p.replay_skip != nullptr)
+            for (int b = 0; b < B; ++b)
+                if (p.replay_skip[b]) sig.replay_bits |= 1ull << b;
+        sig.lat = lat_dev;
+        sig.v = v_dev;
+        sig.trace = ctx->trace;
+        run_graph(ctx, sig, body);
+    }
     if (ctx->prof_on) {
         if (ctx->pass_seq < ctx->prof_cap)
             CK(cudaMemcpyAsync(ctx->dec_log + (size_t)ctx->pass_seq * B, ctx->flags, B, cudaMemcpyDeviceToDevice, st));
@@ -564,6 +666,8 @@ static void prof_free(xc_ctx *ctx);
 void xc_destroy(xc_ctx *ctx) {
     if (ctx == nullptr) return;
     cudaStreamSynchronize(ctx->st);
+    drop_graphs(ctx);
+    if (ctx->cap_st != nullptr) cudaStreamDestroy(ctx->cap_st);
     prof_free(ctx);
     for (void *p : ctx->allocs) cudaFree(p);
     if (ctx->h_flags) cudaFreeHost(ctx->h_flags);
@@ -689,6 +793,9 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->e = dalloc<float>(ctx, d * sizeof(float));
         ctx->mods = dalloc<float>(ctx, (size_t)B * 6 * d * sizeof(float));
         ctx->hmod = dalloc<float>(ctx, 2 * (size_t)d * sizeof(float));
+        ctx->act_dev = dalloc<float>(ctx, 8 * sizeof(float));
+        CK(cudaStreamCreateWithFlags(&ctx->cap_st, cudaStreamNonBlocking));
+        ctx->graphs_on = true;
 
         // ring and caches
         ctx->ring_k = dalloc<void>(ctx, (size_t)B * ctx->Wkv * Ld * es);

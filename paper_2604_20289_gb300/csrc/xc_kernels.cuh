@@ -21,6 +21,7 @@ struct GateArgs {
     float *phi;
     float *phi_act;
     float action[8];
+    const float *action_dev;      // if set, the action is read from device memory (chunk step)
     int A;
     GateCell *cell;
     int mode;
@@ -64,6 +65,7 @@ struct CondArgs {
     const float *t_w1, *t_b1, *a_w1, *a_b1, *t_w2, *t_b2, *a_w2, *a_b2;
     const float *mod_w, *mod_b, *blk_mod, *head_w, *head_b, *head_tab;
     float *ht, *ha, *e, *mods, *hmod;
+    float *act_out;               // device copy of the action (read by the gate kernels)
 };
 cudaError_t conditioning(const CondArgs &c, cudaStream_t st);
 template <typename T>
