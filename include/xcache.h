@@ -149,6 +149,13 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
  *   gate    NULL = Table 1 defaults.
  *   v_out   host or device float32 [L][c_latent] velocity, or NULL.
  *   stats   NULL or filled as documented above (synchronising).
+ * Execution: the conditioning and the chunk's RoPE table are launched
+ * directly; the rest of the pass (patch embedding, every block, the head)
+ * is captured into a CUDA graph the first time its host inputs (pass index,
+ * ring slot and fill, gate parameters and replay bits, latent / v_out /
+ * trace pointers) occur, and replayed whenever they recur.  Gate decisions
+ * stay on the device, so one graph serves every decision pattern.  While
+ * profiling (xc_profile_start) passes are launched directly.
  * Errors: XC_EINVAL, XC_ESTATE, XC_ECUDA, XC_ETIMEOUT (device wait expired). */
 xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, float sigma,
                         int step_index, int is_kv_update, const xc_gate_params *gate,
