@@ -12,4 +12,5 @@ from .xcache_oracle import (  # noqa: F401
     to_bf16, layer_norm, silu, gelu_tanh, timestep_embedding, rope_pair_table,
     apply_rope, token_positions, attention, grid_allocation, axis_indices,
     fingerprint_rows, cosine, max_token_deviation, gate_decide, rollout, SIGMAS,
+    group_token_positions, linear_rows, group_fingerprint_rows, gate_metrics,
 )

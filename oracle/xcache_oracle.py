@@ -94,6 +94,20 @@ def token_positions(n_cams: int, frames: int, gh: int, gw: int, chunk: int) -> n
     return pos.astype(np.float64)
 
 
+def group_token_positions(groups, frames: int, chunk: int) -> np.ndarray:
+    """[L, 4] positions of a chunk made of view groups ((cameras, gh, gw), ...)
+    whose tokens follow one another: within a group as token_positions, the
+    camera coordinate counting on across groups (one camera index per
+    physical camera)."""
+    out, cam0 = [], 0
+    for V, gh, gw in groups:
+        pos = token_positions(V, frames, gh, gw, chunk)
+        pos[:, 0] += cam0
+        out.append(pos)
+        cam0 += V
+    return np.concatenate(out, axis=0)
+
+
 def apply_rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
     """Rotate interleaved pairs of x [L, H, hd] by angle pos[axis(p)] * freq(p):
     (x0, x1) -> (x0 cos - x1 sin, x0 sin + x1 cos)."""
@@ -171,6 +185,34 @@ def fingerprint_rows(n_cams: int, frames: int, gh: int, gw: int, K: int) -> np.n
     return np.stack(rows)
 
 
+def linear_rows(n_tok: int, K: int) -> np.ndarray:
+    """1-D fallback of Section 2.3.1 (grid shape unavailable): K uniformly
+    spaced, cell-centred indices along a camera's token axis of length n_tok,
+    floor((2j + 1) n_tok / (2K)) (reading c7 applied to one axis); all tokens
+    when n_tok <= K."""
+    if n_tok <= K:
+        return np.arange(n_tok)
+    return axis_indices(n_tok, K)
+
+
+def group_fingerprint_rows(groups, frames: int, K: int, linear: bool = False) -> list:
+    """Spatial-sample rows of every view group (Section 2.3.1: one fingerprint
+    per group, its cameras stacked along V): a list with one [V_g, k_g] array
+    of chunk token indices per group.  ``linear`` takes the 1-D fallback
+    instead of the 3-D grid sample."""
+    out, tok0 = [], 0
+    for V, gh, gw in groups:
+        npc = frames * gh * gw
+        if linear:
+            loc = linear_rows(npc, K)
+            rows = np.stack([c * npc + loc for c in range(V)])
+        else:
+            rows = fingerprint_rows(V, frames, gh, gw, K)
+        out.append(rows + tok0)
+        tok0 += V * npc
+    return out
+
+
 # ---------------------------------------------------------------------------
 # Gate metrics (Eq. 5 - 9)
 # ---------------------------------------------------------------------------
@@ -199,6 +241,21 @@ def max_token_deviation(cur: np.ndarray, prev: np.ndarray, eps: float) -> float:
     return math.inf if math.isnan(d) else d
 
 
+def gate_metrics(phi, cached, eps: float):
+    """Eq. 5 - 6 over a fingerprint with one spatial and one global entry per
+    view group plus the action entry: s_cos = min of the cosines of all
+    entries (Eq. 5); d_max = max over the groups' spatial entries of Eq. 6
+    (reading c24: every group's sample must pass the deviation test).
+    ``phi`` and ``cached`` are (spatial list, global list, action)."""
+    sp, gl, ac = phi
+    csp, cgl, cac = cached
+    s = min([cosine(a, c) for a, c in zip(sp, csp)]
+            + [cosine(a, c) for a, c in zip(gl, cgl)]
+            + [cosine(ac, cac)])
+    dmax = max(max_token_deviation(a, c, eps) for a, c in zip(sp, csp))
+    return s, dmax
+
+
 @dataclass
 class GateParams:
     """Gate knobs; defaults are the paper's Table 1 (tau_floor 0.97 per Table 1
@@ -218,6 +275,7 @@ class GateParams:
     step0_strict_tau: float = 0.0   # 0 = off, else e.g. 0.999
     fp_tokens: int = 32
     fp_refresh: int = 0          # 0 = refresh on compute, 1 = on every evaluation
+    fp_linear: bool = False      # 1-D fallback sample instead of the 3-D grid
 
 
 class Decision(IntEnum):
@@ -228,12 +286,13 @@ class Decision(IntEnum):
 
 @dataclass
 class GateCell:
-    """Per-(t, b) cache: residual r_hat (Eq. 3), cached fingerprint entries,
-    EMA of the cosine (Eq. 8), consecutive-skip counter (max staleness)."""
+    """Per-(t, b) cache: residual r_hat (Eq. 3), cached fingerprint entries
+    (spatial and global entry of every view group, the action), EMA of the
+    cosine (Eq. 8), consecutive-skip counter (max staleness)."""
     valid: bool = False
     r_hat: np.ndarray | None = None
-    phi_sp: np.ndarray | None = None
-    phi_gl: np.ndarray | None = None
+    phi_sp: list | None = None
+    phi_gl: list | None = None
     phi_act: np.ndarray | None = None
     ema: float = 0.0
     has_hist: bool = False
@@ -340,16 +399,21 @@ class OracleXCache:
     mechanisms (2.5).
 
     Rolling KV cache: per block a FIFO of the clean (k, v) of the last
-    kv_window - 1 chunks, written by the KV-update pass (Section 2.1) with the
-    oldest chunk evicted; every pass attends to those plus the current chunk's
-    own (k, v) (reading c18)."""
+    kv_window - 1 KV-update chunks, written by the KV-update pass (Section
+    2.1) with the oldest chunk evicted; every pass attends to those plus the
+    current chunk's own (k, v) (reading c18).
+
+    KV-update chunks (Section 2.5 (3), reading c23): with kv_period P = 0
+    every chunk ends with the KV-update pass and only that pass is forced
+    full.  With P > 0 only chunks n with n mod P == P - 1 have one; their
+    denoising passes run in force-compute mode (every block computes, the
+    gate is not evaluated, the residual and fingerprint caches are
+    refreshed), and a chunk without one ends after its last denoising pass."""
 
     def __init__(self, cfg, weights: dict):
         self.cfg = cfg
         self.model = OracleModel(cfg, weights)
-        V, Fr, gh, gw = cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w
         self._fp_rows = {}
-        self.npc = Fr * gh * gw
         self.reset()
 
     def reset(self):
@@ -360,19 +424,28 @@ class OracleXCache:
         self.ring_v = [[] for _ in range(cfg.n_blocks)]
         self.cells = [[GateCell() for _ in range(cfg.n_blocks)] for _ in range(cfg.n_steps)]
 
-    def fp_rows(self, K: int) -> np.ndarray:
-        if K not in self._fp_rows:
-            c = self.cfg
-            self._fp_rows[K] = fingerprint_rows(c.n_cams, c.frames, c.grid_h, c.grid_w, K)
-        return self._fp_rows[K]
+    def is_kv_chunk(self, n: int) -> bool:
+        P = getattr(self.cfg, "kv_period", 0)
+        return P == 0 or n % P == P - 1
 
-    def fingerprint(self, x: np.ndarray, action: np.ndarray, K: int):
-        """phi(x): spatial entry [V, k, d] (Section 2.3.1), global channel =
-        per-camera token mean [V, d], condition channel = the action (2.3.2)."""
-        V = self.cfg.n_cams
-        sp = x[self.fp_rows(K)]                                   # [V, k, d]
-        gl = x.reshape(V, self.npc, -1).mean(axis=1)              # [V, d]
-        return sp.copy(), gl, np.asarray(action, np.float64).copy()
+    def fp_rows(self, K: int, linear: bool = False) -> list:
+        key = (K, bool(linear))
+        if key not in self._fp_rows:
+            c = self.cfg
+            self._fp_rows[key] = group_fingerprint_rows(c.groups, c.frames, K, linear)
+        return self._fp_rows[key]
+
+    def fingerprint(self, x: np.ndarray, action: np.ndarray, K: int, linear: bool = False):
+        """phi(x), per view group (Section 2.3.1): spatial entry [V_g, k_g, d]
+        and global channel = per-camera token mean [V_g, d]; condition channel
+        = the action (2.3.2).  Returns (spatial list, global list, action)."""
+        sp, gl, tok0 = [], [], 0
+        for (V, gh, gw), rows in zip(self.cfg.groups, self.fp_rows(K, linear)):
+            npc = self.cfg.frames * gh * gw
+            sp.append(x[rows].copy())                                        # [V_g, k_g, d]
+            gl.append(x[tok0:tok0 + V * npc].reshape(V, npc, -1).mean(axis=1))   # [V_g, d]
+            tok0 += V * npc
+        return sp, gl, np.asarray(action, np.float64).copy()
 
     def chunk_step(self, latent, action, sigma: float, step: int, is_kv_update: bool,
                    p: GateParams, replay=None, trace: list | None = None):
@@ -383,14 +456,18 @@ class OracleXCache:
         cfg, M = self.cfg, self.model
         B = cfg.n_blocks
         S = cfg.n_steps
+        n = self.n
+        kv_chunk = self.is_kv_chunk(n)
         if is_kv_update:
             if self.next_step not in (0, S):
                 raise RuntimeError("KV-update pass out of order")
+            if not kv_chunk:
+                raise RuntimeError("KV-update pass on a chunk without one")
         elif step != self.next_step or step >= S:
             raise RuntimeError("denoising step out of order")
-        n = self.n
+        forced_chunk = getattr(cfg, "kv_period", 0) > 0 and kv_chunk
         mods, hm = M.cond(sigma, action)
-        pos = token_positions(cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, n)
+        pos = group_token_positions(cfg.groups, cfg.frames, n)
         x = M.patch_embed(latent)
         kv_new = {}
         stats = dict(decision=np.zeros(B, np.int64), s_cos=np.full(B, np.nan),
@@ -402,14 +479,12 @@ class OracleXCache:
             phi = None
             if gated_block:
                 cell = self.cells[step][b]
-                phi = self.fingerprint(x, action, p.fp_tokens)
+                phi = self.fingerprint(x, action, p.fp_tokens, p.fp_linear)
                 eligible = (n >= p.warmup_chunks and not (p.protect_step0 and step == 0)
-                            and cell.valid)
+                            and not forced_chunk and cell.valid)
                 if eligible:
-                    sp, gl, ac = phi
-                    s = min(cosine(sp, cell.phi_sp), cosine(gl, cell.phi_gl),
-                            cosine(ac, cell.phi_act))                        # Eq. 5
-                    dmax = max_token_deviation(sp, cell.phi_sp, p.eps_dev)   # Eq. 6
+                    s, dmax = gate_metrics(phi, (cell.phi_sp, cell.phi_gl, cell.phi_act),
+                                           p.eps_dev)                        # Eq. 5 - 6
                     skip, tau = gate_decide(cell, s, dmax, step, p,
                                             None if replay is None else bool(replay[b]))
                     stats["s_cos"][b], stats["d_max"][b], stats["tau"][b] = s, dmax, tau
@@ -442,6 +517,9 @@ class OracleXCache:
                     self.ring_v[b].pop(0)
             self.n += 1
             self.next_step = 0
+        elif step == S - 1 and not kv_chunk:
+            self.n += 1                     # chunk without a KV-update pass
+            self.next_step = 0
         else:
             self.next_step = step + 1
         return v, stats
@@ -456,9 +534,11 @@ SIGMAS = (1.0, 0.75, 0.5, 0.25, 0.0)
 def rollout(cfg, weights, traj, params: GateParams, n_chunks: int, replay=None,
             keep_trace: bool = False):
     """Chunk n: x = eps_n; for t < S: v = step(x, sigma_t); x += (sigma_{t+1} -
-    sigma_t) v (Euler, flow matching); then the KV-update pass on the chunk's
-    clean latent x_c[n] at sigma = 0 (teacher-forced, reading c22).
-    Returns dict(final [n][L, C], stats [n][t] (t = S is the KV pass), trace)."""
+    sigma_t) v (Euler, flow matching); then, on a KV-update chunk, the
+    KV-update pass on the chunk's clean latent x_c[n] at sigma = 0
+    (teacher-forced, reading c22).
+    Returns dict(final [n][L, C], stats [n][t] (t = S is the KV pass, absent
+    on chunks without one), trace)."""
     oc = OracleXCache(cfg, weights)
     S = cfg.n_steps
     finals, stats, traces = [], [], []
@@ -473,8 +553,9 @@ def rollout(cfg, weights, traj, params: GateParams, n_chunks: int, replay=None,
             x = x + (SIGMAS[t + 1] - SIGMAS[t]) * v
             st_n.append(st)
             tr_n.append(tr)
-        _, st = oc.chunk_step(traj.clean(n), a, 0.0, S, True, params)
-        st_n.append(st)
+        if oc.is_kv_chunk(n):
+            _, st = oc.chunk_step(traj.clean(n), a, 0.0, S, True, params)
+            st_n.append(st)
         finals.append(x)
         stats.append(st_n)
         traces.append(tr_n)

@@ -409,3 +409,153 @@ def test_ring_is_fifo_over_window():
     near = O.rollout(cfg, w, Pert(1), p, 4)["final"][3]    # still resident
     np.testing.assert_array_equal(far, ref)
     assert np.abs(near - ref).max() > 1e-6
+
+
+# ------------------------------------------------ view groups (Section 2.3.1)
+def test_group_token_positions_brute_force():
+    groups, Fr, chunk = ((2, 2, 3), (1, 4, 5)), 2, 3
+    want = []
+    cam = 0
+    for V, gh, gw in groups:                      # explicit loops in token order
+        for c in range(V):
+            for f in range(Fr):
+                for h in range(gh):
+                    for w in range(gw):
+                        want.append((cam + c, chunk * Fr + f, h, w))
+        cam += V
+    np.testing.assert_array_equal(O.group_token_positions(groups, Fr, chunk), np.array(want, float))
+
+
+def test_linear_rows_hand_values():
+    # 1344 tokens, K = 32: floor((2j + 1) * 1344 / 64) = 21 (2j + 1)
+    np.testing.assert_array_equal(O.linear_rows(1344, 32), 21 * (2 * np.arange(32) + 1))
+    np.testing.assert_array_equal(O.linear_rows(100, 3), [16, 50, 83])
+    np.testing.assert_array_equal(O.linear_rows(20, 32), np.arange(20))
+
+
+def test_group_fingerprint_rows_enumeration():
+    groups, Fr = ((2, 16, 28), (1, 4, 4)), 3
+    rows = O.group_fingerprint_rows(groups, Fr, 32)
+    assert [r.shape for r in rows] == [(2, 32), (1, 18)]
+    # group 0 starts at token 0: the single-group sample
+    np.testing.assert_array_equal(rows[0], O.fingerprint_rows(2, 3, 16, 28, 32))
+    # group 1 (3 x 4 x 4 = 48 > 32 tokens) starts after 2 x 1344 tokens; its
+    # allocation is (2, 3, 3): f in {0, 2}, h and w in {0, 2, 3}
+    got = set()
+    for r in rows[1][0]:
+        rem = int(r) - 2688
+        f, rem = divmod(rem, 16)
+        h, w = divmod(rem, 4)
+        assert f in (0, 2) and h in (0, 2, 3) and w in (0, 2, 3)
+        got.add((f, h, w))
+    assert len(got) == 18
+    # 1-D fallback: per camera, linear_rows along its own token axis
+    lin = O.group_fingerprint_rows(groups, Fr, 32, linear=True)
+    np.testing.assert_array_equal(lin[0][1], 1344 + 21 * (2 * np.arange(32) + 1))
+    np.testing.assert_array_equal(lin[1][0], 2688 + O.linear_rows(48, 32))
+
+
+def test_gate_metrics_over_groups_closed_forms():
+    sp = [rng.standard_normal((2, 32, 8)), rng.standard_normal((1, 18, 8))]
+    gl = [rng.standard_normal((2, 8)), rng.standard_normal((1, 8))]
+    ac = rng.standard_normal(2)
+    twice = ([2 * a for a in sp], [2 * a for a in gl], 2 * ac)
+    s, d = O.gate_metrics(twice, (sp, gl, ac), 1e-6)
+    assert s == pytest.approx(1.0, abs=1e-13)
+    # d over the groups: max|2a - a| / (mean|a| + eps), the larger of the two
+    want = max(np.abs(a).max() / (np.abs(a).mean() + 1e-6) for a in sp)
+    assert d == pytest.approx(want, rel=1e-12)
+    # one group's spatial sample flipped: that entry's cosine -1 is the minimum
+    flip = ([sp[0], -sp[1]], gl, ac)
+    s, d = O.gate_metrics(flip, (sp, gl, ac), 1e-6)
+    assert s == pytest.approx(-1.0, abs=1e-13)
+    assert d == pytest.approx(2 * np.abs(sp[1]).max() / (np.abs(sp[1]).mean() + 1e-6), rel=1e-12)
+    # one group's global entry orthogonalised: cosine 0 is the minimum
+    g1 = gl[1].ravel()
+    o = rng.standard_normal(g1.size)
+    o -= (o @ g1) / (g1 @ g1) * g1
+    s, _ = O.gate_metrics((sp, [gl[0], o.reshape(gl[1].shape)], ac), (sp, gl, ac), 1e-6)
+    assert s == pytest.approx(0.0, abs=1e-12)
+
+
+def test_single_view_group_equals_plain_grid():
+    cfg = X.TINY_F32.replace(name="pin_tiny_groups", n_chunks=3)
+    grp = cfg.replace(view_groups=((cfg.n_cams, cfg.grid_h, cfg.grid_w),))
+    p = O.GateParams(tau_floor=0.5, margin=0.02, tau_dev=10.0)
+    w = X.make_weights(cfg)
+    a = O.rollout(cfg, w, X.Trajectory(cfg, n_chunks=3), p, 3)
+    b = O.rollout(grp, w, X.Trajectory(grp, n_chunks=3), p, 3)
+    for n in range(3):
+        np.testing.assert_array_equal(a["final"][n], b["final"][n])
+
+
+# ----------------------------------- KV-update chunks (Section 2.5 (3), c23)
+def test_kv_period_one_is_all_blocks():
+    """P = 1: every chunk is a KV-update chunk, so every denoising pass runs
+    in force-compute mode: no skip, outputs equal to the gate switched off."""
+    cfg = X.TINY_F32.replace(name="pin_tiny_p1", n_chunks=4, kv_period=1)
+    w = X.make_weights(cfg)
+    lax = O.GateParams(tau_floor=0.0, margin=1.0, tau_dev=1e9)
+    r = O.rollout(cfg, w, X.Trajectory(cfg, n_chunks=4), lax, 4)
+    off = O.rollout(cfg.replace(kv_period=0), w, X.Trajectory(cfg, n_chunks=4),
+                    O.GateParams(enabled=False), 4)
+    for n in range(4):
+        np.testing.assert_array_equal(r["final"][n], off["final"][n])
+        assert all((st["decision"] == O.Decision.FORCED).all() for st in r["stats"][n])
+
+
+def test_kv_period_forced_chunks_and_skip_bound():
+    P, N = 3, 7
+    cfg = X.TINY_F32.replace(name="pin_tiny_p3", n_chunks=N, kv_period=P)
+    lax = O.GateParams(tau_floor=0.0, margin=1.0, tau_dev=1e9)
+    r = O.rollout(cfg, X.make_weights(cfg), X.Trajectory(cfg, n_chunks=N), lax, N)
+    S, B = cfg.n_steps, cfg.n_blocks
+    gated = skipped = 0
+    for n, st_n in enumerate(r["stats"]):
+        kv = n % P == P - 1
+        assert len(st_n) == S + (1 if kv else 0)          # KV pass on KV chunks only
+        dec = np.array([s["decision"] for s in st_n])
+        if kv or n < lax.warmup_chunks:
+            assert (dec == O.Decision.FORCED).all()
+        else:                                            # lax thresholds: every gated block skips
+            assert (dec[:, 1:] == O.Decision.SKIP).all()
+        if n >= lax.warmup_chunks:
+            gated += S * (B - 1)
+            skipped += int((dec[:S, 1:] == O.Decision.SKIP).sum())
+    # each forced chunk takes its share: skip rate <= (P - 1) / P
+    assert skipped / gated <= (P - 1) / P
+
+
+def test_kv_period_ring_holds_kv_chunks_only():
+    """P = 2, W = 3: the ring holds the clean K/V of the last two KV-update
+    chunks (n = 1, 3, 5, ...).  One block, so a chunk's K/V depend on its own
+    clean latent alone."""
+    cfg = X.TINY_F32.replace(name="pin_tiny_p2", n_blocks=1, kv_period=2)
+    base = X.Trajectory(cfg, n_chunks=7)
+
+    class Pert:
+        def __init__(self, which):
+            self.which = which
+
+        def noise(self, n):
+            return base.noise(n)
+
+        def action(self, n):
+            return base.action(n)
+
+        def clean(self, n):
+            c = base.clean(n)
+            return c + 0.5 if n == self.which else c
+
+    p = O.GateParams(enabled=False)
+    w = X.make_weights(cfg)
+    ref = O.rollout(cfg, w, base, p, 7)["final"]
+    not_kv = O.rollout(cfg, w, Pert(0), p, 7)["final"]     # chunk 0 has no KV pass
+    kv1 = O.rollout(cfg, w, Pert(1), p, 7)["final"]        # written after chunk 1
+    for n in range(7):
+        np.testing.assert_array_equal(not_kv[n], ref[n])
+    for n in (0, 1):
+        np.testing.assert_array_equal(kv1[n], ref[n])
+    for n in (2, 3, 4, 5):                                  # resident: (1), (1, 3)
+        assert np.abs(kv1[n] - ref[n]).max() > 1e-6
+    np.testing.assert_array_equal(kv1[6], ref[6])          # ring (3, 5): chunk 1 evicted

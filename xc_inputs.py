@@ -103,7 +103,14 @@ class ModelCfg:
 
     A chunk holds ``n_cams * frames * grid_h * grid_w`` tokens, ordered
     (camera, frame, h, w) row-major.  ``kv_window`` counts ring slots
-    including the current chunk."""
+    including the current chunk.
+
+    ``view_groups`` (optional) replaces the single camera grid with groups of
+    cameras that share a grid shape: a tuple of (cameras, grid_h, grid_w);
+    the groups' tokens follow one another in that order, each group camera by
+    camera, and ``n_cams`` is then the total camera count.  ``kv_period`` P
+    > 0 makes every P-th chunk (n mod P == P - 1) the one whose clean latent
+    feeds the KV-update pass; 0 runs that pass after every chunk."""
     name: str
     n_blocks: int
     d_model: int
@@ -123,10 +130,19 @@ class ModelCfg:
     t_freq: int = 256
     ln_eps: float = 1e-6
     rope_theta: float = 10000.0
+    view_groups: tuple = ()
+    kv_period: int = 0
+
+    @property
+    def groups(self) -> tuple:
+        """((cameras, grid_h, grid_w), ...) of the view groups in token order."""
+        if self.view_groups:
+            return tuple(tuple(g) for g in self.view_groups)
+        return ((self.n_cams, self.grid_h, self.grid_w),)
 
     @property
     def tokens(self) -> int:
-        return self.n_cams * self.frames * self.grid_h * self.grid_w
+        return sum(c * self.frames * h * w for c, h, w in self.groups)
 
     def replace(self, **kw) -> "ModelCfg":
         return dataclasses.replace(self, **kw)
