@@ -49,6 +49,12 @@ def parse():
     ap.add_argument("--workload", default="small", choices=sorted(WORKLOADS))
     ap.add_argument("--tau-floor", type=float, default=GATE["tau_floor"])
     ap.add_argument("--tau-dev", type=float, default=GATE["tau_dev"])
+    ap.add_argument("--kv-period", type=int, default=0,
+                    help="KV-update pass only on chunks n mod P == P-1, whose denoising passes "
+                         "run in force-compute mode (0 = KV-update pass after every chunk)")
+    ap.add_argument("--view-groups", default="",
+                    help="view groups of the chunk as CAMSxHxW,... (e.g. 3x20x36,2x16x28,2x12x20); "
+                         "default: the workload's single camera grid")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--calibrate", action="store_true", help="print gate-metric quantiles and exit")
@@ -159,7 +165,7 @@ def oracle_block_sample(cfg, seed: int = 0) -> float:
               for i in range(cfg.kv_window - 1)]
     past_v = [R(X.random_tensor(seed, f"bench/v{i}", (L, H, hd)).astype(np.float64))
               for i in range(cfg.kv_window - 1)]
-    pos = O.token_positions(cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, cfg.kv_window)
+    pos = O.group_token_positions(cfg.groups, cfg.frames, cfg.kv_window)
     t0 = time.perf_counter()
     m.block(0, x, mods[0], past_k, past_v, pos)
     return time.perf_counter() - t0
@@ -169,8 +175,8 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    cfg = WORKLOADS[args.workload]
-    passes = cfg.n_blocks * (cfg.n_steps + 1)
+    cfg = workload_cfg(args)
+    passes = cfg.n_blocks * (cfg.n_steps + (1 if cfg.kv_period == 0 else 1.0 / cfg.kv_period))
     times = []
     for i in range(args.warmup + args.steps):
         t = oracle_block_sample(cfg, seed=i)
@@ -193,11 +199,32 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def workload_cfg(args):
+    """The named workload with the --view-groups / --kv-period overrides."""
+    cfg = WORKLOADS[args.workload]
+    if args.view_groups:
+        groups = tuple(tuple(int(v) for v in g.split("x")) for g in args.view_groups.split(","))
+        cfg = cfg.replace(name=f"{cfg.name}_groups_{args.view_groups}", view_groups=groups,
+                          n_cams=sum(g[0] for g in groups), grid_h=groups[0][1], grid_w=groups[0][2])
+    if args.kv_period:
+        cfg = cfg.replace(name=f"{cfg.name}_kvperiod{args.kv_period}", kv_period=args.kv_period)
+    return cfg
+
+
+def has_kv_pass(cfg, n: int) -> bool:
+    """Chunk n ends with a KV-update pass (every chunk when kv_period = 0)."""
+    P = cfg.kv_period
+    return P == 0 or n % P == P - 1
+
+
 def config_of(cfg, args):
     return {"workload": cfg.name, "blocks": cfg.n_blocks, "d_model": cfg.d_model,
             "heads": f"{cfg.n_heads}x{cfg.head_dim}", "d_ffn": cfg.d_ffn,
             "tokens_per_chunk": cfg.tokens, "kv_window_chunks": cfg.kv_window,
-            "keys_max": cfg.kv_window * cfg.tokens, "passes_per_chunk": cfg.n_steps + 1,
+            "keys_max": cfg.kv_window * cfg.tokens,
+            "passes_per_chunk": cfg.n_steps + 1 if cfg.kv_period == 0 else
+            f"{cfg.n_steps} + a KV-update pass every {cfg.kv_period} chunks",
+            "view_groups": [list(g) for g in cfg.groups],
             "gate": {"tau_floor": args.tau_floor, "tau_dev": args.tau_dev, "other": "Table 1 defaults"},
             "l2": "not flushed: per-chunk working set (KV ring + residual cache + weights) > 129 MB L2",
             "parallelism": f"replicas x{args.gpus}"}
@@ -220,7 +247,7 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl")
-    cfg = WORKLOADS[args.workload]
+    cfg = workload_cfg(args)
     n_total = args.warmup + args.steps
     traj = X.Trajectory(cfg, n_chunks=n_total)
     w = X.make_weights(cfg)
@@ -239,7 +266,11 @@ def main():
         for t in range(S):
             xc.chunk_step(x, acts[n], SIGMAS[t], t, False, gate, v_out=v, want_stats=False)
             xc.euler(x, v, SIGMAS[t + 1] - SIGMAS[t])
-        xc.chunk_step(clean[n], acts[n], 0.0, S, True, gate, want_stats=False)
+        if has_kv_pass(cfg, n):
+            xc.chunk_step(clean[n], acts[n], 0.0, S, True, gate, want_stats=False)
+
+    # kind of every timed pass, in issue order: True = KV-update pass
+    kv_of_pass = [p for n in range(args.warmup, n_total) for p in [False] * S + [True] * has_kv_pass(cfg, n)]
 
     def barrier():
         torch.cuda.synchronize()
@@ -291,7 +322,7 @@ def main():
 
     # skip rates over the timed chunks (decisions logged per (pass, block))
     dec = np.array([r["decision"] for r in recs])
-    den = np.array([r["pass_seq"] % (S + 1) < S for r in recs])
+    den = np.array([not kv_of_pass[r["pass_seq"]] for r in recs])
     skip_all = float(np.mean(dec == xb.XC_DEC_SKIP)) if len(dec) else 0.0
     skip_den = float(np.mean(dec[den] == xb.XC_DEC_SKIP)) if den.any() else 0.0
 
@@ -333,7 +364,7 @@ def main():
         line["e2e"] = e2e(xc, traj, acts, cfg, args, gate, world, dev)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         t_block = oracle_block_sample(cfg)
-        computed = (1.0 - skip_all) * cfg.n_blocks * (S + 1)
+        computed = (1.0 - skip_all) * cfg.n_blocks * len(kv_of_pass) / args.steps
         line["cpu_baseline"] = {
             "kind": "oracle", "value": 1.0 / (t_block * computed), "unit": "chunks/s",
             "cores": os.cpu_count(),
@@ -352,7 +383,7 @@ def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
     """Speedup predicted from kernel times (untimed, profiled re-run of both
     arms over the same chunks): T_all / (T_all - sum over skipped block-passes
     of (T_block - T_gate - T_reuse) + sum over gated block-passes of T_gate),
-    per chunk, T_block from the all-blocks arm at the same (chunk, pass, block)."""
+    per chunk, T_block from the all-blocks arm at the same (pass, block)."""
     from paper_2604_20289_gb300 import xcache as xb
     S = cfg.n_steps
     n_total = args.warmup + args.steps
@@ -376,13 +407,13 @@ def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
             kernel_us[kind] = round(1e3 * float(np.mean(ms)), 2)
     for r in recs_all:
         if r["kind"] in block_kinds:
-            key = (r["chunk"], r["pass_seq"] % (S + 1), r["block"])
+            key = (r["pass_seq"], r["block"])
             t_block[key] = t_block.get(key, 0.0) + r["ms"]
     saved = gated = 0.0
     per = {}
     for r in run(gate):
         if r["kind"] in ("gate", "reuse") and r["block"] >= 0:
-            key = (r["chunk"], r["pass_seq"] % (S + 1), r["block"])
+            key = (r["pass_seq"], r["block"])
             d = per.setdefault(key, {"dec": r["decision"], "gate": 0.0, "reuse": 0.0})
             d[r["kind"]] += r["ms"]
     for key, d in per.items():
@@ -492,8 +523,9 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
         for t in range(S):
             xc.chunk_step(x_np, acts[n], SIGMAS[t], t, False, gate, v_out=v_np, want_stats=False)
             np.add(x_np, np.float32(SIGMAS[t + 1] - SIGMAS[t]) * v_np, out=x_np)
-        c_np[:] = traj.clean(n)
-        xc.chunk_step(c_np, acts[n], 0.0, S, True, gate, want_stats=False)
+        if has_kv_pass(cfg, n):
+            c_np[:] = traj.clean(n)
+            xc.chunk_step(c_np, acts[n], 0.0, S, True, gate, want_stats=False)
 
     xc.reset()
     for n in range(args.warmup):
@@ -510,8 +542,9 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         sec = float(t.item())
     nbytes = L * C * 4
+    kv = sum(has_kv_pass(cfg, n) for n in range(args.warmup, args.warmup + args.steps)) / args.steps
     return {"value": args.steps * world / sec, "unit": "chunks/s",
-            "h2d_bytes_per_step": (S + 1) * nbytes + (S + 1) * cfg.action_dim * 4,
+            "h2d_bytes_per_step": (S + kv) * (nbytes + cfg.action_dim * 4),
             "d2h_bytes_per_step": S * nbytes}
 
 
@@ -535,7 +568,8 @@ def calibrate(xc, chunk, cfg, args):
             ok = st["decision"] == xb.XC_DEC_COMPUTE
             s_all += list(st["s_cos"][ok])
             d_all += list(st["d_max"][ok])
-        xc.chunk_step(torch.from_numpy(traj.clean(n)).cuda(), traj.action(n), 0.0, S, True, g)
+        if has_kv_pass(cfg, n):
+            xc.chunk_step(torch.from_numpy(traj.clean(n)).cuda(), traj.action(n), 0.0, S, True, g)
     q = [0.1, 0.25, 0.5, 0.75, 0.9]
     print(json.dumps({"s_cos_q": dict(zip(map(str, q), np.quantile(s_all, q).tolist())),
                       "d_max_q": dict(zip(map(str, q), np.quantile(d_all, q).tolist())),

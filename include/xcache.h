@@ -36,6 +36,7 @@ extern "C" {
 #endif
 
 #define XC_MAX_BLOCKS 64
+#define XC_MAX_GROUPS 4
 
 typedef enum {
     XC_OK = 0,
@@ -63,12 +64,31 @@ typedef enum {
  * order.  kv_window_chunks counts ring slots INCLUDING the current chunk.
  * Constraints: d_model = n_heads*head_dim; head_dim % 16 == 0; for XC_BF16
  * head_dim in {64, 128}, d_model % 256 == 0 and d_ffn % 256 == 0;
- * n_blocks <= XC_MAX_BLOCKS; t_freq_dim even and <= 512. */
+ * n_blocks <= XC_MAX_BLOCKS; t_freq_dim even and <= 512.
+ *
+ * View groups (Section 2.3.1): with n_groups = 0 all cameras share the grid
+ * (grid_h, grid_w).  With 1 <= n_groups <= XC_MAX_GROUPS, group g holds
+ * group_cams[g] cameras of grid (group_h[g], group_w[g]); the groups' tokens
+ * follow one another in group order (each group camera by camera, then
+ * (frame, h, w) row-major), n_cams must equal the sum of group_cams, the
+ * RoPE camera coordinate counts on across groups, and grid_h / grid_w are not
+ * used.  The gate keeps one spatial and one global fingerprint entry per group.
+ *
+ * kv_period (Section 2.5 (3)): 0 = every chunk ends with a KV-update pass, the
+ * only pass forced to compute every block.  P > 0 = only chunks n with
+ * n mod P == P - 1 have a KV-update pass; their denoising passes run in
+ * force-compute mode (every block computes, the gate is not evaluated, the
+ * residual and fingerprint caches are refreshed), and a chunk without one
+ * ends after its last denoising pass.  The ring then holds the clean K/V of
+ * the last kv_window_chunks - 1 KV-update chunks. */
 typedef struct {
     int n_blocks, d_model, n_heads, head_dim, d_ffn, c_latent, action_dim;
     int n_cams, frames, grid_h, grid_w;
     int kv_window_chunks, n_denoise_steps, dtype, t_freq_dim;
     float ln_eps, rope_theta;
+    int kv_period;
+    int n_groups;
+    int group_cams[XC_MAX_GROUPS], group_h[XC_MAX_GROUPS], group_w[XC_MAX_GROUPS];
 } xc_model_cfg;
 
 /* Host float32 weights, math convention y = x @ W with W stored [in][out]
@@ -98,6 +118,11 @@ typedef struct {
  * KV-update protection is always on: the KV pass never evaluates the gate.
  *   fp_refresh  0: cached fingerprint refreshed when the block computes;
  *               1: refreshed on every evaluation.
+ *   fp_linear   0: spatial sample on the 3-D (frame, h, w) grid of each view
+ *               group; 1: the 1-D fallback -- fp_tokens uniformly spaced,
+ *               cell-centred indices along each camera's token axis
+ *               (Section 2.3.1).  Changing fp_tokens or fp_linear between calls
+ *               rebuilds the sample and clears every gate cell.
  *   replay_skip host [n_blocks] or NULL: decision-replay mode -- for blocks the
  *               gate evaluates, the decision is replay_skip[b] != 0 instead of
  *               Eq. 7 (metrics, EMA and staleness are still updated). */
@@ -107,7 +132,7 @@ typedef struct {
     int front_anchors, back_anchors, warmup_chunks, max_skips;
     int protect_step0;
     float step0_strict_tau;
-    int fp_tokens, fp_refresh;
+    int fp_tokens, fp_refresh, fp_linear;
     const uint8_t *replay_skip;
 } xc_gate_params;
 
@@ -142,10 +167,13 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
  *   step_index  t in [0, n_denoise_steps) for a denoising pass; ignored when
  *           is_kv_update != 0.  Passes of a chunk must come in order
  *           t = 0..S-1, then the KV-update pass (which may also come alone at
- *           the start of a chunk); otherwise XC_ESTATE.
+ *           the start of a chunk); otherwise XC_ESTATE.  With kv_period P > 0
+ *           a chunk without a KV-update pass (n mod P != P - 1) ends after
+ *           pass S-1 and a KV-update call on it returns XC_ESTATE.
  *   is_kv_update  the KV-update pass: every block computes (KV-update
  *           protection, Section 2.5 (3)), clean K/V go to ring slot
- *           n mod kv_window_chunks, and the chunk counter advances.
+ *           k mod kv_window_chunks (k = KV-update passes so far; k = n when
+ *           kv_period = 0), and the chunk counter advances.
  *   gate    NULL = Table 1 defaults.
  *   v_out   host or device float32 [L][c_latent] velocity, or NULL.
  *   stats   NULL or filled as documented above (synchronising).

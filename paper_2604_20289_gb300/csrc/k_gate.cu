@@ -2,22 +2,22 @@
 // block input, both gating metrics against the cached fingerprint, adaptive
 // threshold and the skip / recompute flag -- all on the device.
 //
-// Fingerprint (Section 2.3.1-2.3.2), one view group of V cameras:
-//   spatial entry  x at the K-token 3-D grid sample of every camera  [V, k, d]
-//   global channel per-camera mean of x over its tokens                 [V, d]
-//   condition      the chunk's action vector                            [A]
-// Metrics: s_cos = min over entries of the cosine (Eq. 5); d_max = max|cur -
-// prev| / (mean|prev| + eps) over the spatial entry (Eq. 6).  Decision Eq. 7
-// with tau_cos = max(tau_floor, ema - m) (Eq. 9), EMA update (Eq. 8) and the
-// consecutive-skip cap (Section 2.5 (4)).
+// Fingerprint (Section 2.3.1-2.3.2), per view group g of V_g cameras:
+//   spatial entry  x at the K-token sample of every camera of g        [V_g, k_g, d]
+//   global channel per-camera mean of x over its tokens                 [V_g, d]
+// plus the condition entry, the chunk's action vector                   [A]
+// Metrics: s_cos = min over all entries of the cosine (Eq. 5); d_max = max
+// over the groups of max|cur - prev| / (mean|prev| + eps) over the group's
+// spatial entry (Eq. 6).  Decision Eq. 7 with tau_cos = max(tau_floor, ema -
+// m) (Eq. 9), EMA update (Eq. 8) and the consecutive-skip cap (Section 2.5 (4)).
 //
 // Grid: one CTA (512 threads) per (camera c, 64-column slice s).  The CTA
 // streams all of camera c's rows of its slice once (16-byte loads, 8 rows in
 // flight per thread), so it completes that slice's per-camera means by
 // itself; it also takes the slice of the spatial sample.  All reductions run
 // in fp32; each CTA writes 8 partials and takes an atomic ticket; the last
-// CTA combines all partials in a fixed order and makes the decision (the EMA
-// state is kept in fp64).  No spin-wait anywhere; deterministic.  The cached
+// CTA combines the partials of each group in a fixed order and makes the
+// decision (the EMA state is kept in fp64).  No spin-wait anywhere; deterministic.  The cached
 // fingerprint is double-buffered per (t, b): the current fingerprint goes to
 // the inactive half, which becomes active when the block recomputes.
 #include <cmath>
@@ -75,11 +75,24 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int blk = blockIdx.x;
     const int c = blk / g.n_slices, s = blk % g.n_slices;
-    const int d = g.d, npc = g.npc;
+    const int d = g.d;
+    // camera c's group (unrolled compare chain: constant parameter indices)
+    int tok0 = g.g_tok0[0], cam0 = g.g_cam0[0], npc = g.g_npc[0], fp0 = g.g_fp0[0], kfp = g.g_kfp[0];
+#pragma unroll
+    for (int q = 1; q < XC_MAX_GROUPS; ++q)
+        if (q < g.n_groups && c >= g.g_cam0[q]) {
+            tok0 = g.g_tok0[q];
+            cam0 = g.g_cam0[q];
+            npc = g.g_npc[q];
+            fp0 = g.g_fp0[q];
+            kfp = g.g_kfp[q];
+        }
+    const size_t ctok0 = (size_t)tok0 + (size_t)(c - cam0) * npc;   // camera c's first token
+    const int crow0 = fp0 + (c - cam0) * kfp;                        // and first sample row
     const int col0 = s * GATE_CW;
     const T *x = reinterpret_cast<const T *>(g.x);
     const int active = g.cell->active;
-    const int n_sp = g.V * g.kfp * d;
+    const int n_sp = g.n_rows * d;
     const int n_all = n_sp + g.V * d;
     const float *phi_prev = g.phi + (size_t)active * n_all;
     float *phi_next = g.phi + (size_t)(active ^ 1) * n_all;
@@ -90,7 +103,7 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     for (int i = 0; i < VEC; ++i) acc[i] = 0.0f;
     {
         const int ty = tid / TPR, tx = tid % TPR;
-        const T *base = x + (size_t)c * npc * d + col0 + tx * VEC;
+        const T *base = x + ctok0 * d + col0 + tx * VEC;
         // GATE_UNROLL guarded loads in flight per step, the ragged end included
         for (int r = ty; r < npc; r += GATE_UNROLL * RPAR) {
             uint4 u[GATE_UNROLL];
@@ -120,10 +133,10 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         p[7] = prev * prev;
     }
     // 3. spatial sample rows of camera c in this slice
-    for (int it = tid; it < g.kfp * GATE_CW; it += GATE_THREADS) {
+    for (int it = tid; it < kfp * GATE_CW; it += GATE_THREADS) {
         const int i = it / GATE_CW, j = it % GATE_CW;
-        const int row = g.fp_rows[c * g.kfp + i];
-        const size_t e = ((size_t)c * g.kfp + i) * d + col0 + j;
+        const int row = g.fp_rows[crow0 + i];
+        const size_t e = ((size_t)crow0 + i) * d + col0 + j;
         const float cur = to_f(x[(size_t)row * d + col0 + j]);
         const float prev = phi_prev[e];
         phi_next[e] = cur;
@@ -158,30 +171,47 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    float v[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int b = tid; b < (int)gridDim.x; b += GATE_THREADS) {
+    // Per view group: fold the partials of the group's CTAs (cameras
+    // [g_cam0[q], g_cam0[q + 1]), every slice) in a fixed order; thread 0
+    // keeps the running min of the cosines and max of the deviations.
+    float cos_min = INFINITY, dmax = 0.0f;
+#pragma unroll
+    for (int q = 0; q < XC_MAX_GROUPS; ++q) {
+        if (q >= g.n_groups) break;
+        const int b0 = g.g_cam0[q] * g.n_slices, b1 = g.g_cam0[q + 1] * g.n_slices;
+        float v[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int b = b0 + tid; b < b1; b += GATE_THREADS) {
+#pragma unroll
+            for (int k = 0; k < GATE_PARTS; ++k) {
+                const float w = __ldcg(&g.part[(size_t)b * GATE_PARTS + k]);
+                v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
+            }
+        }
 #pragma unroll
         for (int k = 0; k < GATE_PARTS; ++k) {
-            const float q = __ldcg(&g.part[(size_t)b * GATE_PARTS + k]);
-            v[k] = k == 3 ? fmaxf(v[k], q) : v[k] + q;
-        }
-    }
 #pragma unroll
-    for (int k = 0; k < GATE_PARTS; ++k) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float w = __shfl_xor_sync(0xffffffffu, v[k], o);
-            v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
+            for (int o = 16; o > 0; o >>= 1) {
+                const float w = __shfl_xor_sync(0xffffffffu, v[k], o);
+                v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
+            }
+            if (lane == 0) wpart[warp][k] = v[k];
         }
-        if (lane == 0) wpart[warp][k] = v[k];
+        __syncthreads();
+        if (tid == 0) {
+            for (int k = 0; k < GATE_PARTS; ++k) {
+                float a = wpart[0][k];
+                for (int w = 1; w < NW; ++w) a = k == 3 ? fmaxf(a, wpart[w][k]) : a + wpart[w][k];
+                v[k] = a;
+            }
+            const int n_sp_q = (g.g_cam0[q + 1] - g.g_cam0[q]) * g.g_kfp[q] * d;
+            float dq = v[3] / (v[4] / (float)n_sp_q + g.eps_dev);
+            if (isnan(dq)) dq = INFINITY;
+            cos_min = fminf(cos_min, fminf(cos_rule_f(v[0], v[1], v[2]), cos_rule_f(v[5], v[6], v[7])));
+            dmax = fmaxf(dmax, dq);
+        }
+        __syncthreads();
     }
-    __syncthreads();
     if (tid != 0) return;
-    for (int k = 0; k < GATE_PARTS; ++k) {
-        float a = wpart[0][k];
-        for (int w = 1; w < NW; ++w) a = k == 3 ? fmaxf(a, wpart[w][k]) : a + wpart[w][k];
-        v[k] = a;
-    }
     *g.ticket = 0;
 
     // All sums and metrics are fp32 (relative error ~1e-7, far inside the
@@ -196,12 +226,8 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         nb = fmaf(b, b, nb);
         g.phi_act[(active ^ 1) * 8 + i] = g.action_dev != nullptr ? g.action_dev[i] : g.action[i];
     }
-    const float cos_sp = cos_rule_f(v[0], v[1], v[2]);
-    const float cos_gl = cos_rule_f(v[5], v[6], v[7]);
     const float cos_a = cos_rule_f(da, na, nb);
-    const double s_min = (double)fminf(fminf(cos_sp, cos_gl), cos_a);
-    float dmax = v[3] / (v[4] / (float)n_sp + g.eps_dev);
-    if (isnan(dmax)) dmax = INFINITY;
+    const double s_min = (double)fminf(cos_min, cos_a);
 
     GateCell cell = *g.cell;
     uint8_t dec;
@@ -337,10 +363,8 @@ extern "C" xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam
     memset(&g, 0, sizeof g);
     g.x = x;
     g.d = d;
-    g.V = n_cams;
-    g.npc = tokens_per_cam;
+    xc::gate_single_group(g, n_cams, tokens_per_cam, kfp);
     g.fp_rows = fp_rows;
-    g.kfp = kfp;
     g.n_slices = ns;
     g.phi = phi;
     g.phi_act = phi_act;

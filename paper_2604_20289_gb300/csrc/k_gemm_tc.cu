@@ -254,11 +254,11 @@ __global__ void __launch_bounds__(320, 1)
             // RoPE position of this thread's row (camera, frame, h, w), once per tile
             int pos0 = 0, pos1 = 0, pos2 = 0, pos3 = 0;
             if constexpr (EPI == EPI_QKV_ROPE) {
-                pos0 = row / ep.npc;
-                const int rem = row - pos0 * ep.npc;
-                pos1 = rem / (ep.gh * ep.gw);
-                pos2 = (rem / ep.gw) % ep.gh;
-                pos3 = rem % ep.gw;
+                const int4 tp = token_pos(ep, row);
+                pos0 = tp.x;
+                pos1 = tp.y;
+                pos2 = tp.z;
+                pos3 = tp.w;
             }
             ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
             __syncwarp();

@@ -7,6 +7,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -47,6 +48,19 @@ int rope_layout(int hd, const int npos[4], std::vector<int> &axis, std::vector<i
             base += npos[a];
         }
     return base;
+}
+
+// 1-D fallback of the spatial sample (Section 2.3.1): K uniformly spaced,
+// cell-centred indices floor((2j+1) N / (2K)) along each camera's N tokens,
+// every token when N <= K.
+std::vector<int> linear_rows(int V, long long N, int K, int *kfp) {
+    std::vector<int> rows;
+    const int k = N <= K ? (int)N : K;
+    *kfp = k;
+    for (int c = 0; c < V; ++c)
+        for (int j = 0; j < k; ++j)
+            rows.push_back((int)(c * N + (N <= K ? j : ((2LL * j + 1) * N) / (2LL * K))));
+    return rows;
 }
 
 // Spatial sample of the fingerprint (Section 2.3.1): per axis
@@ -113,7 +127,7 @@ struct GraphEntry {
 
 struct xc_ctx {
     xc_model_cfg cfg;
-    int L, d, F, B, S, H, hd, Wkv, C, A, V, npc;
+    int L, d, F, B, S, H, hd, Wkv, C, A, V;
     bool bf;
     size_t esz;
     cudaStream_t st;
@@ -127,7 +141,7 @@ struct xc_ctx {
     float *qkv_b, *o_b, *f1_b, *f2_b;          // [B][N]
     int *rope_axis, *rope_off;                 // per pair
     float2 *rope_cs;                           // per-chunk (cos, sin) table
-    int rope_n;
+    int rope_n, rope_h, rope_w;               // table extent (largest grid of the view groups)
 
     // activations / conditioning
     void *xb[2], *x1, *hbuf, *q, *o, *u;
@@ -140,9 +154,20 @@ struct xc_ctx {
     float *phi;                                // [S][B][2][n_all]
     float *phi_act;                            // [S][B][2][8]
     GateCell *cells;                           // [S][B]
-    int *fp_rows;
-    int fp_K, kfp;
+    int *fp_rows;                              // sample rows, group by group, camera by camera
+    int fp_K, fp_lin, n_rows;
+    int g_kfp[XC_MAX_GROUPS], g_fp0[XC_MAX_GROUPS];
     size_t phi_n_all;
+
+    // view groups (Section 2.3.1): cameras [g_cam0[g], g_cam0[g+1]) of grid
+    // g_gh[g] x g_gw[g], tokens from g_tok0[g]
+    int G;
+    int g_cam0[XC_MAX_GROUPS + 1], g_tok0[XC_MAX_GROUPS], g_npc[XC_MAX_GROUPS], g_gh[XC_MAX_GROUPS],
+        g_gw[XC_MAX_GROUPS];
+
+    // KV-update chunks (Section 2.5 (3)): period (0 = every chunk) and the
+    // number of KV-update passes so far (the ring's write count)
+    int kv_period, kvc;
 
     // per pass
     uint8_t *flags;
@@ -240,8 +265,24 @@ bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
     if (c->d_model % 64 != 0 || c->d_ffn % 16 != 0 || c->d_ffn < 16) return bad("d_model % 64 or d_ffn % 16");
     if (c->c_latent != 16) return bad("c_latent must be 16");
     if (c->action_dim < 1 || c->action_dim > 8) return bad("action_dim out of [1, 8]");
-    if (c->n_cams < 1 || c->frames < 1 || c->grid_h < 1 || c->grid_w < 1) return bad("empty latent grid");
-    if ((long long)c->n_cams * c->frames * c->grid_h * c->grid_w > (1LL << 24)) return bad("chunk too large");
+    if (c->n_groups < 0 || c->n_groups > XC_MAX_GROUPS) return bad("n_groups out of [0, XC_MAX_GROUPS]");
+    if (c->n_cams < 1 || c->frames < 1) return bad("empty latent grid");
+    long long tokens = 0;
+    if (c->n_groups == 0) {
+        if (c->grid_h < 1 || c->grid_w < 1) return bad("empty latent grid");
+        tokens = (long long)c->n_cams * c->frames * c->grid_h * c->grid_w;
+    } else {
+        long long cams = 0;
+        for (int g = 0; g < c->n_groups; ++g) {
+            if (c->group_cams[g] < 1 || c->group_h[g] < 1 || c->group_w[g] < 1) return bad("empty view group");
+            cams += c->group_cams[g];
+            tokens += (long long)c->group_cams[g] * c->frames * c->group_h[g] * c->group_w[g];
+            if (tokens > (1LL << 24)) break;
+        }
+        if (cams != c->n_cams) return bad("n_cams != sum of group_cams");
+    }
+    if (tokens > (1LL << 24)) return bad("chunk too large");
+    if (c->kv_period < 0) return bad("kv_period < 0");
     if (c->kv_window_chunks < 1 || c->n_denoise_steps < 1 || c->n_denoise_steps > 64) return bad("window / steps");
     if (c->t_freq_dim < 2 || c->t_freq_dim % 2 != 0 || c->t_freq_dim > COND_TEMB_MAX)
         return bad("t_freq_dim must be even and at most 512");
@@ -268,6 +309,7 @@ bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
         return bad("negative count");
     if (p->fp_tokens < 1) return bad("fp_tokens < 1");
     if (p->fp_refresh != 0 && p->fp_refresh != 1) return bad("fp_refresh must be 0 or 1");
+    if (p->fp_linear != 0 && p->fp_linear != 1) return bad("fp_linear must be 0 or 1");
     (void)B;
     return true;
 }
@@ -278,11 +320,19 @@ void drop_graphs(xc_ctx *ctx) {
     ctx->graphs.clear();
 }
 
-void ensure_fp(xc_ctx *ctx, int K) {
-    if (ctx->fp_K == K) return;
-    int kfp = 0;
-    std::vector<int> rows = fingerprint_rows(ctx->V, ctx->cfg.frames, ctx->cfg.grid_h, ctx->cfg.grid_w, K, &kfp);
-    const size_t n_all = (size_t)ctx->V * kfp * ctx->d + (size_t)ctx->V * ctx->d;
+void ensure_fp(xc_ctx *ctx, int K, int linear) {
+    if (ctx->fp_K == K && ctx->fp_lin == linear) return;
+    std::vector<int> rows;
+    for (int g = 0; g < ctx->G; ++g) {
+        const int Vg = ctx->g_cam0[g + 1] - ctx->g_cam0[g];
+        int kfp = 0;
+        std::vector<int> r = linear ? linear_rows(Vg, ctx->g_npc[g], K, &kfp)
+                                    : fingerprint_rows(Vg, ctx->cfg.frames, ctx->g_gh[g], ctx->g_gw[g], K, &kfp);
+        ctx->g_fp0[g] = (int)rows.size();
+        ctx->g_kfp[g] = kfp;
+        for (int v : r) rows.push_back(v + ctx->g_tok0[g]);
+    }
+    const size_t n_all = rows.size() * (size_t)ctx->d + (size_t)ctx->V * ctx->d;
     if (ctx->fp_rows != nullptr) {
         CK(cudaStreamSynchronize(ctx->st));
         drop_graphs(ctx);                        // the captured passes point at the old buffers
@@ -301,9 +351,21 @@ void ensure_fp(xc_ctx *ctx, int K) {
     CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * n_all * sizeof(float), ctx->st));
     CK(cudaMemsetAsync(ctx->cells, 0, (size_t)ctx->S * ctx->B * sizeof(GateCell), ctx->st));
     CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
-    ctx->kfp = kfp;
+    ctx->n_rows = (int)rows.size();
     ctx->phi_n_all = n_all;
     ctx->fp_K = K;
+    ctx->fp_lin = linear;
+}
+
+// Chunk n has a KV-update pass (always when kv_period = 0).
+bool kv_chunk(const xc_ctx *ctx, int n) { return ctx->kv_period == 0 || n % ctx->kv_period == ctx->kv_period - 1; }
+
+// The gate is evaluated on denoising pass t of the current chunk: past the
+// warmup chunks, not a protected step 0, not a force-compute (KV-update)
+// chunk of a periodic schedule.
+bool eval_pass(const xc_ctx *ctx, const xc_gate_params &p, int t) {
+    const int n = ctx->n;
+    return n >= p.warmup_chunks && !(p.protect_step0 && t == 0) && !(ctx->kv_period > 0 && kv_chunk(ctx, n));
 }
 
 void clear_state(xc_ctx *ctx) {
@@ -318,6 +380,7 @@ void clear_state(xc_ctx *ctx) {
     CK(cudaMemsetAsync(ctx->g_scratch + ctx->g_ticket_off, 0, sizeof(unsigned), ctx->st));
     CK(cudaStreamSynchronize(ctx->st));
     ctx->n = 0;
+    ctx->kvc = 0;
     ctx->next_step = 0;
 }
 
@@ -417,8 +480,10 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     cudaStream_t st = ctx->st;
     const size_t Ld = (size_t)L * d;
     const int n = ctx->n;
-    const int slot = n % ctx->Wkv;
-    const int n_res = (n + 1 < ctx->Wkv ? n + 1 : ctx->Wkv);
+    // ring: the clean K/V of the last Wkv - 1 KV-update chunks plus this
+    // chunk's own, written to the slot the next KV-update pass fills
+    const int slot = ctx->kvc % ctx->Wkv;
+    const int n_res = (ctx->kvc + 1 < ctx->Wkv ? ctx->kvc + 1 : ctx->Wkv);
     const int n_keys = n_res * L;
     ctx->cur_keys = n_keys;
 
@@ -449,7 +514,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     // RoPE table of this chunk (absolute frames n*F .. n*F + F - 1)
     LAUNCH(XC_K_EMBED, -1, 1,
            rope_table(hd, (double)ctx->cfg.rope_theta, n * ctx->cfg.frames,
-                      make_int4(ctx->V, ctx->cfg.frames, ctx->cfg.grid_h, ctx->cfg.grid_w), ctx->rope_cs,
+                      make_int4(ctx->V, ctx->cfg.frames, ctx->rope_h, ctx->rope_w), ctx->rope_cs,
                       ctx->rope_n, st));
 
     // Everything below takes from the host only what PassSig holds, so it is
@@ -464,7 +529,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
 
     const bool gating = p.enabled != 0 && !kv;
-    const bool eval_mode = n >= p.warmup_chunks && !(p.protect_step0 && t == 0);
+    const bool eval_mode = eval_pass(ctx, p, t);
     T *x1 = reinterpret_cast<T *>(ctx->x1);
     T *hb = reinterpret_cast<T *>(ctx->hbuf);
     T *qb = reinterpret_cast<T *>(ctx->q);
@@ -486,9 +551,17 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.x = xin;
             g.d = d;
             g.V = ctx->V;
-            g.npc = ctx->npc;
             g.fp_rows = ctx->fp_rows;
-            g.kfp = ctx->kfp;
+            g.n_groups = ctx->G;
+            g.n_rows = ctx->n_rows;
+            for (int q = 0; q < ctx->G; ++q) {
+                g.g_cam0[q] = ctx->g_cam0[q];
+                g.g_tok0[q] = ctx->g_tok0[q];
+                g.g_npc[q] = ctx->g_npc[q];
+                g.g_fp0[q] = ctx->g_fp0[q];
+                g.g_kfp[q] = ctx->g_kfp[q];
+            }
+            g.g_cam0[ctx->G] = ctx->V;
             g.n_slices = ctx->g_ns;
             const size_t cell = (size_t)t * B + b;
             g.phi = ctx->phi + cell * 2 * ctx->phi_n_all;
@@ -528,9 +601,14 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.out_v = rv;
         ep.d = d;
         ep.head_dim = hd;
-        ep.npc = ctx->npc;
-        ep.gh = ctx->cfg.grid_h;
-        ep.gw = ctx->cfg.grid_w;
+        ep.n_groups = ctx->G;
+        for (int q = 0; q < ctx->G; ++q) {
+            ep.g_tok0[q] = ctx->g_tok0[q];
+            ep.g_cam0[q] = ctx->g_cam0[q];
+            ep.g_npc[q] = ctx->g_npc[q];
+            ep.g_gh[q] = ctx->g_gh[q];
+            ep.g_gw[q] = ctx->g_gw[q];
+        }
         ep.frames = ctx->cfg.frames;
         ep.frame0 = n * ctx->cfg.frames;
         ep.rope_axis = ctx->rope_axis;
@@ -609,7 +687,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         memset(&sig, 0, sizeof sig);
         sig.t = t;
         sig.kv = kv ? 1 : 0;
-        sig.eval_mode = (n >= p.warmup_chunks && !(p.protect_step0 && t == 0)) ? 1 : 0;
+        sig.eval_mode = eval_pass(ctx, p, t) ? 1 : 0;
         sig.slot = slot;
         sig.n_keys = n_keys;
         sig.p = p;
@@ -709,8 +787,23 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->C = cfg->c_latent;
         ctx->A = cfg->action_dim;
         ctx->V = cfg->n_cams;
-        ctx->npc = cfg->frames * cfg->grid_h * cfg->grid_w;
-        ctx->L = ctx->V * ctx->npc;
+        ctx->G = cfg->n_groups == 0 ? 1 : cfg->n_groups;
+        ctx->L = 0;
+        ctx->g_cam0[0] = 0;
+        ctx->rope_h = ctx->rope_w = 1;
+        for (int g = 0; g < ctx->G; ++g) {
+            const int Vg = cfg->n_groups == 0 ? cfg->n_cams : cfg->group_cams[g];
+            ctx->g_gh[g] = cfg->n_groups == 0 ? cfg->grid_h : cfg->group_h[g];
+            ctx->g_gw[g] = cfg->n_groups == 0 ? cfg->grid_w : cfg->group_w[g];
+            ctx->g_npc[g] = cfg->frames * ctx->g_gh[g] * ctx->g_gw[g];
+            ctx->g_tok0[g] = ctx->L;
+            ctx->g_cam0[g + 1] = ctx->g_cam0[g] + Vg;
+            ctx->L += Vg * ctx->g_npc[g];
+            ctx->rope_h = std::max(ctx->rope_h, ctx->g_gh[g]);
+            ctx->rope_w = std::max(ctx->rope_w, ctx->g_gw[g]);
+        }
+        ctx->kv_period = cfg->kv_period;
+        ctx->kvc = 0;
         ctx->bf = cfg->dtype == XC_BF16;
         ctx->esz = ctx->bf ? 2 : 4;
         ctx->st = reinterpret_cast<cudaStream_t>(cuda_stream);
@@ -769,7 +862,7 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         }
         {
             std::vector<int> ax, off;
-            const int npos[4] = {cfg->n_cams, cfg->frames, cfg->grid_h, cfg->grid_w};
+            const int npos[4] = {cfg->n_cams, cfg->frames, ctx->rope_h, ctx->rope_w};
             ctx->rope_n = rope_layout(ctx->hd, npos, ax, off);
             ctx->rope_axis = dalloc<int>(ctx, ax.size() * sizeof(int));
             ctx->rope_off = dalloc<int>(ctx, off.size() * sizeof(int));
@@ -804,9 +897,10 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->cells = dalloc<GateCell>(ctx, (size_t)ctx->S * B * sizeof(GateCell));
         ctx->phi_act = dalloc<float>(ctx, (size_t)ctx->S * B * 16 * sizeof(float));
         ctx->fp_K = -1;
+        ctx->fp_lin = 0;
         ctx->fp_rows = nullptr;
         ctx->phi = nullptr;
-        ensure_fp(ctx, 32);
+        ensure_fp(ctx, 32, 0);
 
         // per pass
         ctx->flags = dalloc<uint8_t>(ctx, XC_MAX_BLOCKS);
@@ -1038,13 +1132,17 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
             set_err(ctx, "KV-update pass before all %d denoising passes of chunk %d", ctx->S, ctx->n);
             return XC_ESTATE;
         }
+        if (!kv_chunk(ctx, ctx->n)) {
+            set_err(ctx, "chunk %d has no KV-update pass (kv_period %d)", ctx->n, ctx->kv_period);
+            return XC_ESTATE;
+        }
     } else if (step_index != ctx->next_step || step_index >= ctx->S) {
         set_err(ctx, "denoising pass %d out of order (expected %d)", step_index, ctx->next_step);
         return XC_ESTATE;
     }
     const int t = kv ? 0 : step_index;
     try {
-        ensure_fp(ctx, p.fp_tokens);
+        ensure_fp(ctx, p.fp_tokens, p.fp_linear);
         const size_t lat_bytes = (size_t)ctx->L * ctx->C * sizeof(float);
         const float *lat_dev = latent;
         if (is_host_ptr(latent)) {
@@ -1088,6 +1186,10 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
     }
     if (kv) {
         ctx->n += 1;
+        ctx->kvc += 1;
+        ctx->next_step = 0;
+    } else if (step_index == ctx->S - 1 && !kv_chunk(ctx, ctx->n)) {
+        ctx->n += 1;                                 // chunk without a KV-update pass ends here
         ctx->next_step = 0;
     } else {
         ctx->next_step = step_index + 1;
@@ -1205,10 +1307,7 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
     ep.out_v = v;
     ep.d = d;
     ep.head_dim = head_dim;
-    ep.npc = npc;
-    ep.gh = gh;
-    ep.gw = gw;
-    ep.frames = frames;
+    epi_single_grid(ep, frames, gh, gw);
     ep.frame0 = chunk * frames;
     ep.rope_axis = axis;
     ep.rope_off = off;
@@ -1325,10 +1424,8 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
     memset(&g, 0, sizeof g);
     g.x = x;
     g.d = d;
-    g.V = n_cams;
-    g.npc = tokens_per_cam;
+    gate_single_group(g, n_cams, tokens_per_cam, kfp);
     g.fp_rows = fp_rows;
-    g.kfp = kfp;
     g.n_slices = ws.ns;
     g.phi = phi;
     g.phi_act = phi_act;

@@ -109,12 +109,48 @@ struct EpiParams {
     void *out_k;               // [M][d]  QKV kind
     void *out_v;               // [M][d]  QKV kind
     void *rhat;                // [M][N]  residual cache slot or nullptr
-    // RoPE geometry (QKV kind)
-    int d, head_dim, npc, gh, gw, frames, frame0;
+    // RoPE geometry (QKV kind): view group g covers tokens [g_tok0[g],
+    // g_tok0[g + 1]) with cameras g_cam0[g].. of g_npc[g] = frames * g_gh[g]
+    // * g_gw[g] tokens each
+    int d, head_dim, frames, frame0;
+    int n_groups;
+    int g_tok0[XC_MAX_GROUPS], g_cam0[XC_MAX_GROUPS], g_npc[XC_MAX_GROUPS], g_gh[XC_MAX_GROUPS],
+        g_gw[XC_MAX_GROUPS];
     const int *rope_axis;      // [head_dim/2] 0 camera, 1 frame, 2 h, 3 w
     const int *rope_off;       // [head_dim/2] table entry of position 0 of each pair
     const float2 *rope_cs;     // (cos, sin) table of this chunk (rope_table_kernel)
 };
+
+// One view group covering every camera (grid gh x gw).
+inline void epi_single_grid(EpiParams &p, int frames, int gh, int gw) {
+    p.frames = frames;
+    p.n_groups = 1;
+    p.g_tok0[0] = 0;
+    p.g_cam0[0] = 0;
+    p.g_npc[0] = frames * gh * gw;
+    p.g_gh[0] = gh;
+    p.g_gw[0] = gw;
+}
+
+// (camera, frame within the chunk, h, w) of token `row`.  The group is picked
+// by an unrolled compare chain, so the parameter arrays are only read at
+// constant indices.
+__device__ __forceinline__ int4 token_pos(const EpiParams &p, int row) {
+    int tok0 = p.g_tok0[0], cam0 = p.g_cam0[0], npc = p.g_npc[0], gh = p.g_gh[0], gw = p.g_gw[0];
+#pragma unroll
+    for (int g = 1; g < XC_MAX_GROUPS; ++g)
+        if (g < p.n_groups && row >= p.g_tok0[g]) {
+            tok0 = p.g_tok0[g];
+            cam0 = p.g_cam0[g];
+            npc = p.g_npc[g];
+            gh = p.g_gh[g];
+            gw = p.g_gw[g];
+        }
+    const int r = row - tok0;
+    const int cl = r / npc;
+    const int rem = r - cl * npc;
+    return make_int4(cam0 + cl, rem / (gh * gw), (rem / gw) % gh, rem % gw);
+}
 
 enum { EPI_BIAS = XC_EPI_BIAS, EPI_GELU = XC_EPI_GELU, EPI_RESID_GATE = XC_EPI_RESID_GATE,
        EPI_RESID_CACHE = XC_EPI_RESID_CACHE, EPI_QKV_ROPE = 16 };
@@ -203,12 +239,8 @@ __device__ __forceinline__ void epilogue_run(const EpiParams &p, int row, int co
         const int part = col / d;          // 0 q, 1 k, 2 v (runs never straddle: d % 16 == 0)
         const int c = col - part * d;
         if (part < 2) {
-            const int cam = row / p.npc;
-            const int rem = row - cam * p.npc;
-            const int f = rem / (p.gh * p.gw);
-            const int hh = (rem / p.gw) % p.gh;
-            const int ww = rem % p.gw;
-            const int pos[4] = {cam, f, hh, ww};      // frame: index within the chunk
+            const int4 tp = token_pos(p, row);
+            const int pos[4] = {tp.x, tp.y, tp.z, tp.w};      // frame: index within the chunk
             const int pair0 = (c % p.head_dim) >> 1;
 #pragma unroll
             for (int j = 0; j < W / 2; ++j) {

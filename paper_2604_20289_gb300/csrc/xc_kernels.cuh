@@ -14,9 +14,13 @@ struct GateCell {
 };
 struct GateArgs {
     const void *x;
-    int d, V, npc;
-    const int *fp_rows;
-    int kfp;
+    int d, V;                // V: cameras of all view groups
+    const int *fp_rows;      // spatial-sample token rows, group by group, camera by camera
+    // view group g: cameras [g_cam0[g], g_cam0[g + 1]) of g_npc[g] tokens each
+    // from token g_tok0[g]; g_kfp[g] sample rows per camera from row g_fp0[g]
+    int n_groups, n_rows;    // n_rows: sample rows of all cameras
+    int g_cam0[XC_MAX_GROUPS + 1], g_tok0[XC_MAX_GROUPS], g_npc[XC_MAX_GROUPS], g_fp0[XC_MAX_GROUPS],
+        g_kfp[XC_MAX_GROUPS];
     int n_slices;            // 64-column slices: one CTA per (camera, slice)
     float *phi;
     float *phi_act;
@@ -33,6 +37,18 @@ struct GateArgs {
     float *part;             // scratch [V * n_slices][8]
     unsigned *ticket;        // scratch, zero before the launch (left zero)
 };
+// One view group of V cameras, npc tokens and kfp sample rows each.
+inline void gate_single_group(GateArgs &g, int V, int npc, int kfp) {
+    g.V = V;
+    g.n_groups = 1;
+    g.n_rows = V * kfp;
+    g.g_cam0[0] = 0;
+    g.g_cam0[1] = V;
+    g.g_tok0[0] = 0;
+    g.g_npc[0] = npc;
+    g.g_fp0[0] = 0;
+    g.g_kfp[0] = kfp;
+}
 // Bytes of scratch of one gate launch (partials, then the ticket at *ticket_off).
 size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off);
 template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);

@@ -1,7 +1,8 @@
 """AR rollout driver over the C ABI (Section 2.1 inference loop).
 
 Chunk n: x = eps_n; for t < S: v = xc_chunk_step(x, sigma_t, t); x += (sigma_{t+1}
-- sigma_t) v (Euler step, xc_euler_update); then the KV-update pass on the
+- sigma_t) v (Euler step, xc_euler_update); then, on a KV-update chunk (every
+chunk, or n mod P == P - 1 with kv_period P > 0), the KV-update pass on the
 chunk's clean latent at sigma = 0.  Actions are replayed one chunk at a time
 (closed-loop protocol, Section 3.1.3).  All arithmetic runs in the CUDA
 library; this module only moves buffers and sequences calls.
@@ -48,8 +49,10 @@ def rollout(xc: XCache, traj, n_chunks: int, gate: GateParams, sigmas=DEFAULT_SI
                 if keep_trace:
                     tr_n.append(tr.float().cpu().numpy())
                 xc.euler(x, v, sigmas[t + 1] - sigmas[t])
-            clean.copy_(torch.from_numpy(np.ascontiguousarray(traj.clean(n), dtype=np.float32)))
-            st_n.append(xc.chunk_step(clean, a, 0.0, S, True, gate, v_out=None, want_stats=want_stats))
+            P = int(getattr(cfg, "kv_period", 0))
+            if P == 0 or n % P == P - 1:
+                clean.copy_(torch.from_numpy(np.ascontiguousarray(traj.clean(n), dtype=np.float32)))
+                st_n.append(xc.chunk_step(clean, a, 0.0, S, True, gate, v_out=None, want_stats=want_stats))
             finals.append(x.cpu().numpy().astype(np.float64))
             stats.append(st_n)
             traces.append(tr_n)

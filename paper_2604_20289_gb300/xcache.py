@@ -20,6 +20,7 @@ XC_F32, XC_BF16 = 0, 1
 XC_DEC_FORCED, XC_DEC_COMPUTE, XC_DEC_SKIP = 0, 1, 2
 XC_EPI_BIAS, XC_EPI_GELU, XC_EPI_RESID_GATE, XC_EPI_RESID_CACHE = 0, 1, 2, 3
 XC_MAX_BLOCKS = 64
+XC_MAX_GROUPS = 4
 STATUS_NAMES = {0: "XC_OK", 1: "XC_EINVAL", 2: "XC_ESTATE", 3: "XC_ENOMEM", 4: "XC_ECUDA",
                 5: "XC_ENUMERIC", 6: "XC_ETIMEOUT"}
 
@@ -34,7 +35,11 @@ class ModelCfg(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int) for n in (
         "n_blocks", "d_model", "n_heads", "head_dim", "d_ffn", "c_latent", "action_dim",
         "n_cams", "frames", "grid_h", "grid_w", "kv_window_chunks", "n_denoise_steps", "dtype",
-        "t_freq_dim")] + [("ln_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+        "t_freq_dim")] + [("ln_eps", ctypes.c_float), ("rope_theta", ctypes.c_float),
+                          ("kv_period", ctypes.c_int), ("n_groups", ctypes.c_int),
+                          ("group_cams", ctypes.c_int * XC_MAX_GROUPS),
+                          ("group_h", ctypes.c_int * XC_MAX_GROUPS),
+                          ("group_w", ctypes.c_int * XC_MAX_GROUPS)]
 
 
 WEIGHT_NAMES = ("pe_w", "pe_b", "t_w1", "t_b1", "t_w2", "t_b2", "a_w1", "a_b1", "a_w2", "a_b2",
@@ -52,7 +57,7 @@ class GateParams(ctypes.Structure):
                 ("front_anchors", ctypes.c_int), ("back_anchors", ctypes.c_int),
                 ("warmup_chunks", ctypes.c_int), ("max_skips", ctypes.c_int),
                 ("protect_step0", ctypes.c_int), ("step0_strict_tau", ctypes.c_float),
-                ("fp_tokens", ctypes.c_int), ("fp_refresh", ctypes.c_int),
+                ("fp_tokens", ctypes.c_int), ("fp_refresh", ctypes.c_int), ("fp_linear", ctypes.c_int),
                 ("replay_skip", ctypes.POINTER(ctypes.c_uint8))]
 
 
@@ -151,10 +156,19 @@ def dtype_code(dtype) -> int:
 
 
 def model_cfg(cfg) -> ModelCfg:
-    """ModelCfg from any object with the shape attributes (e.g. xc_inputs.ModelCfg)."""
-    return ModelCfg(cfg.n_blocks, cfg.d_model, cfg.n_heads, cfg.head_dim, cfg.d_ffn, cfg.c_latent,
-                    cfg.action_dim, cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, cfg.kv_window,
-                    cfg.n_steps, dtype_code(cfg.dtype), cfg.t_freq, cfg.ln_eps, cfg.rope_theta)
+    """ModelCfg from any object with the shape attributes (e.g. xc_inputs.ModelCfg);
+    optional ``view_groups`` ((cameras, grid_h, grid_w), ...) and ``kv_period``."""
+    m = ModelCfg(cfg.n_blocks, cfg.d_model, cfg.n_heads, cfg.head_dim, cfg.d_ffn, cfg.c_latent,
+                 cfg.action_dim, cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, cfg.kv_window,
+                 cfg.n_steps, dtype_code(cfg.dtype), cfg.t_freq, cfg.ln_eps, cfg.rope_theta)
+    m.kv_period = int(getattr(cfg, "kv_period", 0))
+    groups = tuple(getattr(cfg, "view_groups", ()))
+    if len(groups) > XC_MAX_GROUPS:
+        raise ValueError(f"at most {XC_MAX_GROUPS} view groups")
+    m.n_groups = len(groups)
+    for i, (c, h, w) in enumerate(groups):
+        m.group_cams[i], m.group_h[i], m.group_w[i] = c, h, w
+    return m
 
 
 def gate_params(**kw) -> GateParams:

@@ -71,8 +71,10 @@ def compare_decisions(o_stats, g_stats, p):
     return None
 
 
-def replay_of(o_stats):
-    return [[[d == O.Decision.SKIP for d in s["decision"]] for s in ch[:-1]] for ch in o_stats]
+def replay_of(o_stats, n_steps=4):
+    """Skip decisions of the denoising passes (a chunk's stats end with its
+    KV-update pass, when it has one)."""
+    return [[[d == O.Decision.SKIP for d in s["decision"]] for s in ch[:n_steps]] for ch in o_stats]
 
 
 # ------------------------------------------------------ fp32 tiny model
@@ -224,3 +226,90 @@ def test_reset_reproduces_rollout(cfg):
     for x, y in zip(a["final"], b["final"]):
         np.testing.assert_array_equal(x, y)
     np.testing.assert_array_equal(decisions(a["stats"]), decisions(b["stats"]))
+
+
+# ------------------------------------- view groups, 1-D fallback, KV period
+def _replay_and_free(cfg, op, gp, n_chunks, fp32_tol=None, per_block=False):
+    """Decision-replay numerics (fp32: max|err| <= 1e-4 x RMS per final
+    latent; bf16: per-block rel-L2 <= 1e-2, final <= 3e-2) and free-running
+    decisions against the oracle."""
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=n_chunks)
+    ref = O.rollout(cfg, w, traj, op, n_chunks, keep_trace=per_block)
+    rep = gpu_rollout(xc, traj, n_chunks, gp, replay=replay_of(ref["stats"]), keep_trace=per_block)
+    for n in range(n_chunks):          # chunk by chunk: KV-update passes vary with kv_period
+        np.testing.assert_array_equal(decisions(rep["stats"][n:n + 1]), decisions(ref["stats"][n:n + 1]))
+    for n in range(n_chunks):
+        want, got = ref["final"][n], rep["final"][n]
+        if cfg.dtype == "f32":
+            rms = np.sqrt(np.mean(want ** 2))
+            assert np.max(np.abs(got - want)) <= 1e-4 * rms, (n, np.max(np.abs(got - want)) / rms)
+        else:
+            assert rel_l2(got, want) <= 3e-2, n
+            if per_block:
+                for t in range(cfg.n_steps):
+                    for b in range(cfg.n_blocks):
+                        e = rel_l2(rep["trace"][n][t][b], ref["trace"][n][t][b])
+                        assert e <= 1e-2, (n, t, b, e)
+    xc.reset()
+    free = gpu_rollout(xc, traj, n_chunks, gp)
+    compare_decisions(ref["stats"], free["stats"], op)
+    return ref
+
+
+@pytest.mark.parametrize("linear", [0, 1], ids=["grid", "linear"])
+def test_view_groups_f32_rollout_parity(linear):
+    """Two view groups of different grids (ragged 232-token chunk): per-group
+    fingerprints, the RoPE camera index counting across groups; with
+    ``linear`` the 1-D fallback sample."""
+    op, gp = params(tau_floor=0.93, tau_dev=10.0, fp_linear=linear)
+    ref = _replay_and_free(X.GROUPS_F32, op, gp, X.GROUPS_F32.n_chunks)
+    dec = decisions(ref["stats"])
+    assert (dec == O.Decision.SKIP).any() and (dec == O.Decision.COMPUTE).any()
+
+
+def test_view_groups_bf16_per_block_parity():
+    """Front / side / rear groups of 3 + 2 + 2 cameras on the tensor-core path."""
+    op, gp = params(tau_floor=0.92, tau_dev=10.0)
+    ref = _replay_and_free(X.GROUPS_BF16, op, gp, X.GROUPS_BF16.n_chunks, per_block=True)
+    assert (decisions(ref["stats"]) == O.Decision.SKIP).any()
+
+
+@pytest.mark.parametrize("cfg,P", [(X.TINY_F32, 3), (X.MID_HD64, 2)], ids=["tiny_f32_P3", "mid_bf16_P2"])
+def test_kv_period_rollout_parity(cfg, P):
+    """Periodic KV-update chunks: force-compute denoising passes on chunks
+    n mod P == P - 1, no KV pass elsewhere, ring of KV-update chunks only."""
+    cfg = cfg.replace(name=cfg.name + f"_kvp{P}", kv_period=P)
+    op, gp = params(tau_floor=0.92, tau_dev=10.0)
+    ref = _replay_and_free(cfg, op, gp, cfg.n_chunks, per_block=cfg.dtype == "bf16")
+    for n, ch in enumerate(ref["stats"]):
+        assert len(ch) == cfg.n_steps + (1 if n % P == P - 1 else 0)
+        if n % P == P - 1:
+            assert (decisions([ch]) == O.Decision.FORCED).all()
+    assert any((decisions([ch]) == O.Decision.SKIP).any() for ch in ref["stats"])
+
+
+def test_kv_period_call_order():
+    cfg = X.TINY_F32.replace(name="tiny_f32_kvp3_order", kv_period=3)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=2)
+    x = torch.tensor(traj.noise(0), dtype=torch.float32, device="cuda")
+    a = traj.action(0)
+    g = xb.gate_params()
+    for t in range(cfg.n_steps):
+        xc.chunk_step(x, a, 1.0, t, False, g)
+    # chunk 0 (0 mod 3 != 2) has no KV-update pass: it ended after pass S-1
+    assert xb.LIB.xc_chunk_index(xc.ctx) == 1
+    with pytest.raises(xb.XCacheError):               # nor has chunk 1
+        xc.chunk_step(x, a, 0.0, 0, True, g)
+    assert xb.LIB.xc_chunk_index(xc.ctx) == 1
+    for t in range(cfg.n_steps):
+        xc.chunk_step(x, a, 1.0, t, False, g)
+    assert xb.LIB.xc_chunk_index(xc.ctx) == 2
+    for t in range(cfg.n_steps):
+        xc.chunk_step(x, a, 1.0, t, False, g)
+    assert xb.LIB.xc_chunk_index(xc.ctx) == 2          # chunk 2 waits for its KV pass
+    with pytest.raises(xb.XCacheError):
+        xc.chunk_step(x, a, 1.0, 0, False, g)
+    xc.chunk_step(x, a, 0.0, 0, True, g)
+    assert xb.LIB.xc_chunk_index(xc.ctx) == 3

@@ -162,8 +162,17 @@ STRESS_1P3B = DIT_1P3B.replace(name="stress_dit1p3b_200chunks", n_chunks=200)
 MID_HD64 = ModelCfg("mid_bf16_3blk_d256_hd64", 3, 256, 4, 64, 1024, 2, 3, 10, 14, 3, 4)
 MID_HD128 = ModelCfg("mid_bf16_2blk_d256_hd128", 2, 256, 2, 128, 768, 2, 3, 10, 14, 3, 4)
 
+# View-group parity shapes (grid_h / grid_w repeat group 0's grid): a tiny
+# fp32 model with two groups whose cameras are larger than the K = 32 sample
+# (232 tokens), and a bf16 model with a front / side / rear layout of 3 + 2 + 2
+# cameras (Section 2.3.1; 2196 tokens = 17 x 128 + 20).
+GROUPS_F32 = ModelCfg("groups_f32_2blk_d64_3cam", 2, 64, 4, 16, 256, 3, 2, 6, 8, 3, 6, dtype="f32",
+                      view_groups=((2, 6, 8), (1, 4, 5)))
+GROUPS_BF16 = ModelCfg("groups_bf16_2blk_d256_7cam", 2, 256, 4, 64, 1024, 7, 3, 10, 14, 3, 4,
+                       view_groups=((3, 10, 14), (2, 8, 12), (2, 6, 10)))
+
 ALL_CFGS = {c.name: c for c in (TINY_F32, SMALL_BF16, DIT_1P3B, DIT_14B, STRESS_1P3B,
-                                  MID_HD64, MID_HD128)}
+                                  MID_HD64, MID_HD128, GROUPS_F32, GROUPS_BF16)}
 
 
 # --------------------------------------------------------------------------
