@@ -360,10 +360,34 @@ class OracleModel:
     def ln_mod(self, x, shift, scale):
         return self.R(layer_norm(x, self.cfg.ln_eps) * (1.0 + scale) + shift)
 
+    def context_kv(self, b: int, context: np.ndarray):
+        """Keys and values of block b's cross-attention over the chunk's
+        condition tokens (objects, lanes, text; Section 2.1 and 2.5): the
+        tokens [n_ctx, d_ctx] (rounded to the storage type) times W_kv plus
+        bias, split into k and v [n_ctx, H, hd].  No RoPE."""
+        cfg, w, R = self.cfg, self.w, self.R
+        n, d, H, hd = context.shape[0], cfg.d_model, cfg.n_heads, cfg.head_dim
+        kv = R(R(np.asarray(context, np.float64)) @ w["ca_kv_w"][b] + w["ca_kv_b"][b])
+        return kv[:, :d].reshape(n, H, hd), kv[:, d:].reshape(n, H, hd)
+
+    def cross_attention(self, b: int, x1: np.ndarray, ctx_kv):
+        """Cross-attention layer of block b (reading c26): x1 + (attention of
+        LN(x1) gamma + beta projected by W_q, over the condition keys and
+        values) W_o + b_o.  No modulation and no gate."""
+        cfg, w, R = self.cfg, self.w, self.R
+        L, d, H, hd = x1.shape[0], cfg.d_model, cfg.n_heads, cfg.head_dim
+        h = R(layer_norm(x1, cfg.ln_eps) * w["ca_ln_w"][b] + w["ca_ln_b"][b])
+        q = R(h @ w["ca_q_w"][b] + w["ca_q_b"][b]).reshape(L, H, hd)
+        kc, vc = ctx_kv
+        o = R(attention(q, kc, vc).reshape(L, d))
+        return R(x1 + (o @ w["ca_o_w"][b] + w["ca_o_b"][b]))
+
     def block(self, b: int, x_in: np.ndarray, mod: np.ndarray, past_k: list, past_v: list,
-              pos: np.ndarray):
+              pos: np.ndarray, ctx_kv=None):
         """x_{t,b} = x_{t,b-1} + f_b(x_{t,b-1}; c_t) (Eq. 1).  Returns the block
-        output and this pass's (k, v) of the current chunk [L, H, hd]."""
+        output and this pass's (k, v) of the current chunk [L, H, hd].  With
+        ``ctx_kv`` (this block's condition keys / values) the cross-attention
+        layer sits between the self-attention and the FFN."""
         cfg, w, R = self.cfg, self.w, self.R
         L, d, H, hd = x_in.shape[0], cfg.d_model, cfg.n_heads, cfg.head_dim
         sh1, sc1, g1, sh2, sc2, g2 = mod
@@ -379,6 +403,8 @@ class OracleModel:
         vals = np.concatenate(past_v + [v], axis=0)
         o = R(attention(q, keys, vals).reshape(L, d))
         x1 = R(x_in + g1 * (o @ w["o_w"][b] + w["o_b"][b]))
+        if ctx_kv is not None:
+            x1 = self.cross_attention(b, x1, ctx_kv)
         h2 = self.ln_mod(x1, sh2, sc2)
         u = R(gelu_tanh(h2 @ w["f1_w"][b] + w["f1_b"][b]))
         x2 = R(x1 + g2 * (u @ w["f2_w"][b] + w["f2_b"][b]))
@@ -423,6 +449,12 @@ class OracleXCache:
         self.ring_k = [[] for _ in range(cfg.n_blocks)]
         self.ring_v = [[] for _ in range(cfg.n_blocks)]
         self.cells = [[GateCell() for _ in range(cfg.n_blocks)] for _ in range(cfg.n_steps)]
+        self.ctx_kv = None
+
+    def set_context(self, context: np.ndarray):
+        """Condition tokens for the following passes (models with
+        cross-attention): every block's keys and values over them."""
+        self.ctx_kv = [self.model.context_kv(b, context) for b in range(self.cfg.n_blocks)]
 
     def is_kv_chunk(self, n: int) -> bool:
         P = getattr(self.cfg, "kv_period", 0)
@@ -466,6 +498,9 @@ class OracleXCache:
         elif step != self.next_step or step >= S:
             raise RuntimeError("denoising step out of order")
         forced_chunk = getattr(cfg, "kv_period", 0) > 0 and kv_chunk
+        xattn = getattr(cfg, "d_ctx", 0) > 0
+        if xattn and self.ctx_kv is None:
+            raise RuntimeError("cross-attention model without condition tokens")
         mods, hm = M.cond(sigma, action)
         pos = group_token_positions(cfg.groups, cfg.frames, n)
         x = M.patch_embed(latent)
@@ -495,7 +530,8 @@ class OracleXCache:
                 if p.fp_refresh == 1:
                     cell.phi_sp, cell.phi_gl, cell.phi_act = phi
             else:
-                x_out, k, v = M.block(b, x, mods[b], self.ring_k[b], self.ring_v[b], pos)
+                x_out, k, v = M.block(b, x, mods[b], self.ring_k[b], self.ring_v[b], pos,
+                                      self.ctx_kv[b] if xattn else None)
                 if is_kv_update:
                     kv_new[b] = (k, v)
                 elif gated_block:
@@ -533,7 +569,8 @@ SIGMAS = (1.0, 0.75, 0.5, 0.25, 0.0)
 
 def rollout(cfg, weights, traj, params: GateParams, n_chunks: int, replay=None,
             keep_trace: bool = False):
-    """Chunk n: x = eps_n; for t < S: v = step(x, sigma_t); x += (sigma_{t+1} -
+    """Chunk n: (cross-attention models: set the chunk's condition tokens)
+    x = eps_n; for t < S: v = step(x, sigma_t); x += (sigma_{t+1} -
     sigma_t) v (Euler, flow matching); then, on a KV-update chunk, the
     KV-update pass on the chunk's clean latent x_c[n] at sigma = 0
     (teacher-forced, reading c22).
@@ -545,6 +582,8 @@ def rollout(cfg, weights, traj, params: GateParams, n_chunks: int, replay=None,
     for n in range(n_chunks):
         x = np.asarray(traj.noise(n), np.float64)
         a = traj.action(n)
+        if getattr(cfg, "d_ctx", 0) > 0:
+            oc.set_context(traj.context(n))
         st_n, tr_n = [], []
         for t in range(S):
             tr = [] if keep_trace else None

@@ -559,3 +559,70 @@ def test_kv_period_ring_holds_kv_chunks_only():
     for n in (2, 3, 4, 5):                                  # resident: (1), (1, 3)
         assert np.abs(kv1[n] - ref[n]).max() > 1e-6
     np.testing.assert_array_equal(kv1[6], ref[6])          # ring (3, 5): chunk 1 evicted
+
+
+# --------------------------------------- cross-attention conditioning (c26)
+def _xattn_model():
+    cfg = X.XATTN_F32
+    return cfg, O.OracleModel(cfg, X.make_weights(cfg))
+
+
+def test_cross_attention_brute_force():
+    """Explicit loops over queries, heads and condition tokens."""
+    cfg, m = _xattn_model()
+    d, H, hd, b = cfg.d_model, cfg.n_heads, cfg.head_dim, 1
+    x1 = rng.standard_normal((5, d))
+    ctx = rng.standard_normal((3, cfg.d_ctx))
+    w = m.w
+    got = m.cross_attention(b, x1, m.context_kv(b, ctx))
+    want = np.empty_like(x1)
+    for i in range(x1.shape[0]):
+        mu = sum(x1[i]) / d
+        var = sum((x1[i] - mu) ** 2) / d
+        h = (x1[i] - mu) / math.sqrt(var + cfg.ln_eps) * w["ca_ln_w"][b] + w["ca_ln_b"][b]
+        q = h @ w["ca_q_w"][b] + w["ca_q_b"][b]
+        o = np.zeros(d)
+        for hh in range(H):
+            sl = slice(hh * hd, (hh + 1) * hd)
+            scores = []
+            for j in range(ctx.shape[0]):
+                kv = ctx[j] @ w["ca_kv_w"][b] + w["ca_kv_b"][b]
+                scores.append((float(q[sl] @ kv[:d][sl]) / math.sqrt(hd), kv[d:][sl]))
+            mx = max(s for s, _ in scores)
+            den = sum(math.exp(s - mx) for s, _ in scores)
+            for s, v in scores:
+                o[sl] += math.exp(s - mx) / den * v
+        want[i] = x1[i] + o @ w["ca_o_w"][b] + w["ca_o_b"][b]
+    np.testing.assert_allclose(got, want, rtol=1e-10, atol=1e-10)
+
+
+def test_cross_attention_token_invariances():
+    """No positional encoding on condition tokens: permuting them changes
+    nothing; repeating every token m times changes nothing (softmax over
+    identical keys); one token gives its value to every query."""
+    cfg, m = _xattn_model()
+    x1 = rng.standard_normal((7, cfg.d_model))
+    ctx = rng.standard_normal((4, cfg.d_ctx))
+    base = m.cross_attention(0, x1, m.context_kv(0, ctx))
+    perm = m.cross_attention(0, x1, m.context_kv(0, ctx[[2, 0, 3, 1]]))
+    np.testing.assert_allclose(perm, base, rtol=1e-12, atol=1e-12)
+    rep = m.cross_attention(0, x1, m.context_kv(0, np.repeat(ctx, 3, axis=0)))
+    np.testing.assert_allclose(rep, base, rtol=1e-12, atol=1e-12)
+    k1, v1 = m.context_kv(0, ctx[:1])
+    one = m.cross_attention(0, x1, (k1, v1))
+    v = v1.reshape(1, -1)
+    np.testing.assert_allclose(one - x1, np.broadcast_to(v @ m.w["ca_o_w"][0] + m.w["ca_o_b"][0], x1.shape),
+                               rtol=1e-12, atol=1e-12)
+
+
+def test_cross_attention_with_zero_output_is_plain_block():
+    cfg, m = _xattn_model()
+    m.w["ca_o_w"][:] = 0.0
+    m.w["ca_o_b"][:] = 0.0
+    x = rng.standard_normal((cfg.tokens, cfg.d_model))
+    mods, _ = m.cond(0.5, np.array([0.3, -0.4]))
+    pos = O.token_positions(cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, 0)
+    ctx = rng.standard_normal((5, cfg.d_ctx))
+    a, _, _ = m.block(0, x, mods[0], [], [], pos, m.context_kv(0, ctx))
+    b, _, _ = m.block(0, x, mods[0], [], [], pos)
+    np.testing.assert_array_equal(a, b)

@@ -110,7 +110,9 @@ class ModelCfg:
     the groups' tokens follow one another in that order, each group camera by
     camera, and ``n_cams`` is then the total camera count.  ``kv_period`` P
     > 0 makes every P-th chunk (n mod P == P - 1) the one whose clean latent
-    feeds the KV-update pass; 0 runs that pass after every chunk."""
+    feeds the KV-update pass; 0 runs that pass after every chunk.  ``d_ctx``
+    > 0 adds a cross-attention layer to every block, attending to up to
+    ``max_ctx`` condition tokens of width ``d_ctx`` per chunk."""
     name: str
     n_blocks: int
     d_model: int
@@ -132,6 +134,8 @@ class ModelCfg:
     rope_theta: float = 10000.0
     view_groups: tuple = ()
     kv_period: int = 0
+    d_ctx: int = 0               # > 0: cross-attention to d_ctx-wide condition tokens
+    max_ctx: int = 0             # most condition tokens a chunk may carry
 
     @property
     def groups(self) -> tuple:
@@ -171,8 +175,13 @@ GROUPS_F32 = ModelCfg("groups_f32_2blk_d64_3cam", 2, 64, 4, 16, 256, 3, 2, 6, 8,
 GROUPS_BF16 = ModelCfg("groups_bf16_2blk_d256_7cam", 2, 256, 4, 64, 1024, 7, 3, 10, 14, 3, 4,
                        view_groups=((3, 10, 14), (2, 8, 12), (2, 6, 10)))
 
+# Cross-attention parity shapes: condition tokens of width d_ctx, up to
+# max_ctx per chunk (count varying from chunk to chunk).
+XATTN_F32 = TINY_F32.replace(name="xattn_f32_2blk_d64", d_ctx=32, max_ctx=24)
+XATTN_BF16 = MID_HD64.replace(name="xattn_bf16_3blk_d256_hd64", d_ctx=128, max_ctx=300)
+
 ALL_CFGS = {c.name: c for c in (TINY_F32, SMALL_BF16, DIT_1P3B, DIT_14B, STRESS_1P3B,
-                                  MID_HD64, MID_HD128, GROUPS_F32, GROUPS_BF16)}
+                                  MID_HD64, MID_HD128, GROUPS_F32, GROUPS_BF16, XATTN_F32, XATTN_BF16)}
 
 
 # --------------------------------------------------------------------------
@@ -192,16 +201,22 @@ def weight_shapes(cfg: ModelCfg) -> dict:
         "f2_w": (B, F, d), "f2_b": (B, d),
         "head_w": (d, 2 * d), "head_b": (2 * d,), "head_tab": (2, d),
         "out_w": (d, C), "out_b": (C,),
+        **({} if cfg.d_ctx == 0 else {
+            "ca_ln_w": (B, d), "ca_ln_b": (B, d),
+            "ca_q_w": (B, d, d), "ca_q_b": (B, d),
+            "ca_kv_w": (B, cfg.d_ctx, 2 * d), "ca_kv_b": (B, 2 * d),
+            "ca_o_w": (B, d, d), "ca_o_b": (B, d)}),
     }
 
 
 BIAS_STD = 0.05
 BIASES = ("pe_b", "t_b1", "t_b2", "a_b1", "a_b2", "mod_b", "qkv_b", "o_b", "f1_b", "f2_b",
-          "head_b", "out_b")
+          "head_b", "out_b", "ca_ln_b", "ca_q_b", "ca_kv_b", "ca_o_b")
+GAINS = ("ca_ln_w",)             # 1 + N(0, BIAS_STD^2)
 
 
 def _init_std(name: str, shape: tuple) -> float:
-    if name in BIASES:
+    if name in BIASES or name in GAINS:
         return BIAS_STD
     fan_in, fan_out = shape[-2], shape[-1]           # [in, out]; tables [6|2, d]
     return math.sqrt(2.0 / (fan_in + fan_out))        # Xavier-normal
@@ -220,6 +235,8 @@ def make_weight(cfg: ModelCfg, name: str, seed: int = 0, block: int | None = Non
         per = int(np.prod(shape[1:]))
         w = normal(seed, cfg.name + "/" + name, per, offset=block * per) * std
         out_shape = shape[1:]
+    if name in GAINS:
+        w = 1.0 + w
     w = w.astype(np.float32).reshape(out_shape)
     return bf16_representable(w) if cfg.dtype == "bf16" else w
 
@@ -286,6 +303,23 @@ class Trajectory:
             self._clean.append(xc.astype(np.float32))
             self._eps.append(eps.astype(np.float32))
             self._act.append(np.asarray(a, dtype=np.float32).copy())
+        # condition tokens (cross-attention): a fixed text part of max_ctx / 2
+        # tokens, then object / lane tokens that drift AR(1) from chunk to
+        # chunk and whose count varies in [max_ctx / 4, max_ctx / 2]
+        self._ctx = []
+        if cfg.d_ctx > 0:
+            M, D = cfg.max_ctx, cfg.d_ctx
+            n_text = M // 2
+            text = normal(seed, f"{cfg.name}/ctx_text", n_text * D).reshape(n_text, D)
+            obj = None
+            for n in range(self.n_chunks):
+                rho = _rho_at(traj, n, self.n_chunks)
+                z = normal(seed, f"{cfg.name}/ctx_obj/{n}", (M - n_text) * D).reshape(M - n_text, D)
+                obj = z if obj is None else rho * obj + math.sqrt(1.0 - rho * rho) * z
+                lo = (M - n_text) // 2
+                n_obj = lo + int(uniform(seed, f"{cfg.name}/ctx_len/{n}", 1)[0] * (M - n_text - lo + 1))
+                n_obj = min(n_obj, M - n_text)
+                self._ctx.append(np.concatenate([text, obj[:n_obj]]).astype(np.float32))
 
     def clean(self, n: int) -> np.ndarray:
         return self._clean[n]
@@ -295,6 +329,11 @@ class Trajectory:
 
     def action(self, n: int) -> np.ndarray:
         return self._act[n]
+
+    def context(self, n: int) -> np.ndarray:
+        """Condition tokens of chunk n, [n_ctx(n), d_ctx] float32 (models with
+        cross-attention only)."""
+        return self._ctx[n]
 
 
 SIGMAS = (1.0, 0.75, 0.5, 0.25, 0.0)   # 4 Euler flow-matching passes, then sigma = 0
