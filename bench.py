@@ -55,6 +55,9 @@ def parse():
     ap.add_argument("--view-groups", default="",
                     help="view groups of the chunk as CAMSxHxW,... (e.g. 3x20x36,2x16x28,2x12x20); "
                          "default: the workload's single camera grid")
+    ap.add_argument("--xattn", type=int, default=0,
+                    help="add cross-attention to up to N condition tokens of width d_model per chunk "
+                         "(count varying per chunk in [3N/4, N]); 0 = none")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--calibrate", action="store_true", help="print gate-metric quantiles and exit")
@@ -154,7 +157,10 @@ def oracle_block_sample(cfg, seed: int = 0) -> float:
     w = {k: X.make_weight(cfg, k, seed) for k in ("t_w1", "t_b1", "t_w2", "t_b2", "a_w1", "a_b1", "a_w2",
                                                    "a_b2", "mod_w", "mod_b", "head_w", "head_b", "head_tab",
                                                    "pe_w", "pe_b", "out_w", "out_b")}
-    for k in ("blk_mod", "qkv_w", "qkv_b", "o_w", "o_b", "f1_w", "f1_b", "f2_w", "f2_b"):
+    per_block = ("blk_mod", "qkv_w", "qkv_b", "o_w", "o_b", "f1_w", "f1_b", "f2_w", "f2_b")
+    if cfg.d_ctx:
+        per_block += ("ca_ln_w", "ca_ln_b", "ca_q_w", "ca_q_b", "ca_kv_w", "ca_kv_b", "ca_o_w", "ca_o_b")
+    for k in per_block:
         w[k] = X.make_weight(cfg, k, seed, block=0)[None]
     m = O.OracleModel(cfg, w)
     mods, _ = m.cond(0.75, np.array([0.1, -0.2]))
@@ -166,8 +172,13 @@ def oracle_block_sample(cfg, seed: int = 0) -> float:
     past_v = [R(X.random_tensor(seed, f"bench/v{i}", (L, H, hd)).astype(np.float64))
               for i in range(cfg.kv_window - 1)]
     pos = O.group_token_positions(cfg.groups, cfg.frames, cfg.kv_window)
+    ctx = None
+    if cfg.d_ctx:
+        tokens = X.random_tensor(seed, "bench/ctx", (cfg.max_ctx, cfg.d_ctx)).astype(np.float64)
     t0 = time.perf_counter()
-    m.block(0, x, mods[0], past_k, past_v, pos)
+    if cfg.d_ctx:
+        ctx = m.context_kv(0, tokens)
+    m.block(0, x, mods[0], past_k, past_v, pos, ctx)
     return time.perf_counter() - t0
 
 
@@ -208,6 +219,8 @@ def workload_cfg(args):
                           n_cams=sum(g[0] for g in groups), grid_h=groups[0][1], grid_w=groups[0][2])
     if args.kv_period:
         cfg = cfg.replace(name=f"{cfg.name}_kvperiod{args.kv_period}", kv_period=args.kv_period)
+    if args.xattn:
+        cfg = cfg.replace(name=f"{cfg.name}_xattn{args.xattn}", d_ctx=cfg.d_model, max_ctx=args.xattn)
     return cfg
 
 
@@ -225,6 +238,8 @@ def config_of(cfg, args):
             "passes_per_chunk": cfg.n_steps + 1 if cfg.kv_period == 0 else
             f"{cfg.n_steps} + a KV-update pass every {cfg.kv_period} chunks",
             "view_groups": [list(g) for g in cfg.groups],
+            "cross_attention": None if cfg.d_ctx == 0 else
+            {"d_ctx": cfg.d_ctx, "max_ctx": cfg.max_ctx, "tokens_per_chunk": "3/4 max_ctx .. max_ctx"},
             "gate": {"tau_floor": args.tau_floor, "tau_dev": args.tau_dev, "other": "Table 1 defaults"},
             "l2": "not flushed: per-chunk working set (KV ring + residual cache + weights) > 129 MB L2",
             "parallelism": f"replicas x{args.gpus}"}
@@ -255,6 +270,7 @@ def main():
     noise = torch.stack([torch.from_numpy(traj.noise(n)) for n in range(n_total)]).to(dev)
     clean = torch.stack([torch.from_numpy(traj.clean(n)) for n in range(n_total)]).to(dev)
     acts = [traj.action(n) for n in range(n_total)]
+    ctx_tok = [torch.from_numpy(traj.context(n)).to(dev) for n in range(n_total)] if cfg.d_ctx else None
     stream = torch.cuda.current_stream()
     xc = xb.XCache(cfg, w, stream=stream)
     L, C, S = cfg.tokens, cfg.c_latent, cfg.n_steps
@@ -262,6 +278,8 @@ def main():
     v = torch.empty_like(x)
 
     def chunk(n, gate):
+        if ctx_tok is not None:
+            xc.set_context(ctx_tok[n])
         x.copy_(noise[n])
         for t in range(S):
             xc.chunk_step(x, acts[n], SIGMAS[t], t, False, gate, v_out=v, want_stats=False)
@@ -397,7 +415,7 @@ def predicted_speedup(xc, chunk, gate, args, cfg, t_all):
             chunk(n, g)
         return xc.profile_stop()
 
-    block_kinds = {"ln", "qkv", "attn", "oproj", "ffn1", "ffn2"}
+    block_kinds = {"ln", "qkv", "attn", "oproj", "xattn", "ffn1", "ffn2"}
     t_block = {}
     recs_all = run(xb.gate_params(enabled=0))
     kernel_us = {}
@@ -519,6 +537,8 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
     x_np, v_np, c_np = xh.numpy(), vh.numpy(), ch.numpy()
 
     def chunk(n):
+        if cfg.d_ctx:
+            xc.set_context(traj.context(n))
         x_np[:] = traj.noise(n)
         for t in range(S):
             xc.chunk_step(x_np, acts[n], SIGMAS[t], t, False, gate, v_out=v_np, want_stats=False)
@@ -543,8 +563,11 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
         sec = float(t.item())
     nbytes = L * C * 4
     kv = sum(has_kv_pass(cfg, n) for n in range(args.warmup, args.warmup + args.steps)) / args.steps
+    ctx_b = 0.0
+    if cfg.d_ctx:
+        ctx_b = sum(traj.context(n).nbytes for n in range(args.warmup, args.warmup + args.steps)) / args.steps
     return {"value": args.steps * world / sec, "unit": "chunks/s",
-            "h2d_bytes_per_step": (S + kv) * (nbytes + cfg.action_dim * 4),
+            "h2d_bytes_per_step": (S + kv) * (nbytes + cfg.action_dim * 4) + ctx_b,
             "d2h_bytes_per_step": S * nbytes}
 
 
@@ -561,6 +584,8 @@ def calibrate(xc, chunk, cfg, args):
     x = torch.empty(L, C, device="cuda")
     v = torch.empty_like(x)
     for n in range(args.warmup + args.steps):
+        if cfg.d_ctx:
+            xc.set_context(traj.context(n))
         x.copy_(torch.from_numpy(traj.noise(n)))
         for t in range(S):
             st = xc.chunk_step(x, traj.action(n), SIGMAS[t], t, False, g, v_out=v)

@@ -80,7 +80,16 @@ typedef enum {
  * force-compute mode (every block computes, the gate is not evaluated, the
  * residual and fingerprint caches are refreshed), and a chunk without one
  * ends after its last denoising pass.  The ring then holds the clean K/V of
- * the last kv_window_chunks - 1 KV-update chunks. */
+ * the last kv_window_chunks - 1 KV-update chunks.
+ *
+ * Cross-attention conditioning (condition tokens such as dynamic objects,
+ * lanes and text, Sections 2.1 and 2.5): with d_ctx > 0 every block gets a
+ * cross-attention layer between its self-attention and its FFN,
+ *   x1 <- x1 + softmax(q K_c^T / sqrt(head_dim)) V_c W_o + b_o,
+ *   q = (LN(x1) * gamma + beta) W_q + b_q,  [K_c | V_c] = C W_kv + b_kv,
+ * over the up to max_ctx condition tokens C [n_ctx][d_ctx] given by
+ * xc_set_context (no modulation, no gate, no RoPE).  XC_BF16 needs
+ * d_ctx % 64 == 0, XC_F32 d_ctx % 16 == 0.  d_ctx = 0: no cross-attention. */
 typedef struct {
     int n_blocks, d_model, n_heads, head_dim, d_ffn, c_latent, action_dim;
     int n_cams, frames, grid_h, grid_w;
@@ -89,6 +98,7 @@ typedef struct {
     int kv_period;
     int n_groups;
     int group_cams[XC_MAX_GROUPS], group_h[XC_MAX_GROUPS], group_w[XC_MAX_GROUPS];
+    int d_ctx, max_ctx;
 } xc_model_cfg;
 
 /* Host float32 weights, math convention y = x @ W with W stored [in][out]
@@ -104,12 +114,17 @@ typedef struct {
  *   f1_w [B][d][F] f1_b [B][F]      f2_w [B][F][d] f2_b [B][d]
  *   head_w [d][2d] head_b [2d] head_tab [2][d]    head (shift, scale)
  *   out_w [d][C] out_b [C]
+ * Cross-attention (d_ctx > 0 only, else ignored; D = d_ctx):
+ *   ca_ln_w [B][d] ca_ln_b [B][d]   LN gain gamma and bias beta
+ *   ca_q_w [B][d][d] ca_q_b [B][d]  ca_kv_w [B][D][2d] ca_kv_b [B][2d]
+ *   ca_o_w [B][d][d] ca_o_b [B][d]
  * The pointers are only read during xc_init. */
 typedef struct {
     const float *pe_w, *pe_b, *t_w1, *t_b1, *t_w2, *t_b2, *a_w1, *a_b1, *a_w2, *a_b2;
     const float *mod_w, *mod_b, *blk_mod;
     const float *qkv_w, *qkv_b, *o_w, *o_b, *f1_w, *f1_b, *f2_w, *f2_b;
     const float *head_w, *head_b, *head_tab, *out_w, *out_b;
+    const float *ca_ln_w, *ca_ln_b, *ca_q_w, *ca_q_b, *ca_kv_w, *ca_kv_b, *ca_o_w, *ca_o_b;
 } xc_weights;
 
 /* Gate knobs (Section 2.3-2.5); xc_gate_params_default() gives Table 1:
@@ -189,9 +204,18 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
                         int step_index, int is_kv_update, const xc_gate_params *gate,
                         float *v_out, xc_step_stats *stats);
 
+/* Condition tokens for the following passes (cross-attention models):
+ * context host or device float32 [n_ctx][d_ctx], 1 <= n_ctx <= max_ctx.
+ * Computes every block's condition keys and values on the context's stream;
+ * the tokens stay in use until the next call (and across xc_reset).  Passes
+ * of a cross-attention model before the first call return XC_ESTATE.
+ * Errors: XC_EINVAL (no cross-attention, bad n_ctx or NULL), XC_ENUMERIC
+ * (non-finite host value), XC_ECUDA. */
+xc_status xc_set_context(xc_ctx *ctx, const float *context, int n_ctx);
+
 /* Clears the KV ring, residual / fingerprint caches, EMA, staleness and the
  * chunk counter (the next chunk is a warmup chunk again, Section 2.2.3).
- * Weights are kept. */
+ * Weights and condition tokens are kept. */
 xc_status xc_reset(xc_ctx *ctx);
 
 /* Frees everything the context owns.  NULL is a no-op. */
@@ -214,21 +238,23 @@ xc_status xc_set_block_trace(xc_ctx *ctx, void *dev_buf);
  * error word (bounded-wait timeouts) as XC_ETIMEOUT. */
 xc_status xc_sync(xc_ctx *ctx);
 
-/* Chunk counter n (number of completed KV-update passes since reset). */
+/* Chunk counter n (chunks completed since reset). */
 int xc_chunk_index(const xc_ctx *ctx);
 
 /* ---- measurement (no counterpart in the paper; used by the benchmark) ---- */
 
-/* Kernel kinds of one forward pass. */
+/* Kernel kinds of one forward pass (XC_K_XATTN: the four launches of a
+ * cross-attention layer -- LN, q projection, attention, output projection). */
 typedef enum {
     XC_K_COND = 0, XC_K_EMBED, XC_K_GATE, XC_K_LN, XC_K_QKV, XC_K_ATTN, XC_K_OPROJ,
-    XC_K_FFN1, XC_K_FFN2, XC_K_REUSE, XC_K_HEAD, XC_K_COUNT
+    XC_K_FFN1, XC_K_FFN2, XC_K_REUSE, XC_K_HEAD, XC_K_XATTN, XC_K_COUNT
 } xc_kernel_kind;
 
 /* One timed launch: CUDA-event duration on the context's stream, the block
  * and pass it belongs to, the gate decision of that block in that pass
  * (xc_decision; kernels of a skipped block exit at once), the chunk index
- * and the number of resident keys the pass attended to. */
+ * and the number of resident keys the pass attended to (condition tokens
+ * for XC_K_XATTN). */
 typedef struct {
     int kind, block, pass_seq, decision, chunk, n_keys;
     float ms;

@@ -526,6 +526,24 @@ template cudaError_t head<bf16>(const bf16 *, const float *, const float *, cons
 
 // --------------------------------------------------------- weight layout
 // Wt[n][k] = convert(W[k][n]) for one [K][N] float32 matrix (32x32 tiles).
+// fp32 -> storage type, elementwise (condition tokens of the cross-attention).
+template <typename T>
+__global__ void __launch_bounds__(256) convert_f32_kernel(const float *__restrict__ in, T *__restrict__ out, long n) {
+    for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+        if constexpr (sizeof(T) == 2)
+            out[i] = __float2bfloat16_rn(in[i]);
+        else
+            out[i] = in[i];
+    }
+}
+template <typename T>
+cudaError_t convert_f32(const float *in, T *out, long n, int n_sm, cudaStream_t st) {
+    const long want = (n + 255) / 256, cap = 4L * n_sm;
+    convert_f32_kernel<T><<<(int)(want < cap ? (want > 0 ? want : 1) : cap), 256, 0, st>>>(in, out, n);
+    return cudaGetLastError();
+}
+template cudaError_t convert_f32<bf16>(const float *, bf16 *, long, int, cudaStream_t);
+
 template <typename T>
 __global__ void transpose_convert_kernel(const float *__restrict__ W, T *__restrict__ Wt, int K, int N) {
     __shared__ float tile[32][33];

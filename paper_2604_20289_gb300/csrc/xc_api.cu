@@ -114,7 +114,7 @@ bool is_host_ptr(const void *p) {
 // Everything the per-pass block loop takes from the host (besides buffers
 // that stay fixed for the context's lifetime).
 struct PassSig {
-    int t, kv, eval_mode, slot, n_keys, replay;
+    int t, kv, eval_mode, slot, n_keys, replay, n_ctx;
     uint64_t replay_bits;
     xc_gate_params p;                 // replay_skip pointer cleared
     const void *lat, *v, *trace;
@@ -169,6 +169,18 @@ struct xc_ctx {
     // number of KV-update passes so far (the ring's write count)
     int kv_period, kvc;
 
+    // cross-attention conditioning (d_ctx > 0): per-block weights, the
+    // current condition tokens and their per-block keys / values
+    bool xattn;
+    int d_ctx, max_ctx, n_ctx;                 // n_ctx: current condition tokens (0 = none yet)
+    float *ca_scale, *ca_shift;                // [B][d] gamma - 1 and beta (LN affine run as ln_mod)
+    void *ca_q_wt, *ca_kv_wt, *ca_o_wt;        // [B][d][d], [B][2d][d_ctx], [B][d][d] activation dtype
+    float *ca_q_b, *ca_kv_b, *ca_o_b;          // [B][d], [B][2d], [B][d]
+    float *ones;                               // [d] gate of the ungated residual epilogue
+    float *ctx_in;                             // [max_ctx][d_ctx] fp32 staging
+    void *ctx_act;                             // [max_ctx][d_ctx] bf16 copy (bf16 models)
+    void *ctx_k, *ctx_v;                       // [B][max_ctx][d] condition keys / values
+
     // per pass
     uint8_t *flags;
     float *s_cos, *d_max, *tau;
@@ -201,6 +213,7 @@ struct xc_ctx {
     CUtensorMap tm_h, tm_o, tm_u, tm_q;
     int bn_qkv, bn_o, bn_f1, bn_f2;
     std::vector<CUtensorMap> tm_wqkv, tm_wo, tm_w1, tm_w2, tm_rk, tm_rv;
+    std::vector<CUtensorMap> tm_caq, tm_cao, tm_cak, tm_cav, tm_ck, tm_cv;   // cross-attention
 
     int n, next_step;
     void *trace;
@@ -295,6 +308,13 @@ bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
         if (c->head_dim != 16 && c->head_dim != 32 && c->head_dim != 64) return bad("f32 head_dim");
     } else {
         return bad("dtype must be XC_F32 or XC_BF16");
+    }
+    if (c->d_ctx < 0 || c->max_ctx < 0) return bad("d_ctx / max_ctx < 0");
+    if (c->d_ctx > 0) {
+        if (c->max_ctx < 1) return bad("cross-attention needs max_ctx >= 1");
+        if (c->d_ctx % 16 != 0) return bad("d_ctx % 16 != 0");
+        if (c->dtype == XC_BF16 && c->d_ctx % 64 != 0) return bad("bf16 cross-attention needs d_ctx % 64 == 0");
+        if ((long long)c->max_ctx * c->d_ctx > (1LL << 28) || c->max_ctx > (1 << 24)) return bad("context too large");
     }
     return true;
 }
@@ -416,7 +436,7 @@ int prof_begin(xc_ctx *ctx, int kind, int block) {
     r.pass_seq = ctx->pass_seq;
     r.decision = -1;
     r.chunk = ctx->n;
-    r.n_keys = ctx->cur_keys;
+    r.n_keys = kind == XC_K_XATTN ? ctx->n_ctx : ctx->cur_keys;
     r.ms = 0.0f;
     return i;
 }
@@ -642,6 +662,50 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             const float *W = reinterpret_cast<const float *>(ctx->o_wt) + (size_t)b * d * d;
             LAUNCH(XC_K_OPROJ, b, 1, gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
         }
+        if (ctx->xattn) {
+            // cross-attention layer over the condition tokens, in place on x1:
+            // x1 <- x1 + attn((LN(x1) gamma + beta) W_q + b_q, K_c, V_c) W_o + b_o
+            const size_t cb = (size_t)b * ctx->max_ctx * d;
+            LAUNCH(XC_K_XATTN, b, 1,
+                   ln_mod<T>(x1, ctx->ca_shift + (size_t)b * d, ctx->ca_scale + (size_t)b * d, hb, L, d,
+                             ctx->cfg.ln_eps, flag, st));
+            memset(&ep, 0, sizeof ep);
+            ep.M = L;
+            ep.N = d;
+            ep.bias = ctx->ca_q_b + (size_t)b * d;
+            ep.out = qb;
+            if constexpr (sizeof(T) == 2) {
+                LAUNCH(XC_K_XATTN, b, 1,
+                       gemm_tc(EPI_BIAS, ctx->bn_o, ctx->tm_h, ctx->tm_caq[b], ep, d, flag, ctx->d_err, st));
+                int n_x = 1;
+                LAUNCH(XC_K_XATTN, b, n_x,
+                       attn_tc(hd, ctx->tm_q, ctx->tm_ck[b], ctx->tm_cv[b], reinterpret_cast<bf16 *>(ob), L,
+                               ctx->n_ctx, ctx->H, d, ctx->attn_ws, ctx->attn_ws_bytes, flag, ctx->d_err, &n_x, st));
+            } else {
+                const float *W = reinterpret_cast<const float *>(ctx->ca_q_wt) + (size_t)b * d * d;
+                LAUNCH(XC_K_XATTN, b, 1, gemm_simt(EPI_BIAS, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+                LAUNCH(XC_K_XATTN, b, 1,
+                       attn_simt(hd, reinterpret_cast<const float *>(qb),
+                                 reinterpret_cast<const float *>(ctx->ctx_k) + cb,
+                                 reinterpret_cast<const float *>(ctx->ctx_v) + cb, reinterpret_cast<float *>(ob), L,
+                                 ctx->n_ctx, ctx->H, flag, st));
+            }
+            memset(&ep, 0, sizeof ep);
+            ep.M = L;
+            ep.N = d;
+            ep.bias = ctx->ca_o_b + (size_t)b * d;
+            ep.gate = ctx->ones;
+            ep.resid = x1;
+            ep.out = x1;
+            if constexpr (sizeof(T) == 2) {
+                LAUNCH(XC_K_XATTN, b, 1,
+                       gemm_tc(EPI_RESID_GATE, ctx->bn_o, ctx->tm_o, ctx->tm_cao[b], ep, d, flag, ctx->d_err, st));
+            } else {
+                const float *W = reinterpret_cast<const float *>(ctx->ca_o_wt) + (size_t)b * d * d;
+                LAUNCH(XC_K_XATTN, b, 1,
+                       gemm_simt(EPI_RESID_GATE, ep, reinterpret_cast<const float *>(ob), W, d, flag, st));
+            }
+        }
         LAUNCH(XC_K_LN, b, 1, ln_mod<T>(x1, mb + 3 * d, mb + 4 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
         // FFN up: u = GELU_tanh(h2 W1 + b1)
         memset(&ep, 0, sizeof ep);
@@ -690,6 +754,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         sig.eval_mode = eval_pass(ctx, p, t) ? 1 : 0;
         sig.slot = slot;
         sig.n_keys = n_keys;
+        sig.n_ctx = ctx->n_ctx;
         sig.p = p;
         sig.p.replay_skip = nullptr;
         sig.replay = p.replay_skip != nullptr ? 1 : 0;
@@ -774,6 +839,15 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
             set_err(nullptr, "xc_init: NULL weight pointer");
             return XC_EINVAL;
         }
+    if (cfg->d_ctx > 0) {
+        const float *const req_ca[] = {w->ca_ln_w, w->ca_ln_b, w->ca_q_w, w->ca_q_b,
+                                       w->ca_kv_w, w->ca_kv_b, w->ca_o_w, w->ca_o_b};
+        for (const float *p : req_ca)
+            if (p == nullptr) {
+                set_err(nullptr, "xc_init: NULL cross-attention weight pointer");
+                return XC_EINVAL;
+            }
+    }
     ctx = new xc_ctx();
     try {
         ctx->cfg = *cfg;
@@ -844,9 +918,36 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->o_wt = dalloc<void>(ctx, (size_t)B * d * d * es);
         ctx->f1_wt = dalloc<void>(ctx, (size_t)B * F * d * es);
         ctx->f2_wt = dalloc<void>(ctx, (size_t)B * d * F * es);
+        ctx->xattn = cfg->d_ctx > 0;
+        ctx->d_ctx = cfg->d_ctx;
+        ctx->max_ctx = cfg->max_ctx;
+        ctx->n_ctx = 0;
+        if (ctx->xattn) {
+            const size_t Bd = (size_t)B * d;
+            std::vector<float> gm1(Bd);
+            for (size_t i = 0; i < Bd; ++i) gm1[i] = w->ca_ln_w[i] - 1.0f;   // exact for gains in [0.5, 2]
+            up(ctx->ca_shift, w->ca_ln_b, Bd);
+            up(ctx->ca_scale, gm1.data(), Bd);
+            up(ctx->ca_q_b, w->ca_q_b, Bd);
+            up(ctx->ca_kv_b, w->ca_kv_b, 2 * Bd);
+            up(ctx->ca_o_b, w->ca_o_b, Bd);
+            std::vector<float> one((size_t)d, 1.0f);
+            up(ctx->ones, one.data(), d);
+            ctx->ca_q_wt = dalloc<void>(ctx, Bd * d * es);
+            ctx->ca_kv_wt = dalloc<void>(ctx, 2 * Bd * ctx->d_ctx * es);
+            ctx->ca_o_wt = dalloc<void>(ctx, Bd * d * es);
+            const size_t nc = (size_t)ctx->max_ctx * ctx->d_ctx;
+            ctx->ctx_in = dalloc<float>(ctx, nc * sizeof(float));
+            ctx->ctx_act = ctx->bf ? dalloc<void>(ctx, nc * es) : nullptr;
+            ctx->ctx_k = dalloc<void>(ctx, Bd * ctx->max_ctx * es);
+            ctx->ctx_v = dalloc<void>(ctx, Bd * ctx->max_ctx * es);
+            CK(cudaMemset(ctx->ctx_k, 0, Bd * ctx->max_ctx * es));     // rows past n_ctx stay finite
+            CK(cudaMemset(ctx->ctx_v, 0, Bd * ctx->max_ctx * es));
+        }
         {
             size_t mx = (size_t)3 * d * d;
             if ((size_t)d * F > mx) mx = (size_t)d * F;
+            if (ctx->xattn && (size_t)2 * d * ctx->d_ctx > mx) mx = (size_t)2 * d * ctx->d_ctx;
             float *tmp = nullptr;
             CK(cudaMalloc(&tmp, mx * sizeof(float)));
             try {
@@ -854,6 +955,11 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
                 upload_blocks(ctx, ctx->o_wt, w->o_w, d, d, tmp);
                 upload_blocks(ctx, ctx->f1_wt, w->f1_w, d, F, tmp);
                 upload_blocks(ctx, ctx->f2_wt, w->f2_w, F, d, tmp);
+                if (ctx->xattn) {
+                    upload_blocks(ctx, ctx->ca_q_wt, w->ca_q_w, d, d, tmp);
+                    upload_blocks(ctx, ctx->ca_kv_wt, w->ca_kv_w, ctx->d_ctx, 2 * d, tmp);
+                    upload_blocks(ctx, ctx->ca_o_wt, w->ca_o_w, d, d, tmp);
+                }
             } catch (...) {
                 cudaFree(tmp);
                 throw;
@@ -948,6 +1054,23 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
                 const char *rv = reinterpret_cast<const char *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld * es;
                 tmap(ctx, &ctx->tm_rk[b], rk, (uint64_t)ctx->Wkv * L, d, 128);
                 tmap(ctx, &ctx->tm_rv[b], rv, (uint64_t)ctx->Wkv * L, d, 128);
+            }
+            if (ctx->xattn) {
+                const int D = ctx->d_ctx;
+                for (auto *v : {&ctx->tm_caq, &ctx->tm_cao, &ctx->tm_cak, &ctx->tm_cav, &ctx->tm_ck, &ctx->tm_cv})
+                    v->resize(B);
+                for (int b = 0; b < B; ++b) {
+                    const char *wq = reinterpret_cast<const char *>(ctx->ca_q_wt) + (size_t)b * d * d * es;
+                    const char *wo = reinterpret_cast<const char *>(ctx->ca_o_wt) + (size_t)b * d * d * es;
+                    const char *wkv = reinterpret_cast<const char *>(ctx->ca_kv_wt) + (size_t)b * 2 * d * D * es;
+                    tmap(ctx, &ctx->tm_caq[b], wq, d, d, ctx->bn_o);
+                    tmap(ctx, &ctx->tm_cao[b], wo, d, d, ctx->bn_o);
+                    tmap(ctx, &ctx->tm_cak[b], wkv, d, D, 128);                      // rows [0, d): W_k^T
+                    tmap(ctx, &ctx->tm_cav[b], wkv + (size_t)d * D * es, d, D, 128);  // rows [d, 2d): W_v^T
+                    const size_t cb = (size_t)b * ctx->max_ctx * d * es;
+                    tmap(ctx, &ctx->tm_ck[b], reinterpret_cast<const char *>(ctx->ctx_k) + cb, ctx->max_ctx, d, 128);
+                    tmap(ctx, &ctx->tm_cv[b], reinterpret_cast<const char *>(ctx->ctx_v) + cb, ctx->max_ctx, d, 128);
+                }
             }
         }
         ctx->trace = nullptr;
@@ -1097,6 +1220,68 @@ xc_status xc_euler_update(xc_ctx *ctx, float *x, const float *v, float dsigma, l
     return XC_OK;
 }
 
+xc_status xc_set_context(xc_ctx *ctx, const float *context, int n_ctx) {
+    if (ctx == nullptr) {
+        set_err(nullptr, "xc_set_context: NULL context");
+        return XC_ESTATE;
+    }
+    if (!ctx->xattn) {
+        set_err(ctx, "xc_set_context: the model has no cross-attention (d_ctx = 0)");
+        return XC_EINVAL;
+    }
+    if (context == nullptr || n_ctx < 1 || n_ctx > ctx->max_ctx) {
+        set_err(ctx, "xc_set_context: NULL tokens or n_ctx %d out of [1, %d]", n_ctx, ctx->max_ctx);
+        return XC_EINVAL;
+    }
+    const int d = ctx->d, D = ctx->d_ctx, B = ctx->B;
+    const size_t n = (size_t)n_ctx * D;
+    try {
+        cudaStream_t st = ctx->st;
+        if (is_host_ptr(context)) {
+            for (size_t i = 0; i < n; ++i)
+                if (!std::isfinite(context[i])) {
+                    set_err(ctx, "xc_set_context: non-finite condition token value");
+                    return XC_ENUMERIC;
+                }
+            CK(cudaMemcpyAsync(ctx->ctx_in, context, n * sizeof(float), cudaMemcpyHostToDevice, st));
+            CK(cudaStreamSynchronize(st));           // host buffer consumed before returning
+        } else {
+            CK(cudaMemcpyAsync(ctx->ctx_in, context, n * sizeof(float), cudaMemcpyDeviceToDevice, st));
+        }
+        CUtensorMap tm_a;
+        if (ctx->bf) {
+            CK(convert_f32<bf16>(ctx->ctx_in, reinterpret_cast<bf16 *>(ctx->ctx_act), (long)n, ctx->n_sm, st));
+            if (!make_tmap_bf16(&tm_a, ctx->ctx_act, n_ctx, D, 128)) {
+                set_err(ctx, "xc_set_context: tensor map encoding failed");
+                return XC_ECUDA;
+            }
+        }
+        // [K_c | V_c] = C W_kv + b_kv, one GEMM per half and block
+        for (int b = 0; b < B; ++b)
+            for (int half = 0; half < 2; ++half) {
+                EpiParams ep;
+                memset(&ep, 0, sizeof ep);
+                ep.M = n_ctx;
+                ep.N = d;
+                ep.bias = ctx->ca_kv_b + (size_t)b * 2 * d + (size_t)half * d;
+                ep.out = reinterpret_cast<char *>(half ? ctx->ctx_v : ctx->ctx_k) +
+                         (size_t)b * ctx->max_ctx * d * ctx->esz;
+                if (ctx->bf) {
+                    CK(gemm_tc(EPI_BIAS, 128, tm_a, half ? ctx->tm_cav[b] : ctx->tm_cak[b], ep, D, nullptr,
+                               ctx->d_err, st));
+                } else {
+                    const float *W = reinterpret_cast<const float *>(ctx->ca_kv_wt) + ((size_t)b * 2 + half) * d * D;
+                    CK(gemm_simt(EPI_BIAS, ep, ctx->ctx_in, W, D, nullptr, st));
+                }
+                ctx->launches += 1;
+            }
+        ctx->n_ctx = n_ctx;
+    } catch (Fail &f) {
+        return f.st;
+    }
+    return XC_OK;
+}
+
 xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, float sigma, int step_index,
                         int is_kv_update, const xc_gate_params *gate, float *v_out, xc_step_stats *stats) {
     if (ctx == nullptr) {
@@ -1138,6 +1323,10 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
         }
     } else if (step_index != ctx->next_step || step_index >= ctx->S) {
         set_err(ctx, "denoising pass %d out of order (expected %d)", step_index, ctx->next_step);
+        return XC_ESTATE;
+    }
+    if (ctx->xattn && ctx->n_ctx == 0) {
+        set_err(ctx, "cross-attention model without condition tokens: call xc_set_context first");
         return XC_ESTATE;
     }
     const int t = kv ? 0 : step_index;

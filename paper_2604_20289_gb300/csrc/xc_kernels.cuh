@@ -72,6 +72,8 @@ cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, i
 template <typename T>
 cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t *skip, int n_sm, cudaStream_t st);
 cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_t st);
+template <typename T>
+cudaError_t convert_f32(const float *in, T *out, long n, int n_sm, cudaStream_t st);
 // Fused conditioning (three launches), see k_elem.cu.
 constexpr int COND_TEMB_MAX = 512;
 struct CondArgs {

@@ -1,6 +1,7 @@
 """AR rollout driver over the C ABI (Section 2.1 inference loop).
 
-Chunk n: x = eps_n; for t < S: v = xc_chunk_step(x, sigma_t, t); x += (sigma_{t+1}
+Chunk n: (cross-attention models: xc_set_context with the chunk's condition
+tokens) x = eps_n; for t < S: v = xc_chunk_step(x, sigma_t, t); x += (sigma_{t+1}
 - sigma_t) v (Euler step, xc_euler_update); then, on a KV-update chunk (every
 chunk, or n mod P == P - 1 with kv_period P > 0), the KV-update pass on the
 chunk's clean latent at sigma = 0.  Actions are replayed one chunk at a time
@@ -38,6 +39,8 @@ def rollout(xc: XCache, traj, n_chunks: int, gate: GateParams, sigmas=DEFAULT_SI
     finals, stats, traces = [], [], []
     try:
         for n in range(n_start, n_start + n_chunks):
+            if getattr(cfg, "d_ctx", 0) > 0:
+                xc.set_context(traj.context(n))
             x.copy_(torch.from_numpy(np.ascontiguousarray(traj.noise(n), dtype=np.float32)))
             a = traj.action(n)
             st_n, tr_n = [], []

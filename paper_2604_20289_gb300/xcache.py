@@ -39,12 +39,14 @@ class ModelCfg(ctypes.Structure):
                           ("kv_period", ctypes.c_int), ("n_groups", ctypes.c_int),
                           ("group_cams", ctypes.c_int * XC_MAX_GROUPS),
                           ("group_h", ctypes.c_int * XC_MAX_GROUPS),
-                          ("group_w", ctypes.c_int * XC_MAX_GROUPS)]
+                          ("group_w", ctypes.c_int * XC_MAX_GROUPS),
+                          ("d_ctx", ctypes.c_int), ("max_ctx", ctypes.c_int)]
 
 
 WEIGHT_NAMES = ("pe_w", "pe_b", "t_w1", "t_b1", "t_w2", "t_b2", "a_w1", "a_b1", "a_w2", "a_b2",
                 "mod_w", "mod_b", "blk_mod", "qkv_w", "qkv_b", "o_w", "o_b", "f1_w", "f1_b",
-                "f2_w", "f2_b", "head_w", "head_b", "head_tab", "out_w", "out_b")
+                "f2_w", "f2_b", "head_w", "head_b", "head_tab", "out_w", "out_b",
+                "ca_ln_w", "ca_ln_b", "ca_q_w", "ca_q_b", "ca_kv_w", "ca_kv_b", "ca_o_w", "ca_o_b")
 
 
 class Weights(ctypes.Structure):
@@ -75,7 +77,8 @@ class ProfileRec(ctypes.Structure):
                 ("ms", ctypes.c_float)]
 
 
-KERNEL_KINDS = ("cond", "embed", "gate", "ln", "qkv", "attn", "oproj", "ffn1", "ffn2", "reuse", "head")
+KERNEL_KINDS = ("cond", "embed", "gate", "ln", "qkv", "attn", "oproj", "ffn1", "ffn2", "reuse", "head",
+                "xattn")
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -87,6 +90,7 @@ SIGNATURES = {
     "xc_chunk_step": (_I, [_P, _P, _P, _F, _I, _I, ctypes.POINTER(GateParams), _P,
                            ctypes.POINTER(StepStats)]),
     "xc_reset": (_I, [_P]),
+    "xc_set_context": (_I, [_P, _P, _I]),
     "xc_destroy": (None, [_P]),
     "xc_last_error": (ctypes.c_char_p, [_P]),
     "xc_euler_update": (_I, [_P, _P, _P, _F, _L]),
@@ -168,6 +172,8 @@ def model_cfg(cfg) -> ModelCfg:
     m.n_groups = len(groups)
     for i, (c, h, w) in enumerate(groups):
         m.group_cams[i], m.group_h[i], m.group_w[i] = c, h, w
+    m.d_ctx = int(getattr(cfg, "d_ctx", 0))
+    m.max_ctx = int(getattr(cfg, "max_ctx", 0))
     return m
 
 
@@ -193,9 +199,9 @@ class XCache:
     def __init__(self, cfg, weights: dict, stream=None):
         self.cfg = cfg
         self._c_cfg = model_cfg(cfg)
-        keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in WEIGHT_NAMES}
-        w = Weights(*[v.ctypes.data_as(ctypes.POINTER(ctypes.c_float)) for v in
-                      (keep[k] for k in WEIGHT_NAMES)])
+        keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in WEIGHT_NAMES if k in weights}
+        w = Weights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float)) if k in keep else None
+                      for k in WEIGHT_NAMES])
         ctx = ctypes.c_void_p()
         self._stream = _stream(stream)
         check(LIB.xc_init(ctypes.byref(self._c_cfg), ctypes.byref(w), self._stream, ctypes.byref(ctx)))
@@ -231,6 +237,12 @@ class XCache:
 
     def reset(self):
         check(LIB.xc_reset(self.ctx), self.ctx)
+
+    def set_context(self, tokens):
+        """Condition tokens [n_ctx, d_ctx] (torch CUDA tensor or numpy float32)."""
+        if isinstance(tokens, np.ndarray):
+            tokens = np.ascontiguousarray(tokens, dtype=np.float32)
+        check(LIB.xc_set_context(self.ctx, _ptr(tokens), int(tokens.shape[0])), self.ctx)
 
     def euler(self, x, v, dsigma: float):
         check(LIB.xc_euler_update(self.ctx, _ptr(x), _ptr(v), float(dsigma), x.numel()), self.ctx)

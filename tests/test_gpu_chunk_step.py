@@ -313,3 +313,52 @@ def test_kv_period_call_order():
         xc.chunk_step(x, a, 1.0, 0, False, g)
     xc.chunk_step(x, a, 0.0, 0, True, g)
     assert xb.LIB.xc_chunk_index(xc.ctx) == 3
+
+
+# ------------------------------------------------ cross-attention conditioning
+@pytest.mark.parametrize("cfg", [X.XATTN_F32, X.XATTN_BF16], ids=lambda c: c.name)
+def test_cross_attention_rollout_parity(cfg):
+    """Condition tokens whose count changes from chunk to chunk (ragged key
+    tiles on the tensor-core path), cross-attention in every block."""
+    op, gp = params(tau_floor=0.92, tau_dev=10.0)
+    ref = _replay_and_free(cfg, op, gp, cfg.n_chunks, per_block=cfg.dtype == "bf16")
+    dec = decisions(ref["stats"])
+    assert (dec == O.Decision.SKIP).any() and (dec == O.Decision.COMPUTE).any()
+
+
+def test_cross_attention_force_recompute_and_padding():
+    """Force-recompute equals the gate switched off bit for bit; condition
+    rows past n_ctx left over from a longer context change nothing."""
+    cfg = X.XATTN_BF16
+    _, g_off = params(enabled=False)
+    _, g_fc = params(**FORCE_RECOMPUTE)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=3)
+    a = gpu_rollout(xc, traj, 3, g_off)
+    xc.reset()
+    big = X.random_tensor(7, "xattn/garbage", (cfg.max_ctx, cfg.d_ctx), std=30.0).astype(np.float32)
+    xc.set_context(big)                    # every row written, then shortened by the rollout
+    b = gpu_rollout(xc, traj, 3, g_fc)
+    for n in range(3):
+        np.testing.assert_array_equal(a["final"][n], b["final"][n])
+
+
+def test_cross_attention_argument_errors():
+    cfg = X.XATTN_F32.replace(name="xattn_f32_errors")
+    w = X.make_weights(cfg)
+    xc = xb.XCache(cfg, w)
+    x = torch.zeros(cfg.tokens, cfg.c_latent, device="cuda")
+    with pytest.raises(xb.XCacheError, match="xc_set_context"):     # no condition tokens yet
+        xc.chunk_step(x, np.zeros(2), 1.0, 0, False, xb.gate_params())
+    with pytest.raises(xb.XCacheError):
+        xc.set_context(np.zeros((cfg.max_ctx + 1, cfg.d_ctx), np.float32))
+    bad = np.zeros((3, cfg.d_ctx), np.float32)
+    bad[1, 2] = np.nan
+    with pytest.raises(xb.XCacheError):
+        xc.set_context(bad)
+    xc.set_context(np.zeros((3, cfg.d_ctx), np.float32))
+    xc.chunk_step(x, np.zeros(2), 1.0, 0, False, xb.gate_params())
+    xc.close()
+    _, plain = model(X.TINY_F32)
+    with pytest.raises(xb.XCacheError):
+        plain.set_context(np.zeros((3, 32), np.float32))
