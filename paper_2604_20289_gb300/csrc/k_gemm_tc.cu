@@ -260,6 +260,12 @@ __global__ void __launch_bounds__(320, 1)
                 pos2 = tp.z;
                 pos3 = tp.w;
             }
+            // bias (and gate) of this thread's columns, one value per lane,
+            // fetched one 32-column block ahead and broadcast by shuffles
+            const int colw = n0 + half * (BN / 2);
+            float b_next = ep.bias[colw + lane];
+            float g_next = 0.0f;
+            if constexpr (RES) g_next = ep.gate[colw + lane];
             ok = mbar_wait(&acc_full[buf], use & 1, err, ERR_WAIT_EPI);
             __syncwarp();
             if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
@@ -268,6 +274,11 @@ __global__ void __launch_bounds__(320, 1)
             for (int j = 0; j < BN / 64; ++j) {
                 const int c = half * (BN / 2) + 32 * j;
                 const int col = n0 + c;
+                const float b_cur = b_next, g_cur = g_next;
+                if (j + 1 < BN / 64) {
+                    b_next = ep.bias[col + 32 + lane];
+                    if constexpr (RES) g_next = ep.gate[col + 32 + lane];
+                }
                 float v[32];
                 {
                     float t[16];
@@ -284,12 +295,7 @@ __global__ void __launch_bounds__(320, 1)
                     mbar_arrive(&acc_empty[buf]);
                 }
 #pragma unroll
-                for (int i = 0; i < 32; i += 8) {
-                    float bb[8];
-                    loadW<float, 8>(ep.bias + col + i, bb);
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) v[i + k] += bb[k];
-                }
+                for (int i = 0; i < 32; ++i) v[i] += __shfl_sync(0xffffffffu, b_cur, i);
                 float xi[32];
                 if constexpr (RES) {
                     ok = mbar_wait(lb, (n_ld - 1) & 1, err, ERR_WAIT_EPI);
@@ -300,12 +306,7 @@ __global__ void __launch_bounds__(320, 1)
                     if constexpr (CACHE)
                         if (has_rhat) read_row32(s_xin, lane, xi);
 #pragma unroll
-                    for (int i = 0; i < 32; i += 8) {
-                        float g[8];
-                        loadW<float, 8>(ep.gate + col + i, g);
-#pragma unroll
-                        for (int k = 0; k < 8; ++k) v[i + k] = r[i + k] + g[k] * v[i + k];
-                    }
+                    for (int i = 0; i < 32; ++i) v[i] = r[i] + __shfl_sync(0xffffffffu, g_cur, i) * v[i];
                     __syncwarp();                      // every lane has read the block
                     if (j + 1 < BN / 64) load_res(m0, col + 32);
                 }
