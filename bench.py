@@ -79,6 +79,24 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The largest per-rank value over all ranks (the slowest replica's
+    time); one all-reduce of one scalar, no data-path collective."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, seconds: float) -> float:
+    """Weak scaling: the units all replicas processed over the slowest
+    replica's time."""
+    return units_per_rank * world / seconds
+
+
 class ClockSampler:
     """nvidia-smi clocks / throttle reasons sampled every 200 ms."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -314,11 +332,7 @@ def main():
         per_chunk = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
         launches = xc.launch_count - l0
         recs = xc.profile_stop() if profile else []
-        if world > 1:
-            import torch.distributed as dist
-            t = torch.tensor([ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = max_over_ranks(ms, world, dev)
         return ms, launches, recs, per_chunk
 
     gate = xb.gate_params(tau_floor=args.tau_floor, tau_dev=args.tau_dev)
@@ -360,7 +374,7 @@ def main():
                 "launches": len(work)}
 
     n_chunks = args.steps * world
-    value = n_chunks / (ms_x * 1e-3)
+    value = whole_job_rate(args.steps, world, ms_x * 1e-3)
     line = {"metric": METRIC, "value": value, "unit": "chunks/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_x / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
@@ -555,18 +569,13 @@ def e2e(xc, traj, acts, cfg, args, gate, world, dev):
     for n in range(args.warmup, args.warmup + args.steps):
         chunk(n)
     torch.cuda.synchronize()
-    sec = time.perf_counter() - t0
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([sec], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        sec = float(t.item())
+    sec = max_over_ranks(time.perf_counter() - t0, world, dev)
     nbytes = L * C * 4
     kv = sum(has_kv_pass(cfg, n) for n in range(args.warmup, args.warmup + args.steps)) / args.steps
     ctx_b = 0.0
     if cfg.d_ctx:
         ctx_b = sum(traj.context(n).nbytes for n in range(args.warmup, args.warmup + args.steps)) / args.steps
-    return {"value": args.steps * world / sec, "unit": "chunks/s",
+    return {"value": whole_job_rate(args.steps, world, sec), "unit": "chunks/s",
             "h2d_bytes_per_step": (S + kv) * (nbytes + cfg.action_dim * 4) + ctx_b,
             "d2h_bytes_per_step": S * nbytes}
 
