@@ -161,21 +161,27 @@ __global__ void __launch_bounds__(256)
     for (; row < M; row += nw) {
         const int nrow = row + nw;
         if (nrow < M && act) load16<T>(x + (size_t)nrow * d + 16 * lane, nxt);
-        Moments mo{0.0f, 0.0f, 0.0f};
+        // two passes over the register-resident row: the mean, then the
+        // squared deviations from it (butterfly sums, no Welford merges)
+        float sum = 0.0f;
         if (act) {
-            float sum = 0.0f;
 #pragma unroll
             for (int i = 0; i < 16; ++i) sum += cur[i];
-            mo.n = 16.0f;
-            mo.mean = sum * (1.0f / 16.0f);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) mo.m2 += (cur[i] - mo.mean) * (cur[i] - mo.mean);
         }
-        mo = warp_moments(mo);
-        const float rstd = rsqrtf(mo.m2 / (float)d + eps);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        const float mean = sum / (float)d;
+        float m2 = 0.0f;
         if (act) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) cur[i] = (cur[i] - mo.mean) * rstd * (1.0f + sc[i]) + sh[i];
+            for (int i = 0; i < 16; ++i) m2 = fmaf(cur[i] - mean, cur[i] - mean, m2);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m2 += __shfl_xor_sync(0xffffffffu, m2, o);
+        const float rstd = rsqrtf(m2 / (float)d + eps);
+        if (act) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) cur[i] = (cur[i] - mean) * rstd * (1.0f + sc[i]) + sh[i];
             store16<T>(out + (size_t)row * d + 16 * lane, cur);
         }
 #pragma unroll
