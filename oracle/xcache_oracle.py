@@ -383,11 +383,14 @@ class OracleModel:
         return R(x1 + (o @ w["ca_o_w"][b] + w["ca_o_b"][b]))
 
     def block(self, b: int, x_in: np.ndarray, mod: np.ndarray, past_k: list, past_v: list,
-              pos: np.ndarray, ctx_kv=None):
+              pos: np.ndarray, ctx_kv=None, rows=None):
         """x_{t,b} = x_{t,b-1} + f_b(x_{t,b-1}; c_t) (Eq. 1).  Returns the block
         output and this pass's (k, v) of the current chunk [L, H, hd].  With
         ``ctx_kv`` (this block's condition keys / values) the cross-attention
-        layer sits between the self-attention and the FFN."""
+        layer sits between the self-attention and the FFN.  With ``rows``
+        (token indices) only those rows of the output are computed and
+        returned (keys and values still come from every token): every step
+        after the K/V projection acts on one token row at a time."""
         cfg, w, R = self.cfg, self.w, self.R
         L, d, H, hd = x_in.shape[0], cfg.d_model, cfg.n_heads, cfg.head_dim
         sh1, sc1, g1, sh2, sc2, g2 = mod
@@ -399,6 +402,9 @@ class OracleModel:
         q = R(apply_rope(q, pos, cfg.rope_theta))
         k = R(apply_rope(k, pos, cfg.rope_theta))
         v = R(v)
+        if rows is not None:
+            rows = np.asarray(rows)
+            q, x_in, L = q[rows], x_in[rows], len(rows)
         keys = np.concatenate(past_k + [k], axis=0)
         vals = np.concatenate(past_v + [v], axis=0)
         o = R(attention(q, keys, vals).reshape(L, d))

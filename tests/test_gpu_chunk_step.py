@@ -362,3 +362,41 @@ def test_cross_attention_argument_errors():
     _, plain = model(X.TINY_F32)
     with pytest.raises(xb.XCacheError):
         plain.set_context(np.zeros((3, 32), np.float32))
+
+
+# ------------------------------------------- full size, benchmark configuration
+def test_full_size_first_block_sampled_rows():
+    """The benchmark model at full size in the benchmark's launch
+    configuration (persistent GEMMs, attention split over the SMs with partial
+    merges, CUDA-graph replay of the pass): block 0 of the first pass of
+    chunk 0 on sampled token rows -- the first and last rows, tile edges and a
+    seeded random sample -- against the oracle (keys and values from every
+    token)."""
+    cfg = X.SMALL_BF16
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=1)
+    L, d = cfg.tokens, cfg.d_model
+    tr = torch.empty(cfg.n_blocks, L, d, device="cuda", dtype=torch.bfloat16)
+    x = torch.tensor(traj.noise(0), dtype=torch.float32, device="cuda")
+    v = torch.empty_like(x)
+    g = xb.gate_params()
+    xc.set_trace(tr)
+    try:
+        for _ in range(2):                 # the second run replays the pass's graph
+            xc.reset()
+            xc.chunk_step(x, traj.action(0), 1.0, 0, False, g, v_out=v)
+        xc.sync()
+    finally:
+        xc.set_trace(None)
+    got = tr[0].float().cpu().numpy()
+    M = O.OracleModel(cfg, w)
+    mods, _ = M.cond(1.0, traj.action(0))
+    x0 = M.patch_embed(traj.noise(0))
+    pos = O.group_token_positions(cfg.groups, cfg.frames, 0)
+    rng_rows = np.random.default_rng(5)
+    rows = np.unique(np.r_[0, 1, 127, 128, 255, 256, L // 2, L - 129, L - 128, L - 1,
+                           rng_rows.choice(L, 22, replace=False)])
+    want, _, _ = M.block(0, x0, mods[0], [], [], pos, rows=rows)
+    for i, r in enumerate(rows):
+        assert rel_l2(got[r], want[i]) <= 1e-2, (r, rel_l2(got[r], want[i]))
+    assert rel_l2(got[rows], want) <= 5e-3

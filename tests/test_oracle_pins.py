@@ -626,3 +626,20 @@ def test_cross_attention_with_zero_output_is_plain_block():
     a, _, _ = m.block(0, x, mods[0], [], [], pos, m.context_kv(0, ctx))
     b, _, _ = m.block(0, x, mods[0], [], [], pos)
     np.testing.assert_array_equal(a, b)
+
+
+def test_block_rows_subset_equals_full_block():
+    """A block evaluated on sampled rows gives those rows of the full block."""
+    for cfg in (X.TINY_F32, X.XATTN_F32):
+        m = O.OracleModel(cfg, X.make_weights(cfg))
+        x = rng.standard_normal((cfg.tokens, cfg.d_model))
+        mods, _ = m.cond(0.75, np.array([0.2, -0.1]))
+        pos = O.token_positions(cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, 1)
+        past_k = [rng.standard_normal((cfg.tokens, cfg.n_heads, cfg.head_dim))]
+        past_v = [rng.standard_normal((cfg.tokens, cfg.n_heads, cfg.head_dim))]
+        ctx = m.context_kv(1, rng.standard_normal((5, cfg.d_ctx))) if cfg.d_ctx else None
+        full, k, v = m.block(1, x, mods[1], past_k, past_v, pos, ctx)
+        rows = np.array([0, 7, 33, cfg.tokens - 1])
+        sub, k2, v2 = m.block(1, x, mods[1], past_k, past_v, pos, ctx, rows=rows)
+        np.testing.assert_allclose(sub, full[rows], rtol=1e-12, atol=1e-12)
+        np.testing.assert_array_equal(k2, k)
