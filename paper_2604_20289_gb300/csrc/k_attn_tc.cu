@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(352, 1)
                    const __grid_constant__ CUtensorMap tmV, bf16 *__restrict__ o, const int Lq,
                    const int n_keys, const int d, const AttnSplit sp, float *__restrict__ ws_o,
                    float2 *__restrict__ ws_ml, const uint8_t *__restrict__ skip_flag, int *err) {
+    pdl_wait();
     using A = AttnTile<HD>;
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     extern __shared__ uint8_t smem_raw[];
@@ -486,6 +487,7 @@ __global__ void __launch_bounds__(256)
     attn_combine_kernel(bf16 *__restrict__ o, const int Lq, const int d, const AttnSplit sp,
                         const float *__restrict__ ws_o, const float2 *__restrict__ ws_ml,
                         const uint8_t *__restrict__ skip_flag) {
+    pdl_wait();
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     const int b = blockIdx.x + 1;                      // boundary between CTAs b-1 and b
     const long long it = sp.begin(b);
@@ -551,14 +553,13 @@ static cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, con
     sp.G = split ? n_sm : n_units;
     float *ws_o = split ? reinterpret_cast<float *>(ws) : nullptr;
     float2 *ws_ml = split ? reinterpret_cast<float2 *>(ws_o + 2 * ((size_t)n_sm + 1) * 256 * HD) : nullptr;
-    attn_tc_kernel<HD><<<sp.G, A::THREADS, A::SMEM_BYTES, st>>>(tq, tk, tv, o, Lq, n_keys, d, sp, ws_o, ws_ml, skip,
-                                                                 err);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(attn_tc_kernel<HD>, dim3(sp.G), dim3(A::THREADS), A::SMEM_BYTES, st, tq, tk, tv, o,
+                               Lq, n_keys, d, sp, ws_o, ws_ml, skip, err);
     if (e != cudaSuccess) return e;
     if (n_launched) *n_launched = 1;
     if (split && sp.G > 1) {
-        attn_combine_kernel<HD><<<sp.G - 1, 256, 0, st>>>(o, Lq, d, sp, ws_o, ws_ml, skip);
-        e = cudaGetLastError();
+        e = launch_pdl(attn_combine_kernel<HD>, dim3(sp.G - 1), dim3(256), 0, st, o, Lq, d, sp,
+                       static_cast<const float *>(ws_o), static_cast<const float2 *>(ws_ml), skip);
         if (n_launched) *n_launched = 2;
     }
     return e;

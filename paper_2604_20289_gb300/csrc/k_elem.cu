@@ -14,6 +14,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
     patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w, const float *__restrict__ b,
                        T *__restrict__ out, int L, int d) {
+    pdl_wait();
+    pdl_release();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int run = blockIdx.y * 8 + warp;
     const int row = blockIdx.x * 32 + lane;
@@ -37,8 +39,7 @@ template <typename T>
 cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st) {
     if (C != 16 || d % 16 != 0) return cudaErrorInvalidValue;
     const dim3 grid((L + 31) / 32, (d / 16 + 7) / 8);
-    patch_embed_kernel<T><<<grid, 256, 0, st>>>(z, w, b, out, L, d);
-    return cudaGetLastError();
+    return launch_pdl(patch_embed_kernel<T>, grid, dim3(256), 0, st, z, w, b, out, L, d);
 }
 template cudaError_t patch_embed<float>(const float *, const float *, const float *, float *, int, int, int, cudaStream_t);
 template cudaError_t patch_embed<bf16>(const float *, const float *, const float *, bf16 *, int, int, int, cudaStream_t);
@@ -104,6 +105,8 @@ template <typename T, int NCH>
 __global__ void __launch_bounds__(256)
     ln_mod_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
                   T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
+    pdl_wait();
+    pdl_release();
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
@@ -147,6 +150,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
     ln_mod_row_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
                       T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
+    pdl_wait();
+    pdl_release();
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     const int lane = threadIdx.x & 31;
     const int nw = (gridDim.x * blockDim.x) >> 5;
@@ -202,8 +207,7 @@ static int n_sm_elem() {
 template <typename T, int NCH>
 static cudaError_t ln_mod_n(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
                             const uint8_t *skip, cudaStream_t st) {
-    ln_mod_kernel<T, NCH><<<(M + 7) / 8, 256, 0, st>>>(x, shift, scale, out, M, d, eps, skip);
-    return cudaGetLastError();
+    return launch_pdl(ln_mod_kernel<T, NCH>, dim3((M + 7) / 8), dim3(256), 0, st, x, shift, scale, out, M, d, eps, skip);
 }
 
 template <typename T>
@@ -212,8 +216,7 @@ cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, i
     if (d % 16 != 0) return cudaErrorInvalidValue;
     if (d <= 512) {
         const int want = (M + 7) / 8, cap = 2 * n_sm_elem();
-        ln_mod_row_kernel<T><<<want < cap ? want : cap, 256, 0, st>>>(x, shift, scale, out, M, d, eps, skip);
-        return cudaGetLastError();
+        return launch_pdl(ln_mod_row_kernel<T>, dim3(want < cap ? want : cap), dim3(256), 0, st, x, shift, scale, out, M, d, eps, skip);
     }
     switch ((d + 511) / 512) {
         case 1: return ln_mod_n<T, 1>(x, shift, scale, out, M, d, eps, skip, st);
@@ -237,6 +240,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
     reuse_kernel(const T *__restrict__ x, const T *__restrict__ r, T *__restrict__ out, long n16,
                  const uint8_t *__restrict__ skip_flag) {
+    pdl_wait();
+    pdl_release();
     if (skip_flag != nullptr && *skip_flag != XC_DEC_SKIP) return;
     const long stride = (long)gridDim.x * blockDim.x;
     for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n16; i += stride) {
@@ -256,20 +261,20 @@ cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t
     const long cap = (long)n_sm * 8;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    reuse_kernel<T><<<(unsigned)blocks, 256, 0, st>>>(x, r, out, n16, skip);
-    return cudaGetLastError();
+    return launch_pdl(reuse_kernel<T>, dim3((unsigned)blocks), dim3(256), 0, st, x, r, out, n16, skip);
 }
 template cudaError_t residual_reuse<float>(const float *, const float *, float *, long, const uint8_t *, int, cudaStream_t);
 template cudaError_t residual_reuse<bf16>(const bf16 *, const bf16 *, bf16 *, long, const uint8_t *, int, cudaStream_t);
 
 // -------------------------------------------------------------- Euler step
 __global__ void euler_kernel(float *__restrict__ x, const float *__restrict__ v, float ds, long n) {
+    pdl_wait();
+    pdl_release();
     const long i = blockIdx.x * (long)blockDim.x + threadIdx.x;
     if (i < n) x[i] = fmaf(ds, v[i], x[i]);
 }
 cudaError_t euler_update(float *x, const float *v, float ds, long n, cudaStream_t st) {
-    euler_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(x, v, ds, n);
-    return cudaGetLastError();
+    return launch_pdl(euler_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, x, v, ds, n);
 }
 
 // ----------------------------------------------------------- conditioning
@@ -304,6 +309,8 @@ __device__ __forceinline__ float gemv_col(const float *xs, const float *__restri
 
 template <int STAGE>
 __global__ void __launch_bounds__(GEMV_WARPS * 32) cond_kernel(const CondArgs c) {
+    pdl_wait();
+    pdl_release();
     extern __shared__ float xs[];
     __shared__ float part[GEMV_WARPS][33];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -379,14 +386,12 @@ cudaError_t conditioning(const CondArgs &c, cudaStream_t st) {
     if (c.A < 1 || c.A > 8 || c.tf < 2 || c.tf > COND_TEMB_MAX || (size_t)2 * d * sizeof(float) > 48 * 1024)
         return cudaErrorInvalidValue;
     const int in1 = c.tf > c.A ? c.tf : c.A;
-    cond_kernel<1><<<2 * nb_d, GEMV_WARPS * 32, in1 * sizeof(float), st>>>(c);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(cond_kernel<1>, dim3(2 * nb_d), dim3(GEMV_WARPS * 32), in1 * sizeof(float), st, c);
     if (e != cudaSuccess) return e;
-    cond_kernel<2><<<nb_d, GEMV_WARPS * 32, 2 * d * sizeof(float), st>>>(c);
-    e = cudaGetLastError();
+    e = launch_pdl(cond_kernel<2>, dim3(nb_d), dim3(GEMV_WARPS * 32), 2 * d * sizeof(float), st, c);
     if (e != cudaSuccess) return e;
-    cond_kernel<3><<<(6 * d + 31) / 32 + (2 * d + 31) / 32, GEMV_WARPS * 32, d * sizeof(float), st>>>(c);
-    return cudaGetLastError();
+    return launch_pdl(cond_kernel<3>, dim3((6 * d + 31) / 32 + (2 * d + 31) / 32), dim3(GEMV_WARPS * 32),
+                      d * sizeof(float), st, c);
 }
 
 // RoPE (cos, sin) table of one chunk, double precision.  Axes (camera, frame,
@@ -395,6 +400,8 @@ cudaError_t conditioning(const CondArgs &c, cudaStream_t st) {
 // positions (frame: the chunk's frames, absolute frame = frame0 + p); entry
 // base_a + j * npos[a] + p holds (cos, sin)(pos * freq).
 __global__ void rope_table_kernel(int hd, double theta, int frame0, int4 npos, float2 *__restrict__ out, int n) {
+    pdl_wait();
+    pdl_release();
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= n) return;
     const int pairs[4] = {hd / 16, 3 * hd / 16, hd / 8, hd / 8};
@@ -415,8 +422,7 @@ __global__ void rope_table_kernel(int hd, double theta, int frame0, int4 npos, f
     }
 }
 cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out, int n, cudaStream_t st) {
-    rope_table_kernel<<<(n + 127) / 128, 128, 0, st>>>(hd, theta, frame0, npos, out, n);
-    return cudaGetLastError();
+    return launch_pdl(rope_table_kernel, dim3((n + 127) / 128), dim3(128), 0, st, hd, theta, frame0, npos, out, n);
 }
 
 // ------------------------------------------------------------------- head
@@ -434,6 +440,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
     head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
                 const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
+    pdl_wait();
+    pdl_release();
     __shared__ float hs[HEAD_ROWS * (HEAD_CH + 1)];
     __shared__ float2 stats[HEAD_ROWS];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -522,8 +530,7 @@ template <typename T>
 cudaError_t head(const T *x, const float *hm, const float *w, const float *b, float *v, int L, int d, float eps,
                  cudaStream_t st) {
     if (d % 16 != 0) return cudaErrorInvalidValue;
-    head_kernel<T><<<(L + HEAD_ROWS - 1) / HEAD_ROWS, 256, 0, st>>>(x, hm, w, b, v, L, d, eps);
-    return cudaGetLastError();
+    return launch_pdl(head_kernel<T>, dim3((L + HEAD_ROWS - 1) / HEAD_ROWS), dim3(256), 0, st, x, hm, w, b, v, L, d, eps);
 }
 template cudaError_t head<float>(const float *, const float *, const float *, const float *, float *, int, int, float,
                                  cudaStream_t);
@@ -535,6 +542,8 @@ template cudaError_t head<bf16>(const bf16 *, const float *, const float *, cons
 // fp32 -> storage type, elementwise (condition tokens of the cross-attention).
 template <typename T>
 __global__ void __launch_bounds__(256) convert_f32_kernel(const float *__restrict__ in, T *__restrict__ out, long n) {
+    pdl_wait();
+    pdl_release();
     for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
         if constexpr (sizeof(T) == 2)
             out[i] = __float2bfloat16_rn(in[i]);

@@ -64,6 +64,8 @@ __device__ __forceinline__ void add_vec16(float *acc, const uint4 u) {
 
 template <typename T>
 __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
+    pdl_wait();
+    pdl_release();
     constexpr int VEC = 16 / sizeof(T);
     constexpr int TPR = GATE_CW / VEC;          // threads per row
     constexpr int RPAR = GATE_THREADS / TPR;    // rows per sweep
@@ -268,8 +270,7 @@ size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off) {
 
 template <typename T>
 cudaError_t gate_launch(const GateArgs &g, cudaStream_t st) {
-    gate_kernel<T><<<g.V * g.n_slices, GATE_THREADS, 0, st>>>(g);
-    return cudaGetLastError();
+    return launch_pdl(gate_kernel<T>, dim3(g.V * g.n_slices), dim3(GATE_THREADS), 0, st, g);
 }
 template cudaError_t gate_launch<float>(const GateArgs &, cudaStream_t);
 template cudaError_t gate_launch<bf16>(const GateArgs &, cudaStream_t);

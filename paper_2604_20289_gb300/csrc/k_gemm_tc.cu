@@ -121,6 +121,7 @@ __global__ void __launch_bounds__(320, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ EpiMaps em, const EpiParams ep, const int K,
                    const uint8_t *__restrict__ skip_flag, int *err) {
+    pdl_wait();
     using G = GemmTile<BN, EPI>;
     if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
     extern __shared__ uint8_t smem_raw[];
@@ -506,8 +507,7 @@ static cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tb, const
     const int n_sm = gemm_sm_count();
     const int n_tiles = (ep.N / BN) * ((ep.M + GEMM_BM - 1) / GEMM_BM);
     const int grid = n_tiles < n_sm ? n_tiles : n_sm;
-    kern<<<grid, 320, G::SMEM_BYTES, st>>>(ta, tb, em, ep, K, skip, err);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(grid), dim3(320), G::SMEM_BYTES, st, ta, tb, em, ep, K, skip, err);
 }
 
 template <int BN>

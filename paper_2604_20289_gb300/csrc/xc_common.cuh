@@ -9,6 +9,32 @@
 
 namespace xc {
 
+// Programmatic dependent launch.  Kernels of the chunk step are launched with
+// programmatic stream serialisation: a kernel may be scheduled while its
+// predecessor is still running, and pdl_wait() -- the first statement of each
+// such kernel -- blocks until the predecessor has completed and its memory
+// is visible (so everything earlier in the stream is complete as well).
+// pdl_release() then lets the successor be scheduled.  Without the launch
+// attribute both are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_release() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 typedef __nv_bfloat16 bf16;
 
 // Device error word bits (bounded waits that expired, bad launch state).
