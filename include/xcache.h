@@ -190,7 +190,10 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
  *           k mod kv_window_chunks (k = KV-update passes so far; k = n when
  *           kv_period = 0), and the chunk counter advances.
  *   gate    NULL = Table 1 defaults.
- *   v_out   host or device float32 [L][c_latent] velocity, or NULL.
+ *   v_out   host or device float32 [L][c_latent] velocity, or NULL.  A
+ *           KV-update pass with v_out NULL (and no block trace set) computes
+ *           only what the ring needs: the last block stops after its K/V
+ *           projection and the output head is not run.
  *   stats   NULL or filled as documented above (synchronising).
  * Execution: the conditioning and the chunk's RoPE table are launched
  * directly; the rest of the pass (patch embedding, every block, the head)

@@ -114,7 +114,7 @@ bool is_host_ptr(const void *p) {
 // Everything the per-pass block loop takes from the host (besides buffers
 // that stay fixed for the context's lifetime).
 struct PassSig {
-    int t, kv, eval_mode, slot, n_keys, replay, n_ctx;
+    int t, kv, eval_mode, slot, n_keys, replay, n_ctx, want_v;
     uint64_t replay_bits;
     xc_gate_params p;                 // replay_skip pointer cleared
     const void *lat, *v, *trace;
@@ -495,7 +495,7 @@ void run_graph(xc_ctx *ctx, const PassSig &sig, F &&body) {
 
 template <typename T>
 void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigma, int t, bool kv,
-              const xc_gate_params &p, float *v_dev) {
+              const xc_gate_params &p, float *v_dev, bool want_v) {
     const int L = ctx->L, d = ctx->d, F = ctx->F, B = ctx->B, hd = ctx->hd;
     cudaStream_t st = ctx->st;
     const size_t Ld = (size_t)L * d;
@@ -544,6 +544,10 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     auto body = [&](cudaStream_t st) {
 
     T *X[2] = {reinterpret_cast<T *>(ctx->xb[0]), reinterpret_cast<T *>(ctx->xb[1])};
+    // A KV-update pass whose velocity nobody reads (and with no block trace)
+    // only needs every block's K/V: the last block stops after its K/V
+    // projection and the head is not run.
+    const bool kv_tail_off = kv && !want_v && ctx->trace == nullptr;
     LAUNCH(XC_K_EMBED, -1, 1, patch_embed<T>(lat_dev, ctx->pe_w, ctx->pe_b, X[0], L, ctx->C, d, st));
     CK(cudaMemsetAsync(ctx->flags, 0, B, st));
     CK(cudaMemsetAsync(ctx->s_cos, 0xFF, 3 * B * sizeof(float), st));   // NaN
@@ -636,13 +640,17 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         ep.rope_cs = ctx->rope_cs;
         if constexpr (sizeof(T) == 2) {
             LAUNCH(XC_K_QKV, b, 1, gemm_tc(EPI_QKV_ROPE, ctx->bn_qkv, ctx->tm_h, ctx->tm_wqkv[b], ep, d, flag, ctx->d_err, st));
+        } else {
+            const float *W = reinterpret_cast<const float *>(ctx->qkv_wt) + (size_t)b * 3 * d * d;
+            LAUNCH(XC_K_QKV, b, 1, gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
+        }
+        if (kv_tail_off && b == B - 1) break;       // the ring has this block's K/V
+        if constexpr (sizeof(T) == 2) {
             int n_attn = 1;
             LAUNCH(XC_K_ATTN, b, n_attn,
                    attn_tc(hd, ctx->tm_q, ctx->tm_rk[b], ctx->tm_rv[b], reinterpret_cast<bf16 *>(ob), L, n_keys,
                            ctx->H, d, ctx->attn_ws, ctx->attn_ws_bytes, flag, ctx->d_err, &n_attn, st));
         } else {
-            const float *W = reinterpret_cast<const float *>(ctx->qkv_wt) + (size_t)b * 3 * d * d;
-            LAUNCH(XC_K_QKV, b, 1, gemm_simt(EPI_QKV_ROPE, ep, reinterpret_cast<const float *>(hb), W, d, flag, st));
             const float *Kr = reinterpret_cast<const float *>(ctx->ring_k) + (size_t)b * ctx->Wkv * Ld;
             const float *Vr = reinterpret_cast<const float *>(ctx->ring_v) + (size_t)b * ctx->Wkv * Ld;
             LAUNCH(XC_K_ATTN, b, 1, attn_simt(hd, reinterpret_cast<const float *>(qb), Kr, Vr, reinterpret_cast<float *>(ob), L, n_keys,
@@ -741,7 +749,8 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             CK(cudaMemcpyAsync(reinterpret_cast<char *>(ctx->trace) + (size_t)b * Ld * sizeof(T), xout,
                                Ld * sizeof(T), cudaMemcpyDeviceToDevice, st));
     }
-    LAUNCH(XC_K_HEAD, -1, 1, head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
+    if (!kv_tail_off)
+        LAUNCH(XC_K_HEAD, -1, 1, head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
     };   // body
 
     if (ctx->prof_on || !ctx->graphs_on) {
@@ -755,6 +764,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
         sig.slot = slot;
         sig.n_keys = n_keys;
         sig.n_ctx = ctx->n_ctx;
+        sig.want_v = want_v ? 1 : 0;
         sig.p = p;
         sig.p.replay_skip = nullptr;
         sig.replay = p.replay_skip != nullptr ? 1 : 0;
@@ -1341,9 +1351,9 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
         const bool v_host = v_out != nullptr && is_host_ptr(v_out);
         float *v_dev = (v_out == nullptr || v_host) ? ctx->vout : v_out;
         if (ctx->bf)
-            run_pass<bf16>(ctx, lat_dev, action, sigma, t, kv, p, v_dev);
+            run_pass<bf16>(ctx, lat_dev, action, sigma, t, kv, p, v_dev, v_out != nullptr);
         else
-            run_pass<float>(ctx, lat_dev, action, sigma, t, kv, p, v_dev);
+            run_pass<float>(ctx, lat_dev, action, sigma, t, kv, p, v_dev, v_out != nullptr);
         if (v_host) CK(cudaMemcpyAsync(v_out, ctx->vout, lat_bytes, cudaMemcpyDeviceToHost, ctx->st));
         // Host buffers are consumed / produced synchronously: the caller may
         // reuse them as soon as the call returns.

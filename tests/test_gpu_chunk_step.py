@@ -400,3 +400,32 @@ def test_full_size_first_block_sampled_rows():
     for i, r in enumerate(rows):
         assert rel_l2(got[r], want[i]) <= 1e-2, (r, rel_l2(got[r], want[i]))
     assert rel_l2(got[rows], want) <= 5e-3
+
+
+@pytest.mark.parametrize("cfg", [X.TINY_F32, X.MID_HD64], ids=lambda c: c.name)
+def test_kv_pass_without_velocity_writes_the_same_ring(cfg):
+    """A KV-update pass with v_out NULL skips the last block's attention / FFN
+    and the head; later chunks see the same ring bit for bit."""
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=3)
+    _, g = params(tau_floor=0.92, tau_dev=10.0)
+    S = cfg.n_steps
+    finals = []
+    for want_v in (False, True):
+        xc.reset()
+        x = torch.empty(cfg.tokens, cfg.c_latent, device="cuda")
+        v = torch.empty_like(x)
+        vk = torch.empty_like(x)
+        out = []
+        for n in range(3):
+            x.copy_(torch.from_numpy(traj.noise(n)))
+            for t in range(S):
+                xc.chunk_step(x, traj.action(n), O.SIGMAS[t], t, False, g, v_out=v, want_stats=False)
+                xc.euler(x, v, O.SIGMAS[t + 1] - O.SIGMAS[t])
+            clean = torch.from_numpy(traj.clean(n)).cuda()
+            xc.chunk_step(clean, traj.action(n), 0.0, S, True, g, v_out=vk if want_v else None,
+                          want_stats=False)
+            out.append(x.cpu().numpy())
+        finals.append(out)
+    for a, b in zip(*finals):
+        np.testing.assert_array_equal(a, b)
