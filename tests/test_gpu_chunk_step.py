@@ -316,7 +316,7 @@ def test_kv_period_call_order():
 
 
 # ------------------------------------------------ cross-attention conditioning
-@pytest.mark.parametrize("cfg", [X.XATTN_F32, X.XATTN_BF16], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", [X.XATTN_F32, X.XATTN_BF16, X.XATTN_HD128], ids=lambda c: c.name)
 def test_cross_attention_rollout_parity(cfg):
     """Condition tokens whose count changes from chunk to chunk (ragged key
     tiles on the tensor-core path), cross-attention in every block."""

@@ -179,9 +179,11 @@ GROUPS_BF16 = ModelCfg("groups_bf16_2blk_d256_7cam", 2, 256, 4, 64, 1024, 7, 3, 
 # max_ctx per chunk (count varying from chunk to chunk).
 XATTN_F32 = TINY_F32.replace(name="xattn_f32_2blk_d64", d_ctx=32, max_ctx=24)
 XATTN_BF16 = MID_HD64.replace(name="xattn_bf16_3blk_d256_hd64", d_ctx=128, max_ctx=300)
+XATTN_HD128 = MID_HD128.replace(name="xattn_bf16_2blk_d256_hd128", d_ctx=256, max_ctx=160)
 
 ALL_CFGS = {c.name: c for c in (TINY_F32, SMALL_BF16, DIT_1P3B, DIT_14B, STRESS_1P3B,
-                                  MID_HD64, MID_HD128, GROUPS_F32, GROUPS_BF16, XATTN_F32, XATTN_BF16)}
+                                  MID_HD64, MID_HD128, GROUPS_F32, GROUPS_BF16, XATTN_F32, XATTN_BF16,
+                                  XATTN_HD128)}
 
 
 # --------------------------------------------------------------------------
