@@ -429,3 +429,33 @@ def test_kv_pass_without_velocity_writes_the_same_ring(cfg):
         finals.append(out)
     for a, b in zip(*finals):
         np.testing.assert_array_equal(a, b)
+
+
+def test_graph_cache_eviction_keeps_results():
+    """More distinct pass signatures than the graph cache holds (every pass
+    with its own gate knobs): results equal those of directly launched
+    passes (profiling mode launches without graphs)."""
+    cfg = X.TINY_F32
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=1)
+    x0 = torch.tensor(traj.noise(0), dtype=torch.float32, device="cuda")
+    S = cfg.n_steps
+    outs = []
+    for direct in (True, False):
+        xc.reset()
+        if direct:
+            xc.profile_start(kinds=("ln",), capacity=1 << 16)
+        v = torch.empty_like(x0)
+        got = []
+        for i in range(150):                     # one chunk's worth of passes, repeated
+            t = i % S
+            if i and t == 0:
+                xc.chunk_step(x0, traj.action(0), 0.0, S, True, xb.gate_params(), want_stats=False)
+            g = xb.gate_params(tau_floor=float(np.float32(0.5 + 0.003 * i)), tau_dev=10.0)
+            xc.chunk_step(x0, traj.action(0), O.SIGMAS[t], t, False, g, v_out=v, want_stats=False)
+            got.append(v.cpu().numpy().copy())
+        if direct:
+            xc.profile_stop()
+        outs.append(got)
+    for a, b in zip(*outs):
+        np.testing.assert_array_equal(a, b)
