@@ -35,11 +35,20 @@ constexpr int GEMM_BK = 64;
 constexpr int GEMM_SMEM_LIMIT = 232448;        // dynamic shared memory per CTA on this part
 constexpr int EPI_BLOCK_BYTES = 32 * 32 * 2;   // one 32 x 32 bf16 block
 
-// Staging blocks per epilogue warp: residual cache: out, r_hat, resid, x_in;
-// gated residual: out, resid; the others: out, double-buffered.
-template <int EPI>
+// Residual-cache epilogue with 256-wide tiles: the residual and block-input
+// blocks are loaded into the two buffers that then stage the output and
+// r_hat, so the main loop keeps four pipeline stages in shared memory (the
+// next blocks' loads wait until the stores have read the buffers).
+template <int EPI, int BN>
+__host__ __device__ constexpr bool epi_shared() {
+    return EPI == EPI_RESID_CACHE && BN == 256;
+}
+// Staging blocks per epilogue warp: residual cache: out, r_hat, resid, x_in
+// (2 when shared); gated residual: out, resid; the others: out,
+// double-buffered.
+template <int EPI, int BN>
 __host__ __device__ constexpr int epi_blocks() {
-    return EPI == EPI_RESID_CACHE ? 4 : 2;
+    return (EPI == EPI_RESID_CACHE && !epi_shared<EPI, BN>()) ? 4 : 2;
 }
 
 template <int BN, int EPI>
@@ -47,7 +56,7 @@ struct GemmTile {
     static constexpr int A_BYTES = GEMM_BM * GEMM_BK * 2;
     static constexpr int B_BYTES = BN * GEMM_BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int EPI_BYTES = 8 * epi_blocks<EPI>() * EPI_BLOCK_BYTES;
+    static constexpr int EPI_BYTES = 8 * epi_blocks<EPI, BN>() * EPI_BLOCK_BYTES;
     static constexpr int BAR_BYTES = 512;
     static constexpr int FIT = (GEMM_SMEM_LIMIT - 1024 - BAR_BYTES - EPI_BYTES) / STAGE_BYTES;
     static constexpr int STAGES = FIT > 6 ? 6 : FIT;
@@ -222,15 +231,16 @@ __global__ void __launch_bounds__(320, 1)
         // the tile; thread = row) and column half `half`, in 32-column blocks.
         constexpr bool RES = EPI == EPI_RESID_GATE || EPI == EPI_RESID_CACHE;
         constexpr bool CACHE = EPI == EPI_RESID_CACHE;
+        constexpr bool SHARED = epi_shared<EPI, BN>();
         const int ew = warp - 2;
         const int q = warp & 3;
         const int half = ew >> 2;
         const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
-        uint8_t *eb = smem + G::OFF_EPI + ew * epi_blocks<EPI>() * EPI_BLOCK_BYTES;
+        uint8_t *eb = smem + G::OFF_EPI + ew * epi_blocks<EPI, BN>() * EPI_BLOCK_BYTES;
         uint8_t *s_out0 = eb;
         uint8_t *s_aux = eb + EPI_BLOCK_BYTES;          // r_hat (cache) / resid (gate) / second out
-        uint8_t *s_res = CACHE ? eb + 2 * EPI_BLOCK_BYTES : s_aux;
-        uint8_t *s_xin = eb + 3 * EPI_BLOCK_BYTES;
+        uint8_t *s_res = (CACHE && !SHARED) ? eb + 2 * EPI_BLOCK_BYTES : (SHARED ? s_out0 : s_aux);
+        uint8_t *s_xin = SHARED ? s_aux : eb + 3 * EPI_BLOCK_BYTES;
         uint64_t *lb = &ld_bar[ew];
         const bool has_rhat = CACHE && ep.rhat != nullptr;
         const uint32_t ld_bytes = (uint32_t)EPI_BLOCK_BYTES * (has_rhat ? 2u : 1u);
@@ -251,6 +261,10 @@ __global__ void __launch_bounds__(320, 1)
             const uint32_t use = (uint32_t)(local >> 1);
             const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
             const int row = m0 + q * 32 + lane;
+            if constexpr (SHARED) {
+                if (lane == 0) bulk_wait_read<0>();
+                __syncwarp();
+            }
             if constexpr (RES) load_res(m0, n0 + half * (BN / 2));
             // RoPE position of this thread's row (camera, frame, h, w), once per tile
             int pos0 = 0, pos1 = 0, pos2 = 0, pos3 = 0;
@@ -309,7 +323,7 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = r[i] + __shfl_sync(0xffffffffu, g_cur, i) * v[i];
                     __syncwarp();                      // every lane has read the block
-                    if (j + 1 < BN / 64) load_res(m0, col + 32);
+                    if (!SHARED && j + 1 < BN / 64) load_res(m0, col + 32);
                 }
                 if constexpr (EPI == EPI_GELU) {
 #pragma unroll
@@ -359,6 +373,13 @@ __global__ void __launch_bounds__(320, 1)
                     bulk_commit();
                 }
                 ++n_st;
+                if constexpr (SHARED) {
+                    if (j + 1 < BN / 64) {
+                        if (lane == 0) bulk_wait_read<0>();
+                        __syncwarp();
+                        load_res(m0, col + 32);
+                    }
+                }
             }
         }
         // every TMA store of this warp has completed before the CTA exits

@@ -228,10 +228,11 @@ def test_linear_full_size_sampled(M, N, K, epi):
     b = rt(f"Fb{N}", (N,), std=0.1, bf16=False)
     g = rt(f"Fg{N}", (N,), std=0.5, bf16=False)
     res = rt(f"Fr{M}{N}", (M, N))
+    xin = rt(f"Fx{M}{N}", (M, N))
     out = torch.empty(M, N, device=DEV, dtype=torch.bfloat16)
     rh = torch.empty_like(out)
     xb.op_linear("bf16", epi, dev(A, "bf16"), dev(Wt, "bf16"), dev(b, "f32"), out, gate=dev(g, "f32"),
-                 resid=dev(res, "bf16"), xin=dev(res, "bf16"), rhat=rh)
+                 resid=dev(res, "bf16"), xin=dev(xin, "bf16"), rhat=rh)
     torch.cuda.synchronize()
     rows = np.unique(np.r_[0, 127, 128, M - 1, np.random.default_rng(4).integers(0, M, 100)])
     y = A[rows].astype(np.float64) @ Wt.astype(np.float64).T + b
@@ -242,6 +243,10 @@ def test_linear_full_size_sampled(M, N, K, epi):
     else:
         want = O.to_bf16(res[rows] + g * y)
     assert_close(host(out)[rows], want, "bf16")
+    if epi == xb.XC_EPI_RESID_CACHE:
+        # r_hat of every row (256-wide tiles: the staging buffers are shared
+        # between the residual operands and the two outputs)
+        np.testing.assert_array_equal(host(rh), O.to_bf16(host(out) - xin))
 
 
 # Split-mode cases: more (head, 256-query) units than SMs, few key tiles, so
