@@ -23,6 +23,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -106,7 +107,9 @@ class ClockSampler:
     def __init__(self, gpu: int):
         self.gpu = gpu
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu}.csv")
+        # raw samples go to $XC_BENCH_OUT (default: the system temp directory)
+        out = os.environ.get("XC_BENCH_OUT") or tempfile.gettempdir()
+        self.path = os.path.join(out, f"xc_clocks_gpu{gpu}.csv")
 
     def start(self):
         try:
