@@ -295,15 +295,7 @@ __global__ void __launch_bounds__(320, 1)
                     if constexpr (RES) g_next = ep.gate[col + 32 + lane];
                 }
                 float v[32];
-                {
-                    float t[16];
-                    tmem_ld16_sync(tq + buf * BN + c, t);
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) v[i] = t[i];
-                    tmem_ld16_sync(tq + buf * BN + c + 16, t);
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) v[16 + i] = t[i];
-                }
+                tmem_ld32_sync(tq + buf * BN + c, v);
                 if (j == BN / 64 - 1) {
                     // last TMEM read of this tile: hand the accumulator back
                     tc_fence_before();
