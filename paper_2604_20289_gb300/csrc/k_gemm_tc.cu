@@ -497,11 +497,18 @@ static int gemm_sm_count() {
     return n;
 }
 
-// Output tile width for an M x N GEMM: 256, unless 128 x 256 tiles would
-// leave SMs idle (fewer tiles than SMs) and N allows 128-wide tiles.
+// Output tile width for an M x N GEMM.  128 when 128 x 256 tiles would leave
+// SMs idle.  Otherwise the persistent grid runs ceil(tiles / SMs) rounds of
+// tiles; a 128 x 256 tile costs about 1.75 times a 128 x 128 one (it reuses
+// each A tile for twice the columns), so 256 is taken when its rounds cost no
+// more than the 128-wide tiles' rounds.
 int gemm_tc_bn(int M, int N) {
-    const long tiles256 = (long)((M + GEMM_BM - 1) / GEMM_BM) * (N / 256);
-    return (N % 256 != 0 || (tiles256 < gemm_sm_count() && N % 128 == 0)) ? 128 : 256;
+    if (N % 256 != 0) return 128;
+    const long m_tiles = (M + GEMM_BM - 1) / GEMM_BM, n_sm = gemm_sm_count();
+    if (m_tiles * (N / 256) < n_sm) return 128;
+    const long r256 = (m_tiles * (N / 256) + n_sm - 1) / n_sm;
+    const long r128 = (m_tiles * (N / 128) + n_sm - 1) / n_sm;
+    return 7 * r256 <= 4 * r128 ? 256 : 128;
 }
 
 template <int EPI, int BN>
