@@ -365,14 +365,15 @@ def test_cross_attention_argument_errors():
 
 
 # ------------------------------------------- full size, benchmark configuration
-def test_full_size_first_block_sampled_rows():
-    """The benchmark model at full size in the benchmark's launch
-    configuration (persistent GEMMs, attention split over the SMs with partial
-    merges, CUDA-graph replay of the pass): block 0 of the first pass of
-    chunk 0 on sampled token rows -- the first and last rows, tile edges and a
-    seeded random sample -- against the oracle (keys and values from every
-    token)."""
-    cfg = X.SMALL_BF16
+@pytest.mark.parametrize("cfg", [X.SMALL_BF16, X.DIT_1P3B.replace(name="dit1p3b_shape_2blk", n_blocks=2)],
+                         ids=["small_bf16", "dit1p3b_block_shape"])
+def test_full_size_first_block_sampled_rows(cfg):
+    """Full-size blocks in the benchmark's launch configuration (persistent
+    GEMMs -- 256-wide tiles and the shared-staging residual-cache epilogue at
+    the 1.3B block shape --, attention split over the SMs with partial merges,
+    CUDA-graph replay of the pass): block 0 of the first pass of chunk 0 on
+    sampled token rows -- the first and last rows, tile edges and a seeded
+    random sample -- against the oracle (keys and values from every token)."""
     w, xc = model(cfg)
     traj = X.Trajectory(cfg, n_chunks=1)
     L, d = cfg.tokens, cfg.d_model
