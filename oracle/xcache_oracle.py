@@ -6,8 +6,10 @@ the docstring.  Arithmetic is fp64.  For bf16 models every tensor that a BF16
 forward pass stores (Section 3.1.1: all DiT forward passes run in BF16) is
 rounded to bf16 at the operator's output; fp32 models are left in fp64.
 
-Parity status: primitives, fingerprint geometry and gate equations are pinned
-by tests/test_oracle_pins.py; the composition of a whole DiT block is pinned
+Parity status: primitives, fingerprint geometry and its global channel, the
+gate equations, the conditioning MLPs, the output head and both fingerprint
+refresh rules are pinned by tests/test_oracle_pins.py; the composition of a
+whole DiT block is pinned
 only by brute-force loops on tiny shapes and structural invariants (the
 paper's X-World weights are not available), and the paper's 71% skip rate is
 X-World-specific -- parity unpinned against the paper for those two.

@@ -643,3 +643,172 @@ def test_block_rows_subset_equals_full_block():
         sub, k2, v2 = m.block(1, x, mods[1], past_k, past_v, pos, ctx, rows=rows)
         np.testing.assert_allclose(sub, full[rows], rtol=1e-12, atol=1e-12)
         np.testing.assert_array_equal(k2, k)
+
+
+# ------------------------------- fingerprint global channel (Section 2.3.2)
+def test_fingerprint_global_channel_explicit_camera_loops():
+    """Global entry of every view group = per-camera token mean, summed by
+    explicit loops over each camera's own token slice (two groups of unequal
+    grids, so the camera slices are ragged); shifting one camera's tokens by a
+    constant moves that camera's mean by the constant and nothing else."""
+    cfg = X.GROUPS_F32
+    oc = O.OracleXCache(cfg, X.make_weights(cfg))
+    L, d = cfg.tokens, cfg.d_model
+    x = rng.standard_normal((L, d))
+    act = np.array([0.3, -0.2])
+    _, gl, ac = oc.fingerprint(x, act, 32)
+    want, tok = [], 0
+    for V, gh, gw in cfg.groups:
+        npc = cfg.frames * gh * gw
+        means = np.zeros((V, d))
+        for c in range(V):
+            for j in range(d):
+                s = 0.0
+                for i in range(tok + c * npc, tok + (c + 1) * npc):
+                    s += x[i, j]
+                means[c, j] = s / npc
+        want.append(means)
+        tok += V * npc
+    assert [g.shape for g in gl] == [w.shape for w in want] == [(2, d), (1, d)]
+    for g, w in zip(gl, want):
+        np.testing.assert_allclose(g, w, rtol=1e-12, atol=1e-13)
+    np.testing.assert_array_equal(ac, act)
+    # camera 1 of group 0 occupies tokens [96, 192): shift it by 0.75
+    xs = x.copy()
+    npc0 = cfg.frames * 6 * 8
+    xs[npc0:2 * npc0] += 0.75
+    _, gl2, _ = oc.fingerprint(xs, act, 32)
+    np.testing.assert_allclose(gl2[0][0], gl[0][0], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(gl2[0][1], gl[0][1] + 0.75, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(gl2[1], gl[1], rtol=0, atol=1e-13)
+
+
+# ------------------------------------- conditioning (adaLN-Zero, Section 1)
+COND_CFG = X.ModelCfg("pin_cond_d8", 3, 8, 1, 8, 16, 1, 1, 1, 1, 2, 1, dtype="f32", t_freq=6)
+
+
+def test_cond_with_zero_projections_is_bias_plus_block_table():
+    """Every matrix zero: SiLU(e) W_m vanishes, so the six vectors of block b
+    are b_m (split as shift1, scale1, gate1, shift2, scale2, gate2) plus the
+    block's own table row, and the head's (shift, scale) are b_h + its table."""
+    cfg = COND_CFG
+    w = {k: v.astype(np.float64) for k, v in X.make_weights(cfg).items()}
+    for k in ("t_w1", "t_w2", "a_w1", "a_w2", "mod_w", "head_w"):
+        w[k] = np.zeros_like(w[k])
+    mods, hm = O.OracleModel(cfg, w).cond(0.6, np.array([0.4, -0.7]))
+    d = cfg.d_model
+    for b in range(cfg.n_blocks):
+        for s in range(6):
+            for c in range(d):
+                assert mods[b, s, c] == w["mod_b"][s * d + c] + w["blk_mod"][b, s, c]
+    for s in range(2):
+        for c in range(d):
+            assert hm[s, c] == w["head_b"][s * d + c] + w["head_tab"][s, c]
+
+
+def test_cond_scalar_loops():
+    """The two conditioning MLPs, the shared modulation projection and the
+    head projection as scalar loops (d = 8, 6 sinusoid features):
+      te = [cos(1000 sigma f_i), sin(1000 sigma f_i)], f_i = 10000^(-i/3)
+      e  = (SiLU(te W_t1 + b_t1) W_t2 + b_t2) + (SiLU(a W_a1 + b_a1) W_a2 + b_a2)
+      mods[b][s][c] = sum_k SiLU(e_k) W_m[k][s d + c] + b_m[s d + c] + table[b][s][c]
+      hm[s][c]      = sum_k SiLU(e_k) W_h[k][s d + c] + b_h[s d + c] + table_h[s][c]."""
+    cfg = COND_CFG
+    w = {k: v.astype(np.float64) for k, v in X.make_weights(cfg).items()}
+    for k in w:                       # random biases and tables too
+        if k.endswith("_b") or k in ("blk_mod", "head_tab"):
+            w[k] = rng.standard_normal(w[k].shape) * 0.3
+    sigma, a = 0.35, [0.45, -0.8]
+    mods, hm = O.OracleModel(cfg, w).cond(sigma, np.array(a))
+    d, tf = cfg.d_model, cfg.t_freq
+
+    def silu(v):
+        return v / (1.0 + math.exp(-v))
+
+    half = tf // 2
+    te = [math.cos(1000 * sigma * 10000 ** (-i / half)) for i in range(half)] + \
+         [math.sin(1000 * sigma * 10000 ** (-i / half)) for i in range(half)]
+    ht = [silu(sum(te[i] * w["t_w1"][i, j] for i in range(tf)) + w["t_b1"][j]) for j in range(d)]
+    ha = [silu(sum(a[i] * w["a_w1"][i, j] for i in range(2)) + w["a_b1"][j]) for j in range(d)]
+    e = [sum(ht[k] * w["t_w2"][k, j] for k in range(d)) + w["t_b2"][j]
+         + sum(ha[k] * w["a_w2"][k, j] for k in range(d)) + w["a_b2"][j] for j in range(d)]
+    se = [silu(v) for v in e]
+    for b in range(cfg.n_blocks):
+        for s in range(6):
+            for c in range(d):
+                want = sum(se[k] * w["mod_w"][k, s * d + c] for k in range(d)) + w["mod_b"][s * d + c] \
+                    + w["blk_mod"][b, s, c]
+                assert mods[b, s, c] == pytest.approx(want, rel=1e-12, abs=1e-13)
+    for s in range(2):
+        for c in range(d):
+            want = sum(se[k] * w["head_w"][k, s * d + c] for k in range(d)) + w["head_b"][s * d + c] \
+                + w["head_tab"][s, c]
+            assert hm[s, c] == pytest.approx(want, rel=1e-12, abs=1e-13)
+
+
+# ------------------------------------------------------------ output head
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_head_element_loops(dtype):
+    """v[i][c] = sum_j h[i][j] W_out[j][c] + b_out[c] with
+    h[i][j] = LN(x_i)_j (1 + scale_j) + shift_j, (shift, scale) = hm; the
+    bf16 model rounds h (the stored modulated activation) and keeps v fp64."""
+    cfg = COND_CFG.replace(name=f"pin_head_{dtype}", dtype=dtype)
+    w = X.make_weights(cfg)
+    m = O.OracleModel(cfg, w)
+    W, bo = m.w["out_w"], m.w["out_b"]
+    x = rng.standard_normal((5, cfg.d_model)) * 2.0 + 0.5
+    hm = rng.standard_normal((2, cfg.d_model))
+    got = m.head(x, hm)
+    d, C = cfg.d_model, cfg.c_latent
+    rnd = (lambda t: float(O.to_bf16(t))) if dtype == "bf16" else (lambda t: t)
+    assert got.shape == (5, C)
+    for i in range(5):
+        mu = sum(x[i]) / d
+        var = sum((x[i, j] - mu) ** 2 for j in range(d)) / d
+        h = [rnd((x[i, j] - mu) / math.sqrt(var + cfg.ln_eps) * (1 + hm[1, j]) + hm[0, j]) for j in range(d)]
+        for c in range(C):
+            want = sum(h[j] * W[j, c] for j in range(d)) + bo[c]
+            assert got[i, c] == pytest.approx(want, rel=1e-12, abs=1e-12)
+
+
+# --------------------------- fingerprint refresh on every evaluation (c5)
+@pytest.mark.parametrize("refresh", [0, 1])
+def test_fingerprint_refresh_after_skip(refresh):
+    """fp_refresh = 1 (literal "previous generation" of Eq. 5-6): after an
+    evaluated skip the cell holds the fingerprint of that pass's block input
+    (its sampled rows, per-camera means and the chunk's action).  fp_refresh
+    = 0: a skip leaves the cached fingerprint (the input that produced r_hat)
+    untouched."""
+    cfg = X.TINY_F32.replace(name="pin_refresh", n_chunks=4)
+    w = X.make_weights(cfg)
+    traj = X.Trajectory(cfg, n_chunks=4)
+    p = O.GateParams(tau_floor=0.0, margin=1.0, tau_dev=1e9, fp_refresh=refresh)
+    oc = O.OracleXCache(cfg, w)
+    rows = O.fingerprint_rows(cfg.n_cams, cfg.frames, cfg.grid_h, cfg.grid_w, 32)
+    npc = cfg.frames * cfg.grid_h * cfg.grid_w
+    S = cfg.n_steps
+    n_skips = 0
+    for n in range(4):
+        x = np.asarray(traj.noise(n), np.float64)
+        a = traj.action(n)
+        for t in range(S):
+            before = [(c.phi_sp, c.phi_gl, c.phi_act) for c in oc.cells[t]]
+            tr = []
+            v, st = oc.chunk_step(x, a, O.SIGMAS[t], t, False, p, trace=tr)
+            x_in0 = oc.model.patch_embed(x)
+            for b in range(cfg.n_blocks):
+                if st["decision"][b] != O.Decision.SKIP:
+                    continue
+                n_skips += 1
+                cell = oc.cells[t][b]
+                if refresh == 0:
+                    assert cell.phi_sp is before[b][0] and cell.phi_gl is before[b][1]
+                    continue
+                xin = x_in0 if b == 0 else tr[b - 1]
+                np.testing.assert_array_equal(cell.phi_sp[0], np.stack([xin[r] for r in rows]))
+                means = np.stack([xin[c * npc:(c + 1) * npc].sum(axis=0) / npc for c in range(cfg.n_cams)])
+                np.testing.assert_allclose(cell.phi_gl[0], means, rtol=1e-12, atol=1e-14)
+                np.testing.assert_array_equal(cell.phi_act, a)
+            x = x + (O.SIGMAS[t + 1] - O.SIGMAS[t]) * v
+        oc.chunk_step(traj.clean(n), a, 0.0, S, True, p)
+    assert n_skips > 0
