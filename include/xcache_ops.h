@@ -83,7 +83,8 @@ typedef struct {
     int pad[2];
 } xc_gate_cell;
 
-/* Bytes of device workspace xc_op_gate needs for this geometry. */
+/* Bytes of device workspace xc_op_gate needs for this geometry on the current
+ * device (the gate's grid splits each camera's rows over the device's SMs). */
 size_t xc_op_gate_workspace_bytes(int dtype, int n_cams, int tokens_per_cam, int d);
 
 /* One gate evaluation of one (t, b) cell (Section 2.3-2.5): fingerprint of the
@@ -113,24 +114,30 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
                      float *s_cos, float *d_max, float *tau, void *workspace, size_t workspace_bytes,
                      void *stream);
 
-/* Allocation-free variant of xc_op_gate, for callers that cannot allocate
- * device memory when they call in: code that runs while a stream is being
- * captured into a CUDA graph, code held to a fixed device-memory budget, or an
- * embedding runtime that owns the only allocator.  The paper has no
- * counterpart; this is an interface of this library.
- * Same arguments and results as xc_op_gate minus the workspace: the gate's
- * scratch (column sums, partial metrics, tickets) lives in one file-scope
- * device array of 1 MiB (GATE_STATIC_SCRATCH_BYTES) that every GPU which
- * loads the library keeps until the process exits.  Nothing is allocated or
- * freed; the tickets are cleared with cudaMemsetAsync on each call.
+/* Allocation-free variant of xc_op_gate.  The paper has no counterpart; this
+ * is an interface of this library, for callers that cannot call cudaMalloc
+ * when they call in: a runtime that owns the only device allocator of the
+ * process (a plugin or embedding host), code held to a device-memory budget
+ * fixed at start-up, or a latency-critical loop where an allocation and the
+ * device synchronisation it may bring are not acceptable.
+ * Same arguments, checks and results as xc_op_gate minus the workspace: the
+ * gate's scratch (per-CTA partial metrics and column sums, and the tickets)
+ * lives in one file-scope device array of 1 MiB (GATE_STATIC_SCRATCH_BYTES)
+ * that every GPU which loads the library keeps until the process exits.
+ * Nothing is allocated or freed; the tickets are cleared with
+ * cudaMemsetAsync on each call.
  * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) and should come before any stream capture.
+ * (cudaGetSymbolAddress) and caches it for that device for the rest of the
+ * process; that first call should come before any stream capture.  The
+ * cached address belongs to the device's primary context: do not use this
+ * entry point after cudaDeviceReset() on that device, or from a context other
+ * than the primary one.
  * All calls share the one array and it keeps the last call's contents:
  * calls that overlap on the GPU (different streams, no ordering) race; calls
  * ordered on one stream are safe.
- * Errors: XC_EINVAL for bad arguments or a geometry whose scratch exceeds
- * 1 MiB (the message states the bytes needed), XC_ECUDA if the device or the
- * array's address cannot be obtained. */
+ * Errors: XC_EINVAL for bad arguments (as xc_op_gate) or a geometry whose
+ * scratch exceeds 1 MiB (the message states the bytes needed), XC_ECUDA if
+ * the device or the array's address cannot be obtained. */
 xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam, int d, const void *x,
                             const int *fp_rows, int kfp, float *phi, float *phi_act, xc_gate_cell *cell,
                             const float *action, int action_dim, int mode, int step,

@@ -11,15 +11,24 @@
 // spatial entry (Eq. 6).  Decision Eq. 7 with tau_cos = max(tau_floor, ema -
 // m) (Eq. 9), EMA update (Eq. 8) and the consecutive-skip cap (Section 2.5 (4)).
 //
-// Grid: one CTA (512 threads) per (camera c, 64-column slice s).  The CTA
-// streams all of camera c's rows of its slice once (16-byte loads, 8 rows in
-// flight per thread), so it completes that slice's per-camera means by
-// itself; it also takes the slice of the spatial sample.  All reductions run
-// in fp32; each CTA writes 8 partials and takes an atomic ticket; the last
-// CTA combines the partials of each group in a fixed order and makes the
-// decision (the EMA state is kept in fp64).  No spin-wait anywhere; deterministic.  The cached
-// fingerprint is double-buffered per (t, b): the current fingerprint goes to
-// the inactive half, which becomes active when the block recomputes.
+// Grid: one CTA (256 threads) per (camera c, 64-column slice s, row block r);
+// the row blocks split each camera's tokens so that the grid fills every SM
+// (about eight CTAs per SM).  A CTA streams its rows of its slice once
+// (16-byte loads, 8 rows in flight per thread) into 64 column sums, and takes
+// every R-th row of the camera's spatial sample in its slice.  Three folds
+// follow, each in a fixed order (deterministic, no spin-wait anywhere):
+//   1. the last CTA of a (camera, slice) to arrive (per-slice ticket) adds the
+//      R column-sum partials in row-block order, giving the slice of the
+//      camera's mean, and its global-channel products;
+//   2. every CTA writes 8 partial metrics (its sample products; the slice
+//      folder also its global-channel products);
+//   3. the last CTA of the grid (global ticket) adds the partials of each
+//      view group in CTA order and thread 0 applies Eq. 5-9 (metrics in fp32,
+//      EMA state in fp64), writing the decision byte every later kernel of the
+//      block reads.
+// Every ticket is left at zero for the next launch.  The cached fingerprint
+// is double-buffered per (t, b): the current fingerprint goes to the inactive
+// half, which becomes active when the block recomputes.
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -30,9 +39,10 @@
 namespace xc {
 
 constexpr int GATE_CW = 64;          // columns per CTA
-constexpr int GATE_THREADS = 512;
+constexpr int GATE_THREADS = 256;
 constexpr int GATE_UNROLL = 8;       // rows in flight per thread
 constexpr int GATE_PARTS = 8;        // dot, |cur|^2, |prev|^2, max|diff|, sum|prev| (spatial); dot, |cur|^2, |prev|^2 (global)
+constexpr int GATE_CTAS_PER_SM = 8;  // target CTAs per SM of the row split
 
 // Cosine of one entry from its dot product and squared norms (Eq. 5):
 // both norms < 1e-12 -> 1, exactly one -> 0, NaN -> 0.
@@ -62,6 +72,30 @@ __device__ __forceinline__ void add_vec16(float *acc, const uint4 u) {
     }
 }
 
+// Sum (or, for part 3, max) of the 8 partials over the CTA in a fixed order:
+// butterfly within each warp, then warps in index order by thread 0.
+__device__ __forceinline__ void cta_fold8(float (&v)[GATE_PARTS], float (*wpart)[GATE_PARTS], int lane, int warp,
+                                          int nw) {
+#pragma unroll
+    for (int k = 0; k < GATE_PARTS; ++k) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float w = __shfl_xor_sync(0xffffffffu, v[k], o);
+            v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
+        }
+        if (lane == 0) wpart[warp][k] = v[k];
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+#pragma unroll
+        for (int k = 0; k < GATE_PARTS; ++k) {
+            float a = wpart[0][k];
+            for (int w = 1; w < nw; ++w) a = k == 3 ? fmaxf(a, wpart[w][k]) : a + wpart[w][k];
+            v[k] = a;
+        }
+    }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     pdl_wait();
@@ -76,7 +110,9 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int blk = blockIdx.x;
-    const int c = blk / g.n_slices, s = blk % g.n_slices;
+    const int R = g.R;
+    const int r = blk % R, cs = blk / R;
+    const int c = cs / g.n_slices, s = cs % g.n_slices;
     const int d = g.d;
     // camera c's group (unrolled compare chain: constant parameter indices)
     int tok0 = g.g_tok0[0], cam0 = g.g_cam0[0], npc = g.g_npc[0], fp0 = g.g_fp0[0], kfp = g.g_kfp[0];
@@ -99,20 +135,21 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     const float *phi_prev = g.phi + (size_t)active * n_all;
     float *phi_next = g.phi + (size_t)(active ^ 1) * n_all;
 
-    // 1. column sums of camera c, columns [col0, col0 + 64)
-    float acc[VEC];
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) acc[i] = 0.0f;
+    // 1. column sums of rows [rb0, rb1) of camera c, columns [col0, col0 + 64)
     {
+        const int rb0 = r * g.rows_per;
+        const int rb1 = min(npc, rb0 + g.rows_per);
+        float acc[VEC];
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) acc[i] = 0.0f;
         const int ty = tid / TPR, tx = tid % TPR;
         const T *base = x + ctok0 * d + col0 + tx * VEC;
-        // GATE_UNROLL guarded loads in flight per step, the ragged end included
-        for (int r = ty; r < npc; r += GATE_UNROLL * RPAR) {
+        for (int row = rb0 + ty; row < rb1; row += GATE_UNROLL * RPAR) {
             uint4 u[GATE_UNROLL];
 #pragma unroll
             for (int k = 0; k < GATE_UNROLL; ++k)
-                u[k] = r + k * RPAR < npc ? *reinterpret_cast<const uint4 *>(base + (size_t)(r + k * RPAR) * d)
-                                          : make_uint4(0u, 0u, 0u, 0u);
+                u[k] = row + k * RPAR < rb1 ? *reinterpret_cast<const uint4 *>(base + (size_t)(row + k * RPAR) * d)
+                                            : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
             for (int k = 0; k < GATE_UNROLL; ++k) add_vec16<T>(acc, u[k]);
         }
@@ -120,53 +157,58 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         for (int i = 0; i < VEC; ++i) red[ty * GATE_CW + tx * VEC + i] = acc[i];
     }
     __syncthreads();
-
-    float p[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    // 2. global channel of this slice: per-camera means (threads 0..63)
     if (tid < GATE_CW) {
         float sum = 0.0f;
         for (int t = 0; t < RPAR; ++t) sum += red[t * GATE_CW + tid];
-        const float mean = sum / (float)npc;
-        const size_t e = (size_t)n_sp + (size_t)c * d + col0 + tid;
-        const float prev = phi_prev[e];
-        phi_next[e] = mean;
-        p[5] = mean * prev;
-        p[6] = mean * mean;
-        p[7] = prev * prev;
-    }
-    // 3. spatial sample rows of camera c in this slice
-    for (int it = tid; it < kfp * GATE_CW; it += GATE_THREADS) {
-        const int i = it / GATE_CW, j = it % GATE_CW;
-        const int row = g.fp_rows[crow0 + i];
-        const size_t e = ((size_t)crow0 + i) * d + col0 + j;
-        const float cur = to_f(x[(size_t)row * d + col0 + j]);
-        const float prev = phi_prev[e];
-        phi_next[e] = cur;
-        p[0] = fmaf(cur, prev, p[0]);
-        p[1] = fmaf(cur, cur, p[1]);
-        p[2] = fmaf(prev, prev, p[2]);
-        p[3] = fmaxf(p[3], fabsf(cur - prev));
-        p[4] += fabsf(prev);
-    }
-    // CTA reduction: within warps, then across warps in a fixed order
-#pragma unroll
-    for (int k = 0; k < GATE_PARTS; ++k) {
-        float v = p[k];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float w = __shfl_xor_sync(0xffffffffu, v, o);
-            v = k == 3 ? fmaxf(v, w) : v + w;
-        }
-        if (lane == 0) wpart[warp][k] = v;
-    }
-    __syncthreads();
-    if (tid < GATE_PARTS) {
-        float v = 0.0f;
-        for (int w = 0; w < NW; ++w) v = tid == 3 ? fmaxf(v, wpart[w][tid]) : v + wpart[w][tid];
-        g.part[(size_t)blk * GATE_PARTS + tid] = v;
+        g.colsum[(size_t)blk * GATE_CW + tid] = sum;
     }
 
-    // 4. ticket: the last CTA combines all partials and decides
+    float p[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    // 2. sample rows r, r + R, ... of camera c in this slice
+    {
+        const int n_mine = r < kfp ? (kfp - r + R - 1) / R : 0;
+        for (int it = tid; it < n_mine * GATE_CW; it += GATE_THREADS) {
+            const int i = r + (it / GATE_CW) * R, j = it % GATE_CW;
+            const int row = g.fp_rows[crow0 + i];
+            const size_t e = ((size_t)crow0 + i) * d + col0 + j;
+            const float cur = to_f(x[(size_t)row * d + col0 + j]);
+            const float prev = phi_prev[e];
+            phi_next[e] = cur;
+            p[0] = fmaf(cur, prev, p[0]);
+            p[1] = fmaf(cur, cur, p[1]);
+            p[2] = fmaf(prev, prev, p[2]);
+            p[3] = fmaxf(p[3], fabsf(cur - prev));
+            p[4] += fabsf(prev);
+        }
+    }
+
+    // 3. per-slice ticket: the last row block of (c, s) folds the column sums
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_last = atomicAdd(&g.slice_ticket[cs], 1u) == (unsigned)(R - 1);
+    __syncthreads();
+    if (s_last) {
+        __threadfence();
+        if (tid < GATE_CW) {
+            float sum = 0.0f;
+            for (int rr = 0; rr < R; ++rr) sum += __ldcg(&g.colsum[((size_t)cs * R + rr) * GATE_CW + tid]);
+            const float mean = sum / (float)npc;
+            const size_t e = (size_t)n_sp + (size_t)c * d + col0 + tid;
+            const float prev = phi_prev[e];
+            phi_next[e] = mean;
+            p[5] = mean * prev;
+            p[6] = mean * mean;
+            p[7] = prev * prev;
+        }
+        if (tid == 0) g.slice_ticket[cs] = 0u;
+    }
+    cta_fold8(p, wpart, lane, warp, NW);
+    if (tid == 0) {
+#pragma unroll
+        for (int k = 0; k < GATE_PARTS; ++k) g.part[(size_t)blk * GATE_PARTS + k] = p[k];
+    }
+
+    // 4. global ticket: the last CTA combines all partials and decides
     __threadfence();
     __syncthreads();
     if (tid == 0) s_last = atomicAdd(g.ticket, 1u) == (unsigned)(gridDim.x - 1);
@@ -174,13 +216,13 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     if (!s_last) return;
     __threadfence();
     // Per view group: fold the partials of the group's CTAs (cameras
-    // [g_cam0[q], g_cam0[q + 1]), every slice) in a fixed order; thread 0
-    // keeps the running min of the cosines and max of the deviations.
+    // [g_cam0[q], g_cam0[q + 1]), every slice and row block) in CTA order;
+    // thread 0 keeps the running min of the cosines and max of the deviations.
     float cos_min = INFINITY, dmax = 0.0f;
 #pragma unroll
     for (int q = 0; q < XC_MAX_GROUPS; ++q) {
         if (q >= g.n_groups) break;
-        const int b0 = g.g_cam0[q] * g.n_slices, b1 = g.g_cam0[q + 1] * g.n_slices;
+        const int b0 = g.g_cam0[q] * g.n_slices * R, b1 = g.g_cam0[q + 1] * g.n_slices * R;
         float v[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         for (int b = b0 + tid; b < b1; b += GATE_THREADS) {
 #pragma unroll
@@ -189,22 +231,8 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
                 v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
             }
         }
-#pragma unroll
-        for (int k = 0; k < GATE_PARTS; ++k) {
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const float w = __shfl_xor_sync(0xffffffffu, v[k], o);
-                v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
-            }
-            if (lane == 0) wpart[warp][k] = v[k];
-        }
-        __syncthreads();
+        cta_fold8(v, wpart, lane, warp, NW);
         if (tid == 0) {
-            for (int k = 0; k < GATE_PARTS; ++k) {
-                float a = wpart[0][k];
-                for (int w = 1; w < NW; ++w) a = k == 3 ? fmaxf(a, wpart[w][k]) : a + wpart[w][k];
-                v[k] = a;
-            }
             const int n_sp_q = (g.g_cam0[q + 1] - g.g_cam0[q]) * g.g_kfp[q] * d;
             float dq = v[3] / (v[4] / (float)n_sp_q + g.eps_dev);
             if (isnan(dq)) dq = INFINITY;
@@ -214,7 +242,7 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         __syncthreads();
     }
     if (tid != 0) return;
-    *g.ticket = 0;
+    *g.ticket = 0u;
 
     // All sums and metrics are fp32 (relative error ~1e-7, far inside the
     // 1e-3 band around a threshold): FP64 arithmetic, square roots and divides
@@ -226,7 +254,7 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         da = fmaf(a, b, da);
         na = fmaf(a, a, na);
         nb = fmaf(b, b, nb);
-        g.phi_act[(active ^ 1) * 8 + i] = g.action_dev != nullptr ? g.action_dev[i] : g.action[i];
+        g.phi_act[(active ^ 1) * 8 + i] = a;
     }
     const float cos_a = cos_rule_f(da, na, nb);
     const double s_min = (double)fminf(cos_min, cos_a);
@@ -258,31 +286,117 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     *g.flag = dec;
 }
 
-// Scratch of one gate launch: GATE_PARTS fp32 partials per CTA, then one
-// 32-bit ticket (which must be zero before the launch; the kernel leaves it
-// zero).  Returns the total bytes; *ticket_off receives the ticket's offset.
-size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off) {
-    *n_slices = d / GATE_CW;
-    const size_t part = (size_t)V * *n_slices * GATE_PARTS * sizeof(float);
-    *ticket_off = (part + 255) & ~(size_t)255;
-    return *ticket_off + 256;
+static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Grid and scratch of one gate launch for V cameras of at most max_npc tokens
+// each, d columns, on a device with n_sm SMs.  Scratch: 8 fp32 partials per
+// CTA, 64 fp32 column sums per CTA, then V * n_slices + 1 32-bit tickets
+// (zero before the first launch; every launch leaves them zero).
+GateGeom gate_geometry(int V, int max_npc, int d, int n_sm) {
+    GateGeom gg;
+    gg.n_slices = d / GATE_CW;
+    const int cs = V * gg.n_slices;
+    const int want = (GATE_CTAS_PER_SM * (n_sm > 0 ? n_sm : 1)) / cs;
+    const int most = (max_npc + 31) / 32;                  // at least 32 rows per row block
+    gg.R = want < 1 ? 1 : (want > most ? most : want);
+    gg.rows_per = (max_npc + gg.R - 1) / gg.R;
+    gg.n_ctas = cs * gg.R;
+    gg.colsum_off = align256((size_t)gg.n_ctas * GATE_PARTS * sizeof(float));
+    gg.tickets_off = gg.colsum_off + align256((size_t)gg.n_ctas * GATE_CW * sizeof(float));
+    gg.n_tickets = cs + 1;
+    gg.total = gg.tickets_off + align256((size_t)gg.n_tickets * sizeof(unsigned));
+    return gg;
+}
+
+void gate_bind_scratch(GateArgs &g, const GateGeom &gg, void *scratch) {
+    char *w = reinterpret_cast<char *>(scratch);
+    g.n_slices = gg.n_slices;
+    g.R = gg.R;
+    g.rows_per = gg.rows_per;
+    g.part = reinterpret_cast<float *>(w);
+    g.colsum = reinterpret_cast<float *>(w + gg.colsum_off);
+    g.slice_ticket = reinterpret_cast<unsigned *>(w + gg.tickets_off);
+    g.ticket = g.slice_ticket + gg.n_tickets - 1;
 }
 
 template <typename T>
 cudaError_t gate_launch(const GateArgs &g, cudaStream_t st) {
-    return launch_pdl(gate_kernel<T>, dim3(g.V * g.n_slices), dim3(GATE_THREADS), 0, st, g);
+    return launch_pdl(gate_kernel<T>, dim3(g.V * g.n_slices * g.R), dim3(GATE_THREADS), 0, st, g);
 }
 template cudaError_t gate_launch<float>(const GateArgs &, cudaStream_t);
 template cudaError_t gate_launch<bf16>(const GateArgs &, cudaStream_t);
 
+static int current_sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return 1;
+    return n;
+}
+
+// Checks the arguments of one operator-level gate evaluation (xc_op_gate and
+// xc_op_gate_static take the same ones) and packs them, scratch not bound.
+// Returns XC_OK or XC_EINVAL with the reason in msg.
+static xc_status gate_op_args(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows,
+                              int kfp, float *phi, float *phi_act, xc_gate_cell *cell, const float *action,
+                              int action_dim, int mode, int step, const xc_gate_params *gate, uint8_t *flag,
+                              float *s_cos, float *d_max, float *tau, GateArgs *out, char *msg, size_t msg_n) {
+    if (dtype != XC_F32 && dtype != XC_BF16) {
+        snprintf(msg, msg_n, "dtype");
+        return XC_EINVAL;
+    }
+    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0 || kfp < 1 || kfp > tokens_per_cam ||
+        action_dim < 1 || action_dim > 8 || (mode != 0 && mode != 1) || step < 0) {
+        snprintf(msg, msg_n, "bad shape or mode (d %% 64 == 0, 1 <= kfp <= tokens_per_cam, action_dim <= 8)");
+        return XC_EINVAL;
+    }
+    if (x == nullptr || fp_rows == nullptr || phi == nullptr || phi_act == nullptr || cell == nullptr ||
+        action == nullptr || flag == nullptr || s_cos == nullptr || d_max == nullptr || tau == nullptr) {
+        snprintf(msg, msg_n, "NULL pointer");
+        return XC_EINVAL;
+    }
+    xc_gate_params p;
+    if (gate != nullptr)
+        p = *gate;
+    else
+        xc_gate_params_default(&p);
+    if (!gate_ok(&p, 1, msg, msg_n)) return XC_EINVAL;
+    GateArgs &g = *out;
+    memset(&g, 0, sizeof g);
+    g.x = x;
+    g.d = d;
+    gate_single_group(g, n_cams, tokens_per_cam, kfp);
+    g.fp_rows = fp_rows;
+    g.phi = phi;
+    g.phi_act = phi_act;
+    for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
+    g.A = action_dim;
+    g.cell = reinterpret_cast<GateCell *>(cell);
+    g.mode = mode;
+    g.step = step;
+    g.tau_floor = p.tau_floor;
+    g.margin = p.margin;
+    g.alpha = p.alpha;
+    g.tau_dev = p.tau_dev;
+    g.eps_dev = p.eps_dev;
+    g.strict_tau = p.step0_strict_tau;
+    g.max_skips = p.max_skips;
+    g.fp_refresh = p.fp_refresh;
+    g.replay = p.replay_skip != nullptr ? (p.replay_skip[0] != 0 ? 1 : 0) : -1;
+    g.flag = flag;
+    g.s_cos = s_cos;
+    g.d_max = d_max;
+    g.tau_out = tau;
+    return XC_OK;
+}
+
 // ---------------------------------------------------------------------------
 // Allocation-free gate (xc_op_gate_static).  The gate kernel needs scratch for
-// its partial metrics and its ticket.  Here that scratch is one file-scope
-// device array: every GPU that loads the library holds it until the process
-// exits, and no call allocates or frees anything.  In host code the array's
-// name is only a host-side stand-in, so its device address is looked up once
-// per device with cudaGetSymbolAddress (the first call on a device does this
-// set-up) and passed to the kernel.
+// its partial metrics, column sums and tickets.  Here that scratch is one
+// file-scope device array: every GPU that loads the library holds it until
+// the process exits, and no call allocates or frees anything.  In host code
+// the array's name is only a host-side stand-in, so its device address is
+// looked up once per device with cudaGetSymbolAddress (the first call on a
+// device does this set-up) and passed to the kernel.
 // ---------------------------------------------------------------------------
 constexpr size_t GATE_STATIC_SCRATCH_BYTES = 1u << 20;   // 1 MiB
 static __device__ __align__(256) unsigned char g_gate_scratch[GATE_STATIC_SCRATCH_BYTES];
@@ -310,86 +424,91 @@ static cudaError_t static_scratch(void **out) {
 }  // namespace xc
 
 using xc::GateArgs;
-using xc::GateCell;
+using xc::GateGeom;
 
-extern "C" xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam, int d, const void *x,
-                                       const int *fp_rows, int kfp, float *phi, float *phi_act,
-                                       xc_gate_cell *cell, const float *action, int action_dim, int mode,
-                                       int step, const xc_gate_params *gate, uint8_t *flag, float *s_cos,
-                                       float *d_max, float *tau, void *stream) {
-    char msg[256];
-    auto fail = [&](xc_status s, const char *m) {
-        snprintf(msg, sizeof msg, "xc_op_gate_static: %s", m);
+extern "C" {
+
+size_t xc_op_gate_workspace_bytes(int dtype, int n_cams, int tokens_per_cam, int d) {
+    (void)dtype;
+    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0) return 0;
+    return xc::gate_geometry(n_cams, tokens_per_cam, d, xc::current_sm_count()).total;
+}
+
+static_assert(sizeof(xc_gate_cell) == sizeof(xc::GateCell), "gate cell layout");
+
+xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows, int kfp,
+                     float *phi, float *phi_act, xc_gate_cell *cell, const float *action, int action_dim, int mode,
+                     int step, const xc_gate_params *gate, uint8_t *flag, float *s_cos, float *d_max, float *tau,
+                     void *workspace, size_t workspace_bytes, void *stream) {
+    char why[200], msg[256];
+    GateArgs g;
+    xc_status st = xc::gate_op_args(dtype, n_cams, tokens_per_cam, d, x, fp_rows, kfp, phi, phi_act, cell, action,
+                                    action_dim, mode, step, gate, flag, s_cos, d_max, tau, &g, why, sizeof why);
+    if (st == XC_OK && workspace == nullptr) {
+        snprintf(why, sizeof why, "NULL workspace");
+        st = XC_EINVAL;
+    }
+    const GateGeom gg = xc::gate_geometry(n_cams, tokens_per_cam, d, xc::current_sm_count());
+    if (st == XC_OK && workspace_bytes < gg.total) {
+        snprintf(why, sizeof why, "workspace %zu bytes < %zu needed", workspace_bytes, gg.total);
+        st = XC_EINVAL;
+    }
+    if (st != XC_OK) {
+        snprintf(msg, sizeof msg, "xc_op_gate: %s", why);
         xc::set_global_error(msg);
-        return s;
-    };
-    if (dtype != XC_F32 && dtype != XC_BF16) return fail(XC_EINVAL, "dtype");
-    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0 || kfp < 1 || kfp > tokens_per_cam ||
-        action_dim < 1 || action_dim > 8 || (mode != 0 && mode != 1) || step < 0)
-        return fail(XC_EINVAL, "bad shape or mode (d % 64 == 0, 1 <= kfp <= tokens_per_cam, action_dim <= 8)");
-    if (x == nullptr || fp_rows == nullptr || phi == nullptr || phi_act == nullptr || cell == nullptr ||
-        action == nullptr || flag == nullptr || s_cos == nullptr || d_max == nullptr || tau == nullptr)
-        return fail(XC_EINVAL, "NULL pointer");
-    xc_gate_params p;
-    if (gate != nullptr)
-        p = *gate;
-    else
-        xc_gate_params_default(&p);
-    const float knobs[] = {p.tau_floor, p.margin, p.alpha, p.tau_dev, p.eps_dev, p.step0_strict_tau};
-    for (float v : knobs)
-        if (isnan(v)) return fail(XC_EINVAL, "NaN gate knob");
-    if (p.alpha < 0.0f || p.alpha > 1.0f || p.max_skips < 0 || (p.fp_refresh != 0 && p.fp_refresh != 1))
-        return fail(XC_EINVAL, "gate knob out of range");
+        return st;
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    xc::gate_bind_scratch(g, gg, workspace);
+    cudaError_t e = cudaMemsetAsync(g.slice_ticket, 0, gg.n_tickets * sizeof(unsigned), s);
+    if (e == cudaSuccess) e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, s) : xc::gate_launch<float>(g, s);
+    if (e != cudaSuccess) {
+        snprintf(msg, sizeof msg, "xc_op_gate: %s", cudaGetErrorString(e));
+        xc::set_global_error(msg);
+        return XC_ECUDA;
+    }
+    return XC_OK;
+}
 
-    int ns = 0;
-    size_t ticket_off = 0;
-    const size_t need = xc::gate_scratch(n_cams, d, &ns, &ticket_off);
-    if (need > xc::GATE_STATIC_SCRATCH_BYTES) {
+xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows,
+                            int kfp, float *phi, float *phi_act, xc_gate_cell *cell, const float *action,
+                            int action_dim, int mode, int step, const xc_gate_params *gate, uint8_t *flag,
+                            float *s_cos, float *d_max, float *tau, void *stream) {
+    char why[200], msg[320];
+    GateArgs g;
+    const xc_status st = xc::gate_op_args(dtype, n_cams, tokens_per_cam, d, x, fp_rows, kfp, phi, phi_act, cell,
+                                          action, action_dim, mode, step, gate, flag, s_cos, d_max, tau, &g, why,
+                                          sizeof why);
+    if (st != XC_OK) {
+        snprintf(msg, sizeof msg, "xc_op_gate_static: %s", why);
+        xc::set_global_error(msg);
+        return st;
+    }
+    const GateGeom gg = xc::gate_geometry(n_cams, tokens_per_cam, d, xc::current_sm_count());
+    if (gg.total > xc::GATE_STATIC_SCRATCH_BYTES) {
         snprintf(msg, sizeof msg,
                  "xc_op_gate_static: this geometry needs %zu bytes of scratch, more than the %zu-byte "
                  "static maximum (use xc_op_gate with a workspace)",
-                 need, xc::GATE_STATIC_SCRATCH_BYTES);
+                 gg.total, xc::GATE_STATIC_SCRATCH_BYTES);
         xc::set_global_error(msg);
         return XC_EINVAL;
     }
     void *scratch = nullptr;
-    if (xc::static_scratch(&scratch) != cudaSuccess) return fail(XC_ECUDA, "cudaGetSymbolAddress failed");
-    char *w = reinterpret_cast<char *>(scratch);
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    // the ticket must start at zero; the partials are overwritten
-    if (cudaMemsetAsync(w + ticket_off, 0, sizeof(unsigned), st) != cudaSuccess)
-        return fail(XC_ECUDA, "cudaMemsetAsync");
-
-    GateArgs g;
-    memset(&g, 0, sizeof g);
-    g.x = x;
-    g.d = d;
-    xc::gate_single_group(g, n_cams, tokens_per_cam, kfp);
-    g.fp_rows = fp_rows;
-    g.n_slices = ns;
-    g.phi = phi;
-    g.phi_act = phi_act;
-    for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
-    g.A = action_dim;
-    g.cell = reinterpret_cast<GateCell *>(cell);
-    g.mode = mode;
-    g.step = step;
-    g.tau_floor = p.tau_floor;
-    g.margin = p.margin;
-    g.alpha = p.alpha;
-    g.tau_dev = p.tau_dev;
-    g.eps_dev = p.eps_dev;
-    g.strict_tau = p.step0_strict_tau;
-    g.max_skips = p.max_skips;
-    g.fp_refresh = p.fp_refresh;
-    g.replay = p.replay_skip != nullptr ? (p.replay_skip[0] != 0 ? 1 : 0) : -1;
-    g.flag = flag;
-    g.s_cos = s_cos;
-    g.d_max = d_max;
-    g.tau_out = tau;
-    g.part = reinterpret_cast<float *>(w);
-    g.ticket = reinterpret_cast<unsigned *>(w + ticket_off);
-    const cudaError_t e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, st) : xc::gate_launch<float>(g, st);
-    if (e != cudaSuccess) return fail(XC_ECUDA, cudaGetErrorString(e));
+    if (xc::static_scratch(&scratch) != cudaSuccess) {
+        xc::set_global_error("xc_op_gate_static: cudaGetSymbolAddress failed");
+        return XC_ECUDA;
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    xc::gate_bind_scratch(g, gg, scratch);
+    // the tickets must start at zero; partials and column sums are overwritten
+    cudaError_t e = cudaMemsetAsync(g.slice_ticket, 0, gg.n_tickets * sizeof(unsigned), s);
+    if (e == cudaSuccess) e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, s) : xc::gate_launch<float>(g, s);
+    if (e != cudaSuccess) {
+        snprintf(msg, sizeof msg, "xc_op_gate_static: %s", cudaGetErrorString(e));
+        xc::set_global_error(msg);
+        return XC_ECUDA;
+    }
     return XC_OK;
 }
+
+}  // extern "C"

@@ -188,9 +188,8 @@ struct xc_ctx {
     float *h_stats;                            // pinned [3][B]
     int *d_err;
 
-    // gate scratch
-    int g_ns;
-    size_t g_ticket_off;
+    // gate scratch (grid and layout in g_geom)
+    GateGeom g_geom;
     char *g_scratch;
 
     // attention split workspace (partials of units cut between CTAs)
@@ -245,6 +244,21 @@ void set_err(xc_ctx *c, const char *fmt, ...) {
 }  // namespace
 
 void xc::set_global_error(const char *msg) { set_err(nullptr, "%s", msg); }
+
+bool xc::gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
+    auto bad = [&](const char *m) { snprintf(why, n, "invalid gate params: %s", m); return false; };
+    const float f[] = {p->tau_floor, p->margin, p->alpha, p->tau_dev, p->eps_dev, p->step0_strict_tau};
+    for (float v : f)
+        if (std::isnan(v)) return bad("NaN threshold");
+    if (p->alpha < 0.0f || p->alpha > 1.0f) return bad("alpha out of [0, 1]");
+    if (p->front_anchors < 0 || p->back_anchors < 0 || p->warmup_chunks < 0 || p->max_skips < 0)
+        return bad("negative count");
+    if (p->fp_tokens < 1) return bad("fp_tokens < 1");
+    if (p->fp_refresh != 0 && p->fp_refresh != 1) return bad("fp_refresh must be 0 or 1");
+    if (p->fp_linear != 0 && p->fp_linear != 1) return bad("fp_linear must be 0 or 1");
+    (void)B;
+    return true;
+}
 
 namespace {
 
@@ -319,21 +333,6 @@ bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
     return true;
 }
 
-bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
-    auto bad = [&](const char *m) { snprintf(why, n, "invalid gate params: %s", m); return false; };
-    const float f[] = {p->tau_floor, p->margin, p->alpha, p->tau_dev, p->eps_dev, p->step0_strict_tau};
-    for (float v : f)
-        if (std::isnan(v)) return bad("NaN threshold");
-    if (p->alpha < 0.0f || p->alpha > 1.0f) return bad("alpha out of [0, 1]");
-    if (p->front_anchors < 0 || p->back_anchors < 0 || p->warmup_chunks < 0 || p->max_skips < 0)
-        return bad("negative count");
-    if (p->fp_tokens < 1) return bad("fp_tokens < 1");
-    if (p->fp_refresh != 0 && p->fp_refresh != 1) return bad("fp_refresh must be 0 or 1");
-    if (p->fp_linear != 0 && p->fp_linear != 1) return bad("fp_linear must be 0 or 1");
-    (void)B;
-    return true;
-}
-
 // (Re)build the spatial sample for a token budget K; resets every gate cell.
 void drop_graphs(xc_ctx *ctx) {
     for (GraphEntry &e : ctx->graphs) cudaGraphExecDestroy(e.exec);
@@ -397,7 +396,8 @@ void clear_state(xc_ctx *ctx) {
     CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
     if (ctx->phi != nullptr)
         CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * ctx->phi_n_all * sizeof(float), ctx->st));
-    CK(cudaMemsetAsync(ctx->g_scratch + ctx->g_ticket_off, 0, sizeof(unsigned), ctx->st));
+    CK(cudaMemsetAsync(ctx->g_scratch + ctx->g_geom.tickets_off, 0, ctx->g_geom.n_tickets * sizeof(unsigned),
+                       ctx->st));
     CK(cudaStreamSynchronize(ctx->st));
     ctx->n = 0;
     ctx->kvc = 0;
@@ -586,7 +586,6 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
                 g.g_kfp[q] = ctx->g_kfp[q];
             }
             g.g_cam0[ctx->G] = ctx->V;
-            g.n_slices = ctx->g_ns;
             const size_t cell = (size_t)t * B + b;
             g.phi = ctx->phi + cell * 2 * ctx->phi_n_all;
             g.phi_act = ctx->phi_act + cell * 16;
@@ -608,8 +607,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.s_cos = ctx->s_cos + b;
             g.d_max = ctx->d_max + b;
             g.tau_out = ctx->tau + b;
-            g.part = reinterpret_cast<float *>(ctx->g_scratch);
-            g.ticket = reinterpret_cast<unsigned *>(ctx->g_scratch + ctx->g_ticket_off);
+            gate_bind_scratch(g, ctx->g_geom, ctx->g_scratch);
             LAUNCH(XC_K_GATE, b, 1, gate_launch<T>(g, st));
         }
 
@@ -1029,7 +1027,12 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         CK(cudaMallocHost(reinterpret_cast<void **>(&ctx->h_stats), 3 * XC_MAX_BLOCKS * sizeof(float)));
 
         // gate scratch
-        ctx->g_scratch = dalloc<char>(ctx, gate_scratch(ctx->V, d, &ctx->g_ns, &ctx->g_ticket_off));
+        {
+            int max_npc = 1;
+            for (int g = 0; g < ctx->G; ++g) max_npc = std::max(max_npc, ctx->g_npc[g]);
+            ctx->g_geom = gate_geometry(ctx->V, max_npc, d, ctx->n_sm);
+            ctx->g_scratch = dalloc<char>(ctx, ctx->g_geom.total);
+        }
         if (ctx->bf) {
             ctx->attn_ws_bytes = attn_workspace_bytes(ctx->hd);
             ctx->attn_ws = dalloc<char>(ctx, ctx->attn_ws_bytes);
@@ -1570,88 +1573,6 @@ xc_status xc_op_ln_mod(int dtype, int M, int d, float eps, const void *x, const 
                             eps, nullptr, st));
     else
         OP_FAIL(XC_EINVAL, "xc_op_ln_mod: dtype");
-    return XC_OK;
-}
-
-// Workspace of one gate launch: fp32 partials per CTA, then the ticket.
-struct GateWorkspace {
-    int ns;
-    size_t ticket, total;
-};
-static GateWorkspace gate_workspace(int V, int npc, int d) {
-    (void)npc;
-    GateWorkspace w;
-    w.total = gate_scratch(V, d, &w.ns, &w.ticket);
-    return w;
-}
-
-size_t xc_op_gate_workspace_bytes(int dtype, int n_cams, int tokens_per_cam, int d) {
-    (void)dtype;
-    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0) return 0;
-    return gate_workspace(n_cams, tokens_per_cam, d).total;
-}
-
-static_assert(sizeof(xc_gate_cell) == sizeof(GateCell), "gate cell layout");
-
-xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const void *x, const int *fp_rows, int kfp,
-                     float *phi, float *phi_act, xc_gate_cell *cell, const float *action, int action_dim, int mode,
-                     int step, const xc_gate_params *gate, uint8_t *flag, float *s_cos, float *d_max, float *tau,
-                     void *workspace, size_t workspace_bytes, void *stream) {
-    if (dtype != XC_F32 && dtype != XC_BF16) OP_FAIL(XC_EINVAL, "xc_op_gate: dtype");
-    if (n_cams < 1 || tokens_per_cam < 1 || d < 64 || d % 64 != 0 || kfp < 1 || kfp > tokens_per_cam ||
-        action_dim < 1 || action_dim > 8 || (mode != 0 && mode != 1) || step < 0)
-        OP_FAIL(XC_EINVAL, "xc_op_gate: bad shape or mode (d %% 64 == 0, 1 <= kfp <= tokens_per_cam, "
-                           "action_dim <= 8)");
-    if (x == nullptr || fp_rows == nullptr || phi == nullptr || phi_act == nullptr || cell == nullptr ||
-        action == nullptr || flag == nullptr || s_cos == nullptr || d_max == nullptr || tau == nullptr ||
-        workspace == nullptr)
-        OP_FAIL(XC_EINVAL, "xc_op_gate: NULL pointer");
-    xc_gate_params p;
-    if (gate != nullptr)
-        p = *gate;
-    else
-        xc_gate_params_default(&p);
-    char why[256];
-    if (!gate_ok(&p, 1, why, sizeof why)) OP_FAIL(XC_EINVAL, "xc_op_gate: %s", why);
-    const GateWorkspace ws = gate_workspace(n_cams, tokens_per_cam, d);
-    if (workspace_bytes < ws.total)
-        OP_FAIL(XC_EINVAL, "xc_op_gate: workspace %zu bytes < %zu needed", workspace_bytes, ws.total);
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    char *w = reinterpret_cast<char *>(workspace);
-    OP_CK(cudaMemsetAsync(w + ws.ticket, 0, sizeof(unsigned), st));
-    GateArgs g;
-    memset(&g, 0, sizeof g);
-    g.x = x;
-    g.d = d;
-    gate_single_group(g, n_cams, tokens_per_cam, kfp);
-    g.fp_rows = fp_rows;
-    g.n_slices = ws.ns;
-    g.phi = phi;
-    g.phi_act = phi_act;
-    for (int i = 0; i < action_dim; ++i) g.action[i] = action[i];
-    g.A = action_dim;
-    g.cell = reinterpret_cast<GateCell *>(cell);
-    g.mode = mode;
-    g.step = step;
-    g.tau_floor = p.tau_floor;
-    g.margin = p.margin;
-    g.alpha = p.alpha;
-    g.tau_dev = p.tau_dev;
-    g.eps_dev = p.eps_dev;
-    g.strict_tau = p.step0_strict_tau;
-    g.max_skips = p.max_skips;
-    g.fp_refresh = p.fp_refresh;
-    g.replay = p.replay_skip != nullptr ? (p.replay_skip[0] != 0 ? 1 : 0) : -1;
-    g.flag = flag;
-    g.s_cos = s_cos;
-    g.d_max = d_max;
-    g.tau_out = tau;
-    g.part = reinterpret_cast<float *>(w);
-    g.ticket = reinterpret_cast<unsigned *>(w + ws.ticket);
-    if (dtype == XC_BF16)
-        OP_CK(gate_launch<bf16>(g, st));
-    else
-        OP_CK(gate_launch<float>(g, st));
     return XC_OK;
 }
 

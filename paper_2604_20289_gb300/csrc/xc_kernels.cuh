@@ -21,7 +21,8 @@ struct GateArgs {
     int n_groups, n_rows;    // n_rows: sample rows of all cameras
     int g_cam0[XC_MAX_GROUPS + 1], g_tok0[XC_MAX_GROUPS], g_npc[XC_MAX_GROUPS], g_fp0[XC_MAX_GROUPS],
         g_kfp[XC_MAX_GROUPS];
-    int n_slices;            // 64-column slices: one CTA per (camera, slice)
+    int n_slices;            // 64-column slices
+    int R, rows_per;         // row blocks per camera and rows per row block: one CTA per (camera, slice, row block)
     float *phi;
     float *phi_act;
     float action[8];
@@ -34,8 +35,15 @@ struct GateArgs {
     int max_skips, fp_refresh, replay;
     uint8_t *flag;
     float *s_cos, *d_max, *tau_out;
-    float *part;             // scratch [V * n_slices][8]
+    float *part;             // scratch [V * n_slices * R][8] partial metrics
+    float *colsum;           // scratch [V * n_slices * R][64] column sums
+    unsigned *slice_ticket;  // scratch [V * n_slices], zero before the launch (left zero)
     unsigned *ticket;        // scratch, zero before the launch (left zero)
+};
+// Grid and scratch layout of one gate launch (k_gate.cu).
+struct GateGeom {
+    int n_slices, R, rows_per, n_ctas;
+    size_t colsum_off, tickets_off, n_tickets, total;
 };
 // One view group of V cameras, npc tokens and kfp sample rows each.
 inline void gate_single_group(GateArgs &g, int V, int npc, int kfp) {
@@ -49,8 +57,13 @@ inline void gate_single_group(GateArgs &g, int V, int npc, int kfp) {
     g.g_fp0[0] = 0;
     g.g_kfp[0] = kfp;
 }
-// Bytes of scratch of one gate launch (partials, then the ticket at *ticket_off).
-size_t gate_scratch(int V, int d, int *n_slices, size_t *ticket_off);
+// Gate grid for V cameras of at most max_npc tokens, d columns, n_sm SMs; the
+// scratch holds partials, column sums and tickets (see GateGeom).
+GateGeom gate_geometry(int V, int max_npc, int d, int n_sm);
+// Points the scratch fields (and grid fields) of g into `scratch`.
+void gate_bind_scratch(GateArgs &g, const GateGeom &gg, void *scratch);
+// Validates the gate knobs (NaN thresholds, ranges, counts); the reason goes to why.
+bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n);
 template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);
 bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 int gemm_tc_bn(int M, int N);

@@ -95,7 +95,10 @@ def oracle_eval(case, cell_kw, p, step):
     return s, d, tau, skip, cell
 
 
-CASES = [(X.SMALL_BF16, 0.97), (X.TINY_F32, 0.95), (X.DIT_1P3B.replace(n_blocks=1), 0.96)]
+# small model (8 column slices x 6 cameras, rows split over the SMs), tiny fp32
+# model (one CTA per camera), 1.3B and 14B block inputs (d 1536 and 5120)
+CASES = [(X.SMALL_BF16, 0.97), (X.TINY_F32, 0.95), (X.DIT_1P3B.replace(n_blocks=1), 0.96),
+         (X.DIT_14B.replace(n_blocks=1), 0.96)]
 
 
 @pytest.mark.parametrize("cfg,rho", CASES, ids=lambda v: getattr(v, "name", str(v)))

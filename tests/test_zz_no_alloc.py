@@ -1,10 +1,10 @@
 """The allocation-free gate entry point (xc_op_gate_static) against the
 caller-workspace gate (xc_op_gate), through the C ABI, on two calls in a row.
 
-xc_op_gate_static exists for callers that cannot allocate device memory at
-call time (code running under stream capture, a fixed device-memory budget, an
-embedding runtime that owns the allocator): its scratch is a file-scope device
-array instead of a workspace.  Both run the same deterministic kernel, so the
+xc_op_gate_static exists for callers that cannot call cudaMalloc when they
+call in (a runtime that owns the process's only device allocator, a
+device-memory budget fixed at start-up, a latency-critical loop that must not
+allocate): its scratch is a file-scope device array instead of a workspace.  Both run the same deterministic kernel, so the
 outputs must agree within the gate tests' tolerances (abs 1e-6 on the metrics,
 exact decisions and cached fingerprints).  This file is collected last and
 passes both alone in a fresh process and after the other tests."""
@@ -103,7 +103,10 @@ def test_static_scratch_gate_rejects_geometry_beyond_its_maximum():
     buf = torch.zeros(1024, dtype=torch.uint8, device=DEV)
     p = buf.data_ptr()
     act = np.zeros(2, np.float32)
-    # 64 cameras x d 32768 = 64 x 512 column-slice CTAs x 64 bytes of partials = 2 MiB
+    # 64 cameras x d 32768: 32768 (camera, 64-column slice) CTAs, each with 8
+    # partial metrics and 64 column sums in fp32 -- about 9 MiB of scratch
+    need = xb.op_gate_workspace_bytes("bf16", 64, 8, 32768)
+    assert need > 8 * (1 << 20)
     st = xb.LIB.xc_op_gate_static(xb.XC_BF16, 64, 8, 32768, p, p, 1, p, p, p, act.ctypes.data, 2, 1, 1,
                                   None, p, p, p, p, None)
     assert st == xb.XC_EINVAL
