@@ -101,8 +101,9 @@ typedef struct {
     int d_ctx, max_ctx;
 } xc_model_cfg;
 
-/* Host float32 weights, math convention y = x @ W with W stored [in][out]
- * row-major.  For XC_BF16 models the values are rounded to bf16 on upload.
+/* Float32 weights, host or device pointers (each classified on its own),
+ * math convention y = x @ W with W stored [in][out] row-major.  For XC_BF16
+ * models the values are rounded to bf16 on upload.
  * Shapes (d = d_model, F = d_ffn, B = n_blocks, C = c_latent, A = action_dim,
  * T = t_freq_dim):
  *   pe_w [C][d] pe_b [d]                 patch embedding
@@ -118,7 +119,8 @@ typedef struct {
  *   ca_ln_w [B][d] ca_ln_b [B][d]   LN gain gamma and bias beta
  *   ca_q_w [B][d][d] ca_q_b [B][d]  ca_kv_w [B][D][2d] ca_kv_b [B][2d]
  *   ca_o_w [B][d][d] ca_o_b [B][d]
- * The pointers are only read during xc_init. */
+ * The pointers are only read during xc_init; device weights never pass
+ * through host memory. */
 typedef struct {
     const float *pe_w, *pe_b, *t_w1, *t_b1, *t_w2, *t_b2, *a_w1, *a_b1, *a_w2, *a_b2;
     const float *mod_w, *mod_b, *blk_mod;
@@ -140,7 +142,13 @@ typedef struct {
  *               rebuilds the sample and clears every gate cell.
  *   replay_skip host [n_blocks] or NULL: decision-replay mode -- for blocks the
  *               gate evaluates, the decision is replay_skip[b] != 0 instead of
- *               Eq. 7 (metrics, EMA and staleness are still updated). */
+ *               Eq. 7 (metrics, EMA and staleness are still updated).
+ *   replay_table device uint8 [n_denoise_steps][n_blocks] or NULL: the same
+ *               replay, read by the gate on the device from entry (t, b) when
+ *               the pass runs (takes precedence over replay_skip), so a
+ *               whole chunk's decisions can be set once without host copies.
+ *               The caller keeps the table alive and unchanged until the
+ *               passes that read it have completed. */
 typedef struct {
     int enabled;
     float tau_floor, margin, alpha, tau_dev, eps_dev;
@@ -149,6 +157,7 @@ typedef struct {
     float step0_strict_tau;
     int fp_tokens, fp_refresh, fp_linear;
     const uint8_t *replay_skip;
+    const uint8_t *replay_table;
 } xc_gate_params;
 
 /* Filled by xc_chunk_step when non-NULL (the call then synchronises with its

@@ -267,7 +267,10 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         if (g.strict_tau > 0.0f && g.step == 0) tau = fmax(tau, (double)g.strict_tau);
         bool skip = (s_min >= tau) && (dmax < g.tau_dev);
         if (g.max_skips > 0 && cell.stale >= g.max_skips) skip = false;
-        if (g.replay >= 0) skip = g.replay != 0;
+        if (g.replay_dev != nullptr)
+            skip = *g.replay_dev != 0;
+        else if (g.replay >= 0)
+            skip = g.replay != 0;
         cell.ema = cell.has_hist ? (double)g.alpha * s_min + (1.0 - (double)g.alpha) * cell.ema : s_min;
         cell.has_hist = 1;
         cell.stale = skip ? cell.stale + 1 : 0;

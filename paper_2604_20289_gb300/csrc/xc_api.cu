@@ -279,8 +279,9 @@ P *dalloc(xc_ctx *ctx, size_t bytes) {
     return reinterpret_cast<P *>(p);
 }
 
+// Host or device source: cudaMemcpyDefault classifies the pointer (unified addressing).
 void upload(xc_ctx *ctx, float *dst, const float *src, size_t n) {
-    CK(cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyDefault));
 }
 
 bool cfg_ok(const xc_model_cfg *c, char *why, size_t n) {
@@ -407,7 +408,7 @@ void clear_state(xc_ctx *ctx) {
 // Per-block weight upload: W [K][N] float32 (host) -> Wt [N][K] activation dtype.
 void upload_blocks(xc_ctx *ctx, void *dst, const float *src, int K, int N, float *tmp) {
     for (int b = 0; b < ctx->B; ++b) {
-        CK(cudaMemcpy(tmp, src + (size_t)b * K * N, (size_t)K * N * sizeof(float), cudaMemcpyHostToDevice));
+        CK(cudaMemcpy(tmp, src + (size_t)b * K * N, (size_t)K * N * sizeof(float), cudaMemcpyDefault));
         char *out = reinterpret_cast<char *>(dst) + (size_t)b * K * N * ctx->esz;
         if (ctx->bf)
             CK(transpose_convert<bf16>(tmp, reinterpret_cast<bf16 *>(out), K, N, ctx->st));
@@ -603,6 +604,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.max_skips = p.max_skips;
             g.fp_refresh = p.fp_refresh;
             g.replay = p.replay_skip != nullptr ? (p.replay_skip[b] != 0 ? 1 : 0) : -1;
+            g.replay_dev = p.replay_table != nullptr ? p.replay_table + (size_t)t * B + b : nullptr;
             g.flag = ctx->flags + b;
             g.s_cos = ctx->s_cos + b;
             g.d_max = ctx->d_max + b;
@@ -804,6 +806,7 @@ void xc_gate_params_default(xc_gate_params *p) {
     p->fp_tokens = 32;
     p->fp_refresh = 0;
     p->replay_skip = nullptr;
+    p->replay_table = nullptr;
 }
 
 const char *xc_last_error(const xc_ctx *ctx) {
@@ -933,7 +936,8 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         if (ctx->xattn) {
             const size_t Bd = (size_t)B * d;
             std::vector<float> gm1(Bd);
-            for (size_t i = 0; i < Bd; ++i) gm1[i] = w->ca_ln_w[i] - 1.0f;   // exact for gains in [0.5, 2]
+            CK(cudaMemcpy(gm1.data(), w->ca_ln_w, Bd * sizeof(float), cudaMemcpyDefault));
+            for (size_t i = 0; i < Bd; ++i) gm1[i] -= 1.0f;                  // exact for gains in [0.5, 2]
             up(ctx->ca_shift, w->ca_ln_b, Bd);
             up(ctx->ca_scale, gm1.data(), Bd);
             up(ctx->ca_q_b, w->ca_q_b, Bd);

@@ -32,7 +32,8 @@ struct GateArgs {
     int mode;
     int step;
     float tau_floor, margin, alpha, tau_dev, eps_dev, strict_tau;
-    int max_skips, fp_refresh, replay;
+    int max_skips, fp_refresh, replay;   // replay: -1 off, 0 / 1 the replayed decision
+    const uint8_t *replay_dev;           // device replay entry of this (t, b), or NULL
     uint8_t *flag;
     float *s_cos, *d_max, *tau_out;
     float *part;             // scratch [V * n_slices * R][8] partial metrics

@@ -60,7 +60,8 @@ class GateParams(ctypes.Structure):
                 ("warmup_chunks", ctypes.c_int), ("max_skips", ctypes.c_int),
                 ("protect_step0", ctypes.c_int), ("step0_strict_tau", ctypes.c_float),
                 ("fp_tokens", ctypes.c_int), ("fp_refresh", ctypes.c_int), ("fp_linear", ctypes.c_int),
-                ("replay_skip", ctypes.POINTER(ctypes.c_uint8))]
+                ("replay_skip", ctypes.POINTER(ctypes.c_uint8)),
+                ("replay_table", ctypes.c_void_p)]
 
 
 class StepStats(ctypes.Structure):
@@ -178,10 +179,15 @@ def model_cfg(cfg) -> ModelCfg:
 
 
 def gate_params(**kw) -> GateParams:
-    """Table 1 defaults, overridden by keyword (replay_skip: sequence of 0/1)."""
+    """Table 1 defaults, overridden by keyword (replay_skip: sequence of 0/1;
+    replay_table: torch CUDA uint8 tensor [n_denoise_steps, n_blocks], kept
+    alive by the caller)."""
     p = GateParams()
     LIB.xc_gate_params_default(ctypes.byref(p))
     replay = kw.pop("replay_skip", None)
+    table = kw.pop("replay_table", None)
+    if table is not None:
+        p.replay_table = table.data_ptr()
     for k, v in kw.items():
         if not hasattr(p, k):
             raise KeyError(k)
@@ -199,8 +205,11 @@ class XCache:
     def __init__(self, cfg, weights: dict, stream=None):
         self.cfg = cfg
         self._c_cfg = model_cfg(cfg)
-        keep = {k: np.ascontiguousarray(weights[k], dtype=np.float32) for k in WEIGHT_NAMES if k in weights}
-        w = Weights(*[keep[k].ctypes.data_as(ctypes.POINTER(ctypes.c_float)) if k in keep else None
+        # numpy arrays (host) or contiguous float32 torch CUDA tensors (device)
+        keep = {k: (weights[k] if hasattr(weights[k], "data_ptr") else
+                    np.ascontiguousarray(weights[k], dtype=np.float32))
+                for k in WEIGHT_NAMES if k in weights}
+        w = Weights(*[ctypes.cast(_ptr(keep[k]), ctypes.POINTER(ctypes.c_float)) if k in keep else None
                       for k in WEIGHT_NAMES])
         ctx = ctypes.c_void_p()
         self._stream = _stream(stream)

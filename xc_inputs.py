@@ -346,3 +346,64 @@ def random_tensor(seed: int, name: str, shape: tuple, std: float = 1.0,
     """Generic seeded normal tensor (float32) for kernel-level parity cases."""
     a = (normal(seed, name, int(np.prod(shape))) * std).astype(np.float32).reshape(shape)
     return bf16_representable(a) if bf16 else a
+
+
+# --------------------------------------------------------------------------
+# The same generator on a torch device (large benchmark models)
+# --------------------------------------------------------------------------
+def _i64(v: int) -> int:
+    """A 64-bit pattern as the signed int64 with the same bits."""
+    v &= 0xFFFFFFFFFFFFFFFF
+    return v - (1 << 64) if v >> 63 else v
+
+
+def _mix64_t(z):
+    """SplitMix64 output function on int64 tensors: wrapping products, logical
+    right shifts (arithmetic shift masked to the shifted width)."""
+    m1, m2 = _i64(int(_M1)), _i64(int(_M2))
+    z = (z ^ ((z >> 30) & ((1 << 34) - 1))) * m1
+    z = (z ^ ((z >> 27) & ((1 << 37) - 1))) * m2
+    return z ^ ((z >> 31) & ((1 << 33) - 1))
+
+
+def normal_torch(seed: int, name: str, n: int, device, offset: int = 0, block: int = 1 << 24):
+    """``normal`` computed on a torch device (float64): the same counters,
+    SplitMix64 stream and Box-Muller transform, so the values agree with the
+    numpy ones up to the last bit of the device's log / cos."""
+    import torch
+    key = _i64(int(_stream_key(seed, name)))
+    gamma = _i64(0x9E3779B97F4A7C15)
+    out = torch.empty(n, dtype=torch.float64, device=device)
+    for a in range(0, n, block):
+        m = min(block, n - a)
+        i = torch.arange(2 * (offset + a), 2 * (offset + a + m), dtype=torch.int64, device=device)
+        s = key + (i + 1) * gamma
+        bits = (_mix64_t(s) >> 11) & ((1 << 53) - 1)
+        u = (bits.to(torch.float64) + 0.5) * (1.0 / 9007199254740992.0)
+        u1, u2 = u[0::2], u[1::2]
+        out[a:a + m] = torch.sqrt(-2.0 * torch.log(u1)) * torch.cos(2.0 * math.pi * u2)
+    return out
+
+
+def make_weight_torch(cfg: ModelCfg, name: str, device, seed: int = 0):
+    """``make_weight`` generated on a torch device (float32 tensor)."""
+    import torch
+    shape = weight_shapes(cfg)[name]
+    std = _init_std(name, shape)
+    n = int(np.prod(shape))
+    out = torch.empty(n, dtype=torch.float32, device=device)
+    step = 1 << 26
+    for a in range(0, n, step):
+        m = min(step, n - a)
+        w = normal_torch(seed, cfg.name + "/" + name, m, device, offset=a) * std
+        if name in GAINS:
+            w = 1.0 + w
+        w = w.to(torch.float32)
+        if cfg.dtype == "bf16":
+            w = w.to(torch.bfloat16).to(torch.float32)
+        out[a:a + m] = w
+    return out.reshape(shape)
+
+
+def make_weights_torch(cfg: ModelCfg, device, seed: int = 0) -> dict:
+    return {k: make_weight_torch(cfg, k, device, seed) for k in weight_shapes(cfg)}
