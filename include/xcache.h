@@ -285,6 +285,14 @@ xc_status xc_profile_stop(xc_ctx *ctx, xc_profile_rec *out, int max, int *n_out)
  * (including early-exit launches of skipped blocks). */
 long long xc_launch_count(const xc_ctx *ctx);
 
+/* ---- testing hook (no counterpart in the paper) ----
+ * With n > 0 the n-th device allocation made by the library from now on
+ * (xc_init's weights, ring, caches and scratch; a rebuilt fingerprint
+ * sample) fails as if the device were out of memory: the call reports
+ * XC_ENOMEM and releases everything it had allocated.  n <= 0 switches the
+ * hook off.  Process-wide; for tests of the error paths. */
+void xc_debug_fail_alloc(int n);
+
 #ifdef __cplusplus
 }
 #endif

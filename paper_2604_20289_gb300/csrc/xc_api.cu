@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -271,9 +272,24 @@ namespace {
         }                                                                                   \
     } while (0)
 
+// Test hook (xc_debug_fail_alloc): when positive, the device allocation that
+// brings the count to zero fails as if the device were out of memory.
+std::atomic<int> g_fail_alloc{0};
+
+void maybe_fail_alloc(xc_ctx *ctx) {
+    int n = g_fail_alloc.load();
+    while (n > 0 && !g_fail_alloc.compare_exchange_weak(n, n - 1)) {
+    }
+    if (n == 1) {
+        set_err(ctx, "device allocation failed (injected by xc_debug_fail_alloc)");
+        throw Fail{XC_ENOMEM};
+    }
+}
+
 template <typename P>
 P *dalloc(xc_ctx *ctx, size_t bytes) {
     void *p = nullptr;
+    maybe_fail_alloc(ctx);
     CK(cudaMalloc(&p, bytes < 16 ? 16 : bytes));
     ctx->allocs.push_back(p);
     return reinterpret_cast<P *>(p);
@@ -961,6 +977,7 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
             if ((size_t)d * F > mx) mx = (size_t)d * F;
             if (ctx->xattn && (size_t)2 * d * ctx->d_ctx > mx) mx = (size_t)2 * d * ctx->d_ctx;
             float *tmp = nullptr;
+            maybe_fail_alloc(ctx);
             CK(cudaMalloc(&tmp, mx * sizeof(float)));
             try {
                 upload_blocks(ctx, ctx->qkv_wt, w->qkv_w, d, 3 * d, tmp);
@@ -1118,6 +1135,8 @@ xc_status xc_reset(xc_ctx *ctx) {
 }
 
 int xc_chunk_index(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->n; }
+
+void xc_debug_fail_alloc(int n) { g_fail_alloc.store(n > 0 ? n : 0); }
 
 long long xc_launch_count(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->launches; }
 
