@@ -278,6 +278,7 @@ class GateParams:
     fp_tokens: int = 32
     fp_refresh: int = 0          # 0 = refresh on compute, 1 = on every evaluation
     fp_linear: bool = False      # 1-D fallback sample instead of the 3-D grid
+    chain: bool = False          # lazy residual chaining over runs of skipped blocks (reading c27)
 
 
 class Decision(IntEnum):
@@ -487,6 +488,31 @@ class OracleXCache:
             tok0 += V * npc
         return sp, gl, np.asarray(action, np.float64).copy()
 
+    def chain_sum(self, base: np.ndarray, pending: list) -> np.ndarray:
+        """Reading c27: the block input after a run of skipped blocks, base +
+        r_hat_j + ... + r_hat_{b-1} (Eq. 4 applied over the run), accumulated
+        in float32 in block order and rounded once to the storage type."""
+        acc = np.asarray(base, np.float64).astype(np.float32)
+        for r in pending:
+            acc = acc + np.asarray(r, np.float64).astype(np.float32)
+        return self.model.R(acc.astype(np.float64))
+
+    def chained_fingerprint(self, base: np.ndarray, pending: list, action, K: int, linear: bool = False):
+        """phi of the lazily chained block input (reading c27): the spatial
+        entry is the chained sum on the sampled rows only; the global channel
+        is the per-camera mean of the last materialised input plus the
+        per-camera means of the pending cached residuals."""
+        sp, gl, tok0 = [], [], 0
+        for (V, gh, gw), rows in zip(self.cfg.groups, self.fp_rows(K, linear)):
+            npc = self.cfg.frames * gh * gw
+            sp.append(self.chain_sum(base[rows], [r[rows] for r in pending]))
+            m = np.asarray(base[tok0:tok0 + V * npc], np.float64).reshape(V, npc, -1).mean(axis=1)
+            for r in pending:
+                m = m + np.asarray(r[tok0:tok0 + V * npc], np.float64).reshape(V, npc, -1).mean(axis=1)
+            gl.append(m)
+            tok0 += V * npc
+        return sp, gl, np.asarray(action, np.float64).copy()
+
     def chunk_step(self, latent, action, sigma: float, step: int, is_kv_update: bool,
                    p: GateParams, replay=None, trace: list | None = None):
         """One forward pass over all B blocks.  Returns (v [L, C], stats) where
@@ -515,6 +541,11 @@ class OracleXCache:
         kv_new = {}
         stats = dict(decision=np.zeros(B, np.int64), s_cos=np.full(B, np.nan),
                      d_max=np.full(B, np.nan), tau=np.full(B, np.nan))
+        # Lazy residual chaining (reading c27): x is the last materialised
+        # block input; `pending` the cached residuals of the skipped blocks
+        # after it, added only when a block computes (or before the head).
+        chain = bool(getattr(p, "chain", False)) and not is_kv_update
+        pending = []
         for b in range(B):
             gated_block = (p.enabled and not is_kv_update
                            and p.front_anchors <= b < B - p.back_anchors)
@@ -522,7 +553,10 @@ class OracleXCache:
             phi = None
             if gated_block:
                 cell = self.cells[step][b]
-                phi = self.fingerprint(x, action, p.fp_tokens, p.fp_linear)
+                if chain and pending:
+                    phi = self.chained_fingerprint(x, pending, action, p.fp_tokens, p.fp_linear)
+                else:
+                    phi = self.fingerprint(x, action, p.fp_tokens, p.fp_linear)
                 eligible = (n >= p.warmup_chunks and not (p.protect_step0 and step == 0)
                             and not forced_chunk and cell.valid)
                 if eligible:
@@ -532,12 +566,23 @@ class OracleXCache:
                                             None if replay is None else bool(replay[b]))
                     stats["s_cos"][b], stats["d_max"][b], stats["tau"][b] = s, dmax, tau
                     stats["decision"][b] = Decision.SKIP if skip else Decision.COMPUTE
+            if skip and chain:
+                cell = self.cells[step][b]
+                pending.append(cell.r_hat)                                   # Eq. 4, deferred
+                if p.fp_refresh == 1:
+                    cell.phi_sp, cell.phi_gl, cell.phi_act = phi
+                if trace is not None:
+                    trace.append(self.chain_sum(x, pending))
+                continue
             if skip:
                 cell = self.cells[step][b]
                 x_out = M.R(x + cell.r_hat)                                  # Eq. 4
                 if p.fp_refresh == 1:
                     cell.phi_sp, cell.phi_gl, cell.phi_act = phi
             else:
+                if pending:                                                  # materialise the run
+                    x = self.chain_sum(x, pending)
+                    pending = []
                 x_out, k, v = M.block(b, x, mods[b], self.ring_k[b], self.ring_v[b], pos,
                                       self.ctx_kv[b] if xattn else None)
                 if is_kv_update:
@@ -550,6 +595,8 @@ class OracleXCache:
             if trace is not None:
                 trace.append(x_out)
             x = x_out
+        if pending:
+            x = self.chain_sum(x, pending)
         v = M.head(x, hm)
         if is_kv_update:
             for b in range(B):                                               # FIFO append

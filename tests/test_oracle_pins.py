@@ -812,3 +812,103 @@ def test_fingerprint_refresh_after_skip(refresh):
             x = x + (O.SIGMAS[t + 1] - O.SIGMAS[t]) * v
         oc.chunk_step(traj.clean(n), a, 0.0, S, True, p)
     assert n_skips > 0
+
+
+# ------------------------------- lazy residual chaining (NEXT-2, reading c27)
+def test_chained_fingerprint_explicit_loops():
+    """Fingerprint of a chained input: sampled rows of base + r1 + r2 summed
+    in float32 left to right and rounded once; global channel = per-camera
+    mean of base plus the per-camera means of r1 and r2 (explicit loops)."""
+    cfg = X.GROUPS_F32.replace(name="pin_chain_groups", dtype="bf16")
+    oc = O.OracleXCache(cfg, X.make_weights(cfg))
+    L, d = cfg.tokens, cfg.d_model
+    base = O.to_bf16(rng.standard_normal((L, d)))
+    rs = [O.to_bf16(0.1 * rng.standard_normal((L, d))) for _ in range(2)]
+    sp, gl, _ = oc.chained_fingerprint(base, rs, np.array([0.1, 0.2]), 32)
+    rows = O.group_fingerprint_rows(cfg.groups, cfg.frames, 32)
+    for g, (V, gh, gw) in enumerate(cfg.groups):
+        for c in range(V):
+            for i, row in enumerate(rows[g][c]):
+                for j in range(0, d, 7):
+                    a = np.float32(base[row, j])
+                    a = np.float32(a + np.float32(rs[0][row, j]))
+                    a = np.float32(a + np.float32(rs[1][row, j]))
+                    assert sp[g][c, i, j] == O.to_bf16(float(a))
+    tok = 0
+    for g, (V, gh, gw) in enumerate(cfg.groups):
+        npc = cfg.frames * gh * gw
+        for c in range(V):
+            sl = slice(tok + c * npc, tok + (c + 1) * npc)
+            for j in range(0, d, 5):
+                want = sum(base[sl, j]) / npc + sum(rs[0][sl, j]) / npc + sum(rs[1][sl, j]) / npc
+                assert gl[g][c, j] == pytest.approx(want, rel=1e-12, abs=1e-14)
+        tok += V * npc
+
+
+def test_chain_with_forced_recompute_is_the_plain_path():
+    """No block ever skips, so nothing is chained: bitwise the same rollout."""
+    cfg = X.TINY_F32
+    a, _, _ = _run(cfg, O.GateParams(**FORCE_RECOMPUTE), 4)
+    b, _, _ = _run(cfg, O.GateParams(chain=True, **FORCE_RECOMPUTE), 4)
+    for x, y in zip(a["final"], b["final"]):
+        np.testing.assert_array_equal(x, y)
+
+
+def test_chain_fp32_matches_plain_reuse_closely():
+    """fp32 model: chaining only changes the summation (float32 left to
+    right instead of one block at a time in fp64) and the global channel
+    (sum of means instead of mean of the sum, equal in exact arithmetic), so
+    decisions agree and final latents agree to float32 rounding."""
+    cfg = X.TINY_F32.replace(name="pin_chain_f32", n_chunks=5, n_blocks=4)
+    # the back anchor computes after a run of skipped blocks: its input is
+    # materialised from the chain
+    kw = dict(tau_floor=0.5, margin=1.0, tau_dev=100.0, front_anchors=0, back_anchors=1)
+    a, _, _ = _run(cfg, O.GateParams(**kw), 5)
+    b, _, _ = _run(cfg, O.GateParams(chain=True, **kw), 5)
+    da = np.array([[s["decision"] for s in ch] for ch in a["stats"]])
+    db = np.array([[s["decision"] for s in ch] for ch in b["stats"]])
+    np.testing.assert_array_equal(da, db)
+    assert (da == O.Decision.SKIP).sum() >= 4
+    for x, y in zip(a["final"], b["final"]):
+        np.testing.assert_allclose(y, x, rtol=1e-5, atol=1e-5 * np.abs(x).max())
+
+
+def test_chain_force_reuse_input_of_head_is_one_rounded_sum():
+    """bf16, every gated block skipped after the warmup chunk: the head sees
+    round(x_0 + r_hat_1 + ... + r_hat_{B-1}) summed in float32 block by
+    block (the anchor block 0 computes), checked through the trace's last
+    entry against an explicit loop over the cached residuals."""
+    cfg = X.TINY_F32.replace(name="pin_chain_bf16", dtype="bf16", n_blocks=4)
+    w = X.make_weights(cfg)
+    traj = X.Trajectory(cfg, n_chunks=2)
+    p = O.GateParams(chain=True, **FORCE_REUSE)
+    oc = O.OracleXCache(cfg, w)
+    S = cfg.n_steps
+    for n in range(2):
+        x = np.asarray(traj.noise(n), np.float64)
+        for t in range(S):
+            tr = []
+            v, st = oc.chunk_step(x, traj.action(n), O.SIGMAS[t], t, False, p, trace=tr)
+            if n == 1:
+                assert list(st["decision"][1:]) == [O.Decision.SKIP] * (cfg.n_blocks - 1)
+                acc = np.asarray(tr[0], np.float32)
+                for b in range(1, cfg.n_blocks):
+                    acc = (acc + np.asarray(oc.cells[t][b].r_hat, np.float32)).astype(np.float32)
+                np.testing.assert_array_equal(tr[-1], O.to_bf16(acc.astype(np.float64)))
+                # ... and the velocity is the head applied to that chained input
+                _, hm = oc.model.cond(O.SIGMAS[t], traj.action(n))
+                np.testing.assert_array_equal(v, oc.model.head(tr[-1], hm))
+            x = x + (O.SIGMAS[t + 1] - O.SIGMAS[t]) * v
+        oc.chunk_step(traj.clean(n), traj.action(n), 0.0, S, True, p)
+
+
+def test_chain_sum_accumulates_in_float32():
+    """1 + 2^-8 + 2^-24 + 2^-24 added left to right in float32: each 2^-24 is
+    half a float32 ulp and is lost (ties to even), the sum stays on the bf16
+    tie 1 + 2^-8 and rounds to even, 1.0.  The exact sum 1 + 2^-8 + 2^-23 is
+    a float32 value above the tie and rounds up to 1 + 2^-7."""
+    cfg = X.TINY_F32.replace(name="pin_chain_sum", dtype="bf16")
+    oc = O.OracleXCache(cfg, X.make_weights(cfg))
+    got = oc.chain_sum(np.array([1.0]), [np.array([2.0 ** -8]), np.array([2.0 ** -24]), np.array([2.0 ** -24])])
+    assert got[0] == 1.0
+    assert O.to_bf16(1.0 + 2.0 ** -8 + 2.0 ** -23) == 1.0 + 2.0 ** -7
