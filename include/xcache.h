@@ -140,6 +140,15 @@ typedef struct {
  *               cell-centred indices along each camera's token axis
  *               (Section 2.3.1).  Changing fp_tokens or fp_linear between calls
  *               rebuilds the sample and clears every gate cell.
+ *   chain       0: a skipped block writes x + r_hat at once (Eq. 4);
+ *               1: lazy residual chaining -- a run of skipped blocks writes
+ *               nothing; the gate of the next block takes the fingerprint of
+ *               the chained input from the sampled rows and the cached
+ *               residuals' per-camera means, and the input is written only
+ *               before a block that computes (or the head), as the last
+ *               written activation plus the run's residuals summed in fp32 in
+ *               block order and rounded once.  Switching chaining on clears
+ *               every gate cell; with a block trace set, passes do not chain.
  *   replay_skip host [n_blocks] or NULL: decision-replay mode -- for blocks the
  *               gate evaluates, the decision is replay_skip[b] != 0 instead of
  *               Eq. 7 (metrics, EMA and staleness are still updated).
@@ -156,6 +165,7 @@ typedef struct {
     int protect_step0;
     float step0_strict_tau;
     int fp_tokens, fp_refresh, fp_linear;
+    int chain;
     const uint8_t *replay_skip;
     const uint8_t *replay_table;
 } xc_gate_params;
@@ -256,10 +266,12 @@ int xc_chunk_index(const xc_ctx *ctx);
 /* ---- measurement (no counterpart in the paper; used by the benchmark) ---- */
 
 /* Kernel kinds of one forward pass (XC_K_XATTN: the four launches of a
- * cross-attention layer -- LN, q projection, attention, output projection). */
+ * cross-attention layer -- LN, q projection, attention, output projection;
+ * XC_K_CHAIN: lazy chaining -- the per-camera means of a new cached
+ * residual and the write of a chained input). */
 typedef enum {
     XC_K_COND = 0, XC_K_EMBED, XC_K_GATE, XC_K_LN, XC_K_QKV, XC_K_ATTN, XC_K_OPROJ,
-    XC_K_FFN1, XC_K_FFN2, XC_K_REUSE, XC_K_HEAD, XC_K_XATTN, XC_K_COUNT
+    XC_K_FFN1, XC_K_FFN2, XC_K_REUSE, XC_K_HEAD, XC_K_XATTN, XC_K_CHAIN, XC_K_COUNT
 } xc_kernel_kind;
 
 /* One timed launch: CUDA-event duration on the context's stream, the block

@@ -194,6 +194,124 @@ __global__ void __launch_bounds__(256)
     }
 }
 
+// d > 512: one CTA of LN_CTA threads per row.  The row is loaded once into
+// registers as packed 16-byte vectors (KMAX per thread, all loads in flight),
+// the mean and then the squared deviations are reduced over the CTA (warp
+// butterflies, then the warps in order), and the modulated row is written
+// back; many rows per SM are in flight at once.
+constexpr int LN_CTA = 128;
+
+template <typename T>
+__device__ __forceinline__ void unpack16B(const uint4 u, float (&f)[16 / sizeof(T)]) {
+    if constexpr (sizeof(T) == 2) {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 t = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
+            f[2 * j] = t.x;
+            f[2 * j + 1] = t.y;
+        }
+    } else {
+        f[0] = __uint_as_float(u.x);
+        f[1] = __uint_as_float(u.y);
+        f[2] = __uint_as_float(u.z);
+        f[3] = __uint_as_float(u.w);
+    }
+}
+template <typename T>
+__device__ __forceinline__ uint4 pack16B(const float (&f)[16 / sizeof(T)]) {
+    if constexpr (sizeof(T) == 2) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * j], f[2 * j + 1]);
+            w[j] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    } else {
+        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]), __float_as_uint(f[3]));
+    }
+}
+
+// Sum over the CTA in a fixed order (deterministic).
+__device__ __forceinline__ float cta_sum(float v, float *red) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float s = red[0];
+#pragma unroll
+    for (int w = 1; w < LN_CTA / 32; ++w) s += red[w];
+    return s;
+}
+
+template <typename T, int KMAX>
+__global__ void __launch_bounds__(LN_CTA)
+    ln_mod_cta_kernel(const T *__restrict__ x, const float *__restrict__ shift, const float *__restrict__ scale,
+                      T *__restrict__ out, int M, int d, float eps, const uint8_t *__restrict__ skip_flag) {
+    pdl_wait();
+    pdl_release();
+    if (skip_flag != nullptr && *skip_flag == XC_DEC_SKIP) return;
+    constexpr int VEC = 16 / sizeof(T);
+    __shared__ float red[2][LN_CTA / 32];
+    const int row = blockIdx.x, tid = threadIdx.x;
+    if (row >= M) return;
+    const int nch = d / VEC;
+    const uint4 *xr = reinterpret_cast<const uint4 *>(x + (size_t)row * d);
+    uint4 raw[KMAX];
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) {
+        const int c = tid + k * LN_CTA;
+        raw[k] = c < nch ? xr[c] : make_uint4(0u, 0u, 0u, 0u);
+    }
+    float s = 0.0f;
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) {
+        float f[VEC];
+        unpack16B<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) s += f[i];
+    }
+    const float mean = cta_sum(s, red[0]) / (float)d;
+    float m2 = 0.0f;
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) {
+        if (tid + k * LN_CTA < nch) {
+            float f[VEC];
+            unpack16B<T>(raw[k], f);
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) m2 = fmaf(f[i] - mean, f[i] - mean, m2);
+        }
+    }
+    const float rstd = rsqrtf(cta_sum(m2, red[1]) / (float)d + eps);
+    uint4 *orow = reinterpret_cast<uint4 *>(out + (size_t)row * d);
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) {
+        const int c = tid + k * LN_CTA;
+        if (c < nch) {
+            float f[VEC], sc[VEC], sh[VEC];
+            unpack16B<T>(raw[k], f);
+#pragma unroll
+            for (int i = 0; i < VEC; i += 4) {
+                const float4 a = *reinterpret_cast<const float4 *>(scale + (size_t)c * VEC + i);
+                const float4 b = *reinterpret_cast<const float4 *>(shift + (size_t)c * VEC + i);
+                sc[i] = a.x; sc[i + 1] = a.y; sc[i + 2] = a.z; sc[i + 3] = a.w;
+                sh[i] = b.x; sh[i + 1] = b.y; sh[i + 2] = b.z; sh[i + 3] = b.w;
+            }
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) f[i] = (f[i] - mean) * rstd * (1.0f + sc[i]) + sh[i];
+            orow[c] = pack16B<T>(f);
+        }
+    }
+}
+
+template <typename T, int KMAX>
+static cudaError_t ln_mod_cta(const T *x, const float *shift, const float *scale, T *out, int M, int d, float eps,
+                              const uint8_t *skip, cudaStream_t st) {
+    return launch_pdl(ln_mod_cta_kernel<T, KMAX>, dim3(M), dim3(LN_CTA), 0, st, x, shift, scale, out, M, d, eps,
+                      skip);
+}
+
 static int n_sm_elem() {
     static int n = 0;
     if (n == 0) {
@@ -218,12 +336,15 @@ cudaError_t ln_mod(const T *x, const float *shift, const float *scale, T *out, i
         const int want = (M + 7) / 8, cap = 2 * n_sm_elem();
         return launch_pdl(ln_mod_row_kernel<T>, dim3(want < cap ? want : cap), dim3(256), 0, st, x, shift, scale, out, M, d, eps, skip);
     }
+    // one CTA per row: 16-byte vectors per thread
+    const int per = (d / (16 / (int)sizeof(T)) + LN_CTA - 1) / LN_CTA;
+    if (per <= 2) return ln_mod_cta<T, 2>(x, shift, scale, out, M, d, eps, skip, st);
+    if (per <= 4) return ln_mod_cta<T, 4>(x, shift, scale, out, M, d, eps, skip, st);
+    if (per <= 5) return ln_mod_cta<T, 5>(x, shift, scale, out, M, d, eps, skip, st);
+    if (per <= 6) return ln_mod_cta<T, 6>(x, shift, scale, out, M, d, eps, skip, st);
+    if (per <= 8) return ln_mod_cta<T, 8>(x, shift, scale, out, M, d, eps, skip, st);
+    if (per <= 12) return ln_mod_cta<T, 12>(x, shift, scale, out, M, d, eps, skip, st);
     switch ((d + 511) / 512) {
-        case 1: return ln_mod_n<T, 1>(x, shift, scale, out, M, d, eps, skip, st);
-        case 2: return ln_mod_n<T, 2>(x, shift, scale, out, M, d, eps, skip, st);
-        case 3: return ln_mod_n<T, 3>(x, shift, scale, out, M, d, eps, skip, st);
-        case 4: return ln_mod_n<T, 4>(x, shift, scale, out, M, d, eps, skip, st);
-        case 5: case 6: case 7: case 8: return ln_mod_n<T, 8>(x, shift, scale, out, M, d, eps, skip, st);
         case 9: case 10: case 11: case 12: return ln_mod_n<T, 12>(x, shift, scale, out, M, d, eps, skip, st);
         default: return cudaErrorInvalidValue;
     }
@@ -265,6 +386,57 @@ cudaError_t residual_reuse(const T *x, const T *r, T *out, long n, const uint8_t
 }
 template cudaError_t residual_reuse<float>(const float *, const float *, float *, long, const uint8_t *, int, cudaStream_t);
 template cudaError_t residual_reuse<bf16>(const bf16 *, const bf16 *, bf16 *, long, const uint8_t *, int, cudaStream_t);
+
+// -------------------------------------------------- lazy chaining (Eq. 4)
+// Before block b computes (b = n_blocks: before the head): if blocks j..b-1
+// were all skipped (and block j-1 was not), x_{b-1} has not been
+// materialised; it is x_{j-1} (buffer X[j & 1], written by block j-1 or the
+// patch embedding) plus the cached residuals of the run.  Computed here in
+// fp32 in block order, rounded once, into X[b & 1] (in place when the two are
+// the same buffer: every element is read before it is written, by the same
+// thread).  The decisions are read from the device, so one launch serves
+// every pattern; the kernel exits at once when there is nothing to add.
+template <typename T>
+__global__ void __launch_bounds__(256)
+    chain_apply_kernel(T *__restrict__ x0, T *__restrict__ x1, const T *__restrict__ rhat_t,
+                       const uint8_t *__restrict__ flags, int b, int n_blocks, long n16, long ld) {
+    pdl_wait();
+    pdl_release();
+    if (b < n_blocks && flags[b] == XC_DEC_SKIP) return;
+    if (b == 0 || flags[b - 1] != XC_DEC_SKIP) return;
+    int j = b - 1;
+    while (j > 0 && flags[j - 1] == XC_DEC_SKIP) --j;
+    const T *base = (j & 1) ? x1 : x0;
+    T *out = (b & 1) ? x1 : x0;
+    const long stride = (long)gridDim.x * blockDim.x;
+    for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n16; i += stride) {
+        float a[16];
+        load16<T>(base + i * 16, a);
+        for (int k = j; k < b; ++k) {
+            float r[16];
+            load16<T>(rhat_t + (size_t)k * ld + i * 16, r);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) a[e] += r[e];
+        }
+        store16<T>(out + i * 16, a);
+    }
+}
+
+template <typename T>
+cudaError_t chain_apply(T *x0, T *x1, const T *rhat_t, const uint8_t *flags, int b, int n_blocks, long ld,
+                        int n_sm, cudaStream_t st) {
+    const long n16 = ld / 16;
+    long blocks = (n16 + 255) / 256;
+    const long cap = (long)n_sm * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    return launch_pdl(chain_apply_kernel<T>, dim3((unsigned)blocks), dim3(256), 0, st, x0, x1, rhat_t, flags, b,
+                      n_blocks, n16, ld);
+}
+template cudaError_t chain_apply<float>(float *, float *, const float *, const uint8_t *, int, int, long, int,
+                                        cudaStream_t);
+template cudaError_t chain_apply<bf16>(bf16 *, bf16 *, const bf16 *, const uint8_t *, int, int, long, int,
+                                       cudaStream_t);
 
 // -------------------------------------------------------------- Euler step
 __global__ void euler_kernel(float *__restrict__ x, const float *__restrict__ v, float ds, long n) {

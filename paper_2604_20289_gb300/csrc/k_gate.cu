@@ -11,38 +11,48 @@
 // spatial entry (Eq. 6).  Decision Eq. 7 with tau_cos = max(tau_floor, ema -
 // m) (Eq. 9), EMA update (Eq. 8) and the consecutive-skip cap (Section 2.5 (4)).
 //
-// Grid: one CTA (256 threads) per (camera c, 64-column slice s, row block r);
-// the row blocks split each camera's tokens so that the grid fills every SM
-// (about eight CTAs per SM).  A CTA streams its rows of its slice once
-// (16-byte loads, 8 rows in flight per thread) into 64 column sums, and takes
-// every R-th row of the camera's spatial sample in its slice.  Three folds
-// follow, each in a fixed order (deterministic, no spin-wait anywhere):
-//   1. the last CTA of a (camera, slice) to arrive (per-slice ticket) adds the
-//      R column-sum partials in row-block order, giving the slice of the
-//      camera's mean, and its global-channel products;
-//   2. every CTA writes 8 partial metrics (its sample products; the slice
-//      folder also its global-channel products);
-//   3. the last CTA of the grid (global ticket) adds the partials of each
+// Grid: one CTA (256 threads) per (camera c, column slice s, row block r).
+// The slice width (64 to 512 columns) and the row blocks per camera are
+// chosen so that the grid comes closest to one full wave of resident CTAs
+// (four per SM), and the R row blocks of one (camera, slice) form a
+// thread-block cluster.  A CTA
+// streams its rows of its slice once (16-byte streaming loads, batches of 8
+// rows in flight per thread) into column sums, and takes every R-th row of
+// the camera's spatial sample in its slice.  Two folds follow, each in a
+// fixed order (deterministic; the only waits are one cluster barrier, which
+// every CTA of the cluster reaches, and no spin-wait):
+//   1. every rank stores its column sums into rank 0's shared memory
+//      (distributed shared memory); after the cluster barrier rank 0 adds
+//      them in rank order, giving the slice of the camera's mean, and its
+//      global-channel products; every CTA then writes 8 partial metrics (its
+//      sample products, rank 0 also the global-channel products);
+//   2. the last CTA of the grid (global ticket) adds the partials of each
 //      view group in CTA order and thread 0 applies Eq. 5-9 (metrics in fp32,
 //      EMA state in fp64), writing the decision byte every later kernel of the
 //      block reads.
-// Every ticket is left at zero for the next launch.  The cached fingerprint
+// The ticket is left at zero for the next launch.  The cached fingerprint
 // is double-buffered per (t, b): the current fingerprint goes to the inactive
 // half, which becomes active when the block recomputes.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
 
+#include <cooperative_groups.h>
+
 #include "xc_kernels.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace xc {
 
-constexpr int GATE_CW = 64;          // columns per CTA
+constexpr int GATE_MAX_CW = 512;     // widest column slice of one CTA (64, 128, 256 or 512 columns)
 constexpr int GATE_THREADS = 256;
-constexpr int GATE_UNROLL = 8;       // rows in flight per thread
+constexpr int GATE_UNROLL = 8;       // rows in flight per thread (one unguarded batch)
 constexpr int GATE_PARTS = 8;        // dot, |cur|^2, |prev|^2, max|diff|, sum|prev| (spatial); dot, |cur|^2, |prev|^2 (global)
-constexpr int GATE_CTAS_PER_SM = 8;  // target CTAs per SM of the row split
+constexpr int GATE_CTAS_PER_SM = 4;  // target CTAs per SM of the row split
+constexpr int GATE_MAX_CLUSTER = 8;  // row blocks of one (camera, slice): one cluster (portable size)
 
 // Cosine of one entry from its dot product and squared norms (Eq. 5):
 // both norms < 1e-12 -> 1, exactly one -> 0, NaN -> 0.
@@ -54,21 +64,18 @@ __device__ __forceinline__ float cos_rule_f(float dot, float n1sq, float n2sq) {
     return dot / (a * b);
 }
 
+// Adds one 16-byte vector to running fp32 pair sums: bf16 elements are
+// widened by placing their 16 bits in the high half of an fp32 word (exact).
 template <typename T>
-__device__ __forceinline__ void add_vec16(float *acc, const uint4 u) {
+__device__ __forceinline__ void add_pairs(float2 (&acc)[16 / sizeof(T) / 2], const uint4 u) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
     if constexpr (sizeof(T) == 2) {
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[j]));
-            acc[2 * j] += f.x;
-            acc[2 * j + 1] += f.y;
-        }
+        for (int j = 0; j < 4; ++j)
+            acc[j] = __fadd2_rn(acc[j], make_float2(__uint_as_float(w[j] << 16), __uint_as_float(w[j] & 0xFFFF0000u)));
     } else {
-        acc[0] += __uint_as_float(u.x);
-        acc[1] += __uint_as_float(u.y);
-        acc[2] += __uint_as_float(u.z);
-        acc[3] += __uint_as_float(u.w);
+        acc[0] = __fadd2_rn(acc[0], make_float2(__uint_as_float(w[0]), __uint_as_float(w[1])));
+        acc[1] = __fadd2_rn(acc[1], make_float2(__uint_as_float(w[2]), __uint_as_float(w[3])));
     }
 }
 
@@ -96,82 +103,125 @@ __device__ __forceinline__ void cta_fold8(float (&v)[GATE_PARTS], float (*wpart)
     }
 }
 
+// Column sums of rows [rb0, rb1) (tokens from ctok0) over columns [col0,
+// col0 + cw) of x [.][d]: cw / VEC threads cover a row (16 bytes each),
+// the rest of the CTA takes further rows; full batches of GATE_UNROLL rows go
+// out unguarded (32-bit byte offsets), the sums are kept as fp32 pairs (bf16
+// halves widened by shifts, packed adds).  The CTA's sums land in cluster
+// rank 0's call[r] (distributed shared memory).
 template <typename T>
-__global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
+__device__ __forceinline__ void slice_colsums(const T *x, size_t ctok0, int d, int col0, int cw, int rb0, int rb1,
+                                              int r, float *red, float (*call)[GATE_MAX_CW],
+                                              cg::cluster_group &cluster) {
+    constexpr int VEC = 16 / sizeof(T);
+    const int tid = threadIdx.x;
+    const int TPR = cw / VEC, RPAR = GATE_THREADS / TPR;
+    const int ty = tid / TPR, tx = tid % TPR;
+    const int first = rb0 + ty;
+    const int n = first < rb1 ? (rb1 - first + RPAR - 1) / RPAR : 0;     // rows of this thread
+    const char *p = reinterpret_cast<const char *>(x + (ctok0 + first) * d + col0 + tx * VEC);
+    const uint32_t stride = (uint32_t)RPAR * (uint32_t)d * (uint32_t)sizeof(T);
+    float2 acc2[VEC / 2];
+#pragma unroll
+    for (int i = 0; i < VEC / 2; ++i) acc2[i] = make_float2(0.0f, 0.0f);
+    int i = 0;
+    for (; i + GATE_UNROLL <= n; i += GATE_UNROLL) {
+        uint4 u[GATE_UNROLL];
+#pragma unroll
+        for (int k = 0; k < GATE_UNROLL; ++k) u[k] = __ldcs(reinterpret_cast<const uint4 *>(p + k * stride));
+        p += GATE_UNROLL * stride;
+#pragma unroll
+        for (int k = 0; k < GATE_UNROLL; ++k) add_pairs<T>(acc2, u[k]);
+    }
+    for (; i < n; ++i) {
+        add_pairs<T>(acc2, __ldcs(reinterpret_cast<const uint4 *>(p)));
+        p += stride;
+    }
+#pragma unroll
+    for (int i2 = 0; i2 < VEC / 2; ++i2) {
+        red[ty * cw + tx * VEC + 2 * i2] = acc2[i2].x;
+        red[ty * cw + tx * VEC + 2 * i2 + 1] = acc2[i2].y;
+    }
+    __syncthreads();
+    for (int j = tid; j < cw; j += GATE_THREADS) {
+        float sum = 0.0f;
+        for (int t = 0; t < RPAR; ++t) sum += red[t * cw + j];
+        *cluster.map_shared_rank(&call[r][j], 0) = sum;
+    }
+}
+
+// Camera c's view group: first token, first camera, tokens per camera,
+// first sample row and sample rows per camera (unrolled compare chain:
+// constant parameter indices).
+struct CamGroup {
+    int tok0, cam0, npc, fp0, kfp;
+};
+__device__ __forceinline__ CamGroup cam_group(const GateArgs &g, int c) {
+    CamGroup q0{g.g_tok0[0], g.g_cam0[0], g.g_npc[0], g.g_fp0[0], g.g_kfp[0]};
+#pragma unroll
+    for (int q = 1; q < XC_MAX_GROUPS; ++q)
+        if (q < g.n_groups && c >= g.g_cam0[q]) q0 = CamGroup{g.g_tok0[q], g.g_cam0[q], g.g_npc[q], g.g_fp0[q], g.g_kfp[q]};
+    return q0;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(GATE_THREADS, GATE_CTAS_PER_SM) gate_kernel(const GateArgs g) {
     pdl_wait();
     pdl_release();
     constexpr int VEC = 16 / sizeof(T);
-    constexpr int TPR = GATE_CW / VEC;          // threads per row
-    constexpr int RPAR = GATE_THREADS / TPR;    // rows per sweep
     constexpr int NW = GATE_THREADS / 32;
-    __shared__ float red[RPAR * GATE_CW];
+    __shared__ float red[GATE_THREADS * VEC];
     __shared__ float wpart[NW][GATE_PARTS];
+    __shared__ float call[GATE_MAX_CLUSTER][GATE_MAX_CW];   // column sums of every rank (rank 0's copy is used)
     __shared__ int s_last;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int blk = blockIdx.x;
-    const int R = g.R;
+    const int R = g.R, cw = g.cw;
     const int r = blk % R, cs = blk / R;
     const int c = cs / g.n_slices, s = cs % g.n_slices;
     const int d = g.d;
-    // camera c's group (unrolled compare chain: constant parameter indices)
-    int tok0 = g.g_tok0[0], cam0 = g.g_cam0[0], npc = g.g_npc[0], fp0 = g.g_fp0[0], kfp = g.g_kfp[0];
-#pragma unroll
-    for (int q = 1; q < XC_MAX_GROUPS; ++q)
-        if (q < g.n_groups && c >= g.g_cam0[q]) {
-            tok0 = g.g_tok0[q];
-            cam0 = g.g_cam0[q];
-            npc = g.g_npc[q];
-            fp0 = g.g_fp0[q];
-            kfp = g.g_kfp[q];
-        }
-    const size_t ctok0 = (size_t)tok0 + (size_t)(c - cam0) * npc;   // camera c's first token
-    const int crow0 = fp0 + (c - cam0) * kfp;                        // and first sample row
-    const int col0 = s * GATE_CW;
+    const CamGroup cg0 = cam_group(g, c);
+    const int npc = cg0.npc, kfp = cg0.kfp;
+    const size_t ctok0 = (size_t)cg0.tok0 + (size_t)(c - cg0.cam0) * npc;   // camera c's first token
+    const int crow0 = cg0.fp0 + (c - cg0.cam0) * kfp;                        // and first sample row
+    const int col0 = s * cw;
     const T *x = reinterpret_cast<const T *>(g.x);
     const int active = g.cell->active;
     const int n_sp = g.n_rows * d;
     const int n_all = n_sp + g.V * d;
     const float *phi_prev = g.phi + (size_t)active * n_all;
     float *phi_next = g.phi + (size_t)(active ^ 1) * n_all;
+    cg::cluster_group cluster = cg::this_cluster();
 
-    // 1. column sums of rows [rb0, rb1) of camera c, columns [col0, col0 + 64)
-    {
-        const int rb0 = r * g.rows_per;
-        const int rb1 = min(npc, rb0 + g.rows_per);
-        float acc[VEC];
-#pragma unroll
-        for (int i = 0; i < VEC; ++i) acc[i] = 0.0f;
-        const int ty = tid / TPR, tx = tid % TPR;
-        const T *base = x + ctok0 * d + col0 + tx * VEC;
-        for (int row = rb0 + ty; row < rb1; row += GATE_UNROLL * RPAR) {
-            uint4 u[GATE_UNROLL];
-#pragma unroll
-            for (int k = 0; k < GATE_UNROLL; ++k)
-                u[k] = row + k * RPAR < rb1 ? *reinterpret_cast<const uint4 *>(base + (size_t)(row + k * RPAR) * d)
-                                            : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-            for (int k = 0; k < GATE_UNROLL; ++k) add_vec16<T>(acc, u[k]);
-        }
-#pragma unroll
-        for (int i = 0; i < VEC; ++i) red[ty * GATE_CW + tx * VEC + i] = acc[i];
-    }
-    __syncthreads();
-    if (tid < GATE_CW) {
-        float sum = 0.0f;
-        for (int t = 0; t < RPAR; ++t) sum += red[t * GATE_CW + tid];
-        g.colsum[(size_t)blk * GATE_CW + tid] = sum;
-    }
+    // 1. column sums of rows [rb0, rb1) of camera c, columns [col0, col0 + cw),
+    //    into rank 0's shared memory -- unless the previous block was skipped
+    //    under lazy chaining (Section 2.2, reading c27): then the input is not
+    //    materialised and its per-camera mean is the running chained mean
+    const bool chained = g.chain && g.prev_flag != nullptr && *g.prev_flag == XC_DEC_SKIP;
+    if (!chained)
+        slice_colsums<T>(x, ctok0, d, col0, cw, r * g.rows_per, min(npc, r * g.rows_per + g.rows_per), r, red, call,
+                         cluster);
 
     float p[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     // 2. sample rows r, r + R, ... of camera c in this slice
     {
         const int n_mine = r < kfp ? (kfp - r + R - 1) / R : 0;
-        for (int it = tid; it < n_mine * GATE_CW; it += GATE_THREADS) {
-            const int i = r + (it / GATE_CW) * R, j = it % GATE_CW;
+        for (int it = tid; it < n_mine * cw; it += GATE_THREADS) {
+            const int i = r + (it / cw) * R, j = it % cw;
             const int row = g.fp_rows[crow0 + i];
             const size_t e = ((size_t)crow0 + i) * d + col0 + j;
-            const float cur = to_f(x[(size_t)row * d + col0 + j]);
+            float cur;
+            if (chained) {
+                // chained input on the sampled rows: running fp32 sum of the last
+                // materialised rows and the pending residuals, rounded once
+                const float sum = g.csp_in[e] + to_f(reinterpret_cast<const T *>(g.rhat_prev)[(size_t)row * d + col0 + j]);
+                g.csp_out[e] = sum;
+                cur = round_to<T>(sum);
+            } else {
+                cur = to_f(x[(size_t)row * d + col0 + j]);
+                if (g.chain) g.csp_out[e] = cur;
+            }
             const float prev = phi_prev[e];
             phi_next[e] = cur;
             p[0] = fmaf(cur, prev, p[0]);
@@ -182,39 +232,47 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         }
     }
 
-    // 3. per-slice ticket: the last row block of (c, s) folds the column sums
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) s_last = atomicAdd(&g.slice_ticket[cs], 1u) == (unsigned)(R - 1);
-    __syncthreads();
-    if (s_last) {
-        __threadfence();
-        if (tid < GATE_CW) {
-            float sum = 0.0f;
-            for (int rr = 0; rr < R; ++rr) sum += __ldcg(&g.colsum[((size_t)cs * R + rr) * GATE_CW + tid]);
-            const float mean = sum / (float)npc;
-            const size_t e = (size_t)n_sp + (size_t)c * d + col0 + tid;
+    // 3. the R CTAs of (c, s) form one thread-block cluster; after the
+    //    cluster barrier rank 0 holds every rank's column sums and adds them
+    //    in rank order (the other ranks do not touch shared memory again)
+    cluster.sync();
+    if (r == 0) {
+        for (int j = tid; j < cw; j += GATE_THREADS) {
+            const size_t cm = (size_t)c * d + col0 + j;
+            float mean;
+            if (chained) {
+                mean = g.cgm_in[cm] + g.rmean_prev[cm];      // mean(x_{j-1}) + sum of the residuals' means
+            } else {
+                float sum = call[0][j];
+                for (int rr = 1; rr < R; ++rr) sum += call[rr][j];
+                mean = sum / (float)npc;
+            }
+            if (g.chain) g.cgm_out[cm] = mean;
+            const size_t e = (size_t)n_sp + cm;
             const float prev = phi_prev[e];
             phi_next[e] = mean;
-            p[5] = mean * prev;
-            p[6] = mean * mean;
-            p[7] = prev * prev;
+            p[5] = fmaf(mean, prev, p[5]);
+            p[6] = fmaf(mean, mean, p[6]);
+            p[7] = fmaf(prev, prev, p[7]);
         }
-        if (tid == 0) g.slice_ticket[cs] = 0u;
     }
     cta_fold8(p, wpart, lane, warp, NW);
     if (tid == 0) {
-#pragma unroll
-        for (int k = 0; k < GATE_PARTS; ++k) g.part[(size_t)blk * GATE_PARTS + k] = p[k];
+        float4 *dst = reinterpret_cast<float4 *>(g.part + (size_t)blk * GATE_PARTS);
+        dst[0] = make_float4(p[0], p[1], p[2], p[3]);
+        dst[1] = make_float4(p[4], p[5], p[6], p[7]);
     }
 
-    // 4. global ticket: the last CTA combines all partials and decides
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) s_last = atomicAdd(g.ticket, 1u) == (unsigned)(gridDim.x - 1);
+    // 4. global ticket: the last CTA combines all partials and decides.  The
+    //    partials are written by thread 0, which fences (release) before its
+    //    ticket; the last CTA's thread 0 fences (acquire) before the barrier.
+    if (tid == 0) {
+        __threadfence();
+        s_last = atomicAdd(g.ticket, 1u) == (unsigned)(gridDim.x - 1);
+        if (s_last) __threadfence();
+    }
     __syncthreads();
     if (!s_last) return;
-    __threadfence();
     // Per view group: fold the partials of the group's CTAs (cameras
     // [g_cam0[q], g_cam0[q + 1]), every slice and row block) in CTA order;
     // thread 0 keeps the running min of the cosines and max of the deviations.
@@ -224,12 +282,18 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
         if (q >= g.n_groups) break;
         const int b0 = g.g_cam0[q] * g.n_slices * R, b1 = g.g_cam0[q + 1] * g.n_slices * R;
         float v[GATE_PARTS] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
         for (int b = b0 + tid; b < b1; b += GATE_THREADS) {
-#pragma unroll
-            for (int k = 0; k < GATE_PARTS; ++k) {
-                const float w = __ldcg(&g.part[(size_t)b * GATE_PARTS + k]);
-                v[k] = k == 3 ? fmaxf(v[k], w) : v[k] + w;
-            }
+            const float4 lo = __ldcg(reinterpret_cast<const float4 *>(g.part + (size_t)b * GATE_PARTS));
+            const float4 hi = __ldcg(reinterpret_cast<const float4 *>(g.part + (size_t)b * GATE_PARTS + 4));
+            v[0] += lo.x;
+            v[1] += lo.y;
+            v[2] += lo.z;
+            v[3] = fmaxf(v[3], lo.w);
+            v[4] += hi.x;
+            v[5] += hi.y;
+            v[6] += hi.z;
+            v[7] += hi.w;
         }
         cta_fold8(v, wpart, lane, warp, NW);
         if (tid == 0) {
@@ -289,45 +353,114 @@ __global__ void __launch_bounds__(GATE_THREADS) gate_kernel(const GateArgs g) {
     *g.flag = dec;
 }
 
+// Per-camera column means of a cached residual r_hat [L][d] (lazy chaining,
+// reading c27): the same grid, streaming and cluster fold as the gate's
+// global channel; rank 0 writes mean[c][col].  Runs after the block's FFN
+// down-projection and exits at once unless the block computed.
+template <typename T>
+__global__ void __launch_bounds__(GATE_THREADS, GATE_CTAS_PER_SM) camera_mean_kernel(const GateArgs g) {
+    pdl_wait();
+    pdl_release();
+    constexpr int VEC = 16 / sizeof(T);
+    __shared__ float red[GATE_THREADS * VEC];
+    __shared__ float call[GATE_MAX_CLUSTER][GATE_MAX_CW];
+    if (g.flag != nullptr && *g.flag == XC_DEC_SKIP) return;     // uniform over the grid
+    const int blk = blockIdx.x, R = g.R, cw = g.cw;
+    const int r = blk % R, cs = blk / R;
+    const int c = cs / g.n_slices, s = cs % g.n_slices;
+    const CamGroup cg0 = cam_group(g, c);
+    const size_t ctok0 = (size_t)cg0.tok0 + (size_t)(c - cg0.cam0) * cg0.npc;
+    cg::cluster_group cluster = cg::this_cluster();
+    slice_colsums<T>(reinterpret_cast<const T *>(g.x), ctok0, g.d, s * cw, cw, r * g.rows_per,
+                     min(cg0.npc, r * g.rows_per + g.rows_per), r, red, call, cluster);
+    cluster.sync();
+    if (r == 0)
+        for (int j = threadIdx.x; j < cw; j += GATE_THREADS) {
+            float sum = call[0][j];
+            for (int rr = 1; rr < R; ++rr) sum += call[rr][j];
+            g.cam_mean_out[(size_t)c * g.d + s * cw + j] = sum / (float)cg0.npc;
+        }
+}
+
 static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // Grid and scratch of one gate launch for V cameras of at most max_npc tokens
-// each, d columns, on a device with n_sm SMs.  Scratch: 8 fp32 partials per
-// CTA, 64 fp32 column sums per CTA, then V * n_slices + 1 32-bit tickets
-// (zero before the first launch; every launch leaves them zero).
+// each, d columns, on a device with n_sm SMs.  The row blocks R of one
+// (camera, slice) form a thread-block cluster, so R <= GATE_MAX_CLUSTER.
+// Scratch: 8 fp32 partials per CTA, then one 32-bit ticket (zero before the
+// first launch; every launch leaves it zero).
 GateGeom gate_geometry(int V, int max_npc, int d, int n_sm) {
     GateGeom gg;
-    gg.n_slices = d / GATE_CW;
-    const int cs = V * gg.n_slices;
-    const int want = (GATE_CTAS_PER_SM * (n_sm > 0 ? n_sm : 1)) / cs;
-    const int most = (max_npc + 31) / 32;                  // at least 32 rows per row block
-    gg.R = want < 1 ? 1 : (want > most ? most : want);
+    const int target = GATE_CTAS_PER_SM * (n_sm > 0 ? n_sm : 1);   // resident CTA slots
+    const int most = (max_npc + 63) / 64;                  // at least 64 rows per row block
+    // the (slice width, row blocks) whose grid comes closest to one full wave
+    // of resident CTAs -- every SM then streams about the same share -- the
+    // wider slice (longer contiguous runs) on a tie
+    int best_n = -1;
+    gg.cw = 64;
+    gg.R = 1;
+    for (int cw = GATE_MAX_CW; cw >= 64; cw /= 2) {
+        if (d % cw != 0) continue;
+        const int cs = V * (d / cw);
+        int R = target / cs;
+        if (R > most) R = most;
+        if (R > GATE_MAX_CLUSTER) R = GATE_MAX_CLUSTER;
+        if (R < 1) R = 1;
+        if (cs * R > best_n) {
+            best_n = cs * R;
+            gg.cw = cw;
+            gg.R = R;
+        }
+    }
+    gg.n_slices = d / gg.cw;
     gg.rows_per = (max_npc + gg.R - 1) / gg.R;
-    gg.n_ctas = cs * gg.R;
-    gg.colsum_off = align256((size_t)gg.n_ctas * GATE_PARTS * sizeof(float));
-    gg.tickets_off = gg.colsum_off + align256((size_t)gg.n_ctas * GATE_CW * sizeof(float));
-    gg.n_tickets = cs + 1;
-    gg.total = gg.tickets_off + align256((size_t)gg.n_tickets * sizeof(unsigned));
+    gg.n_ctas = V * gg.n_slices * gg.R;
+    gg.tickets_off = align256((size_t)gg.n_ctas * GATE_PARTS * sizeof(float));
+    gg.n_tickets = 1;
+    gg.total = gg.tickets_off + 256;
     return gg;
 }
 
 void gate_bind_scratch(GateArgs &g, const GateGeom &gg, void *scratch) {
     char *w = reinterpret_cast<char *>(scratch);
     g.n_slices = gg.n_slices;
+    g.cw = gg.cw;
     g.R = gg.R;
     g.rows_per = gg.rows_per;
     g.part = reinterpret_cast<float *>(w);
-    g.colsum = reinterpret_cast<float *>(w + gg.colsum_off);
-    g.slice_ticket = reinterpret_cast<unsigned *>(w + gg.tickets_off);
-    g.ticket = g.slice_ticket + gg.n_tickets - 1;
+    g.ticket = reinterpret_cast<unsigned *>(w + gg.tickets_off);
 }
 
 template <typename T>
+static cudaError_t cluster_launch(void (*kern)(GateArgs), const GateArgs &g, cudaStream_t st) {
+    if (g.R < 1 || g.R > GATE_MAX_CLUSTER) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.V * g.n_slices * g.R);
+    cfg.blockDim = dim3(GATE_THREADS);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)g.R;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, kern, g);
+}
+template <typename T>
 cudaError_t gate_launch(const GateArgs &g, cudaStream_t st) {
-    return launch_pdl(gate_kernel<T>, dim3(g.V * g.n_slices * g.R), dim3(GATE_THREADS), 0, st, g);
+    return cluster_launch<T>(gate_kernel<T>, g, st);
+}
+template <typename T>
+cudaError_t camera_mean_launch(const GateArgs &g, cudaStream_t st) {
+    return cluster_launch<T>(camera_mean_kernel<T>, g, st);
 }
 template cudaError_t gate_launch<float>(const GateArgs &, cudaStream_t);
 template cudaError_t gate_launch<bf16>(const GateArgs &, cudaStream_t);
+template cudaError_t camera_mean_launch<float>(const GateArgs &, cudaStream_t);
+template cudaError_t camera_mean_launch<bf16>(const GateArgs &, cudaStream_t);
 
 static int current_sm_count() {
     int dev = 0, n = 0;
@@ -463,7 +596,7 @@ xc_status xc_op_gate(int dtype, int n_cams, int tokens_per_cam, int d, const voi
     }
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     xc::gate_bind_scratch(g, gg, workspace);
-    cudaError_t e = cudaMemsetAsync(g.slice_ticket, 0, gg.n_tickets * sizeof(unsigned), s);
+    cudaError_t e = cudaMemsetAsync(g.ticket, 0, sizeof(unsigned), s);
     if (e == cudaSuccess) e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, s) : xc::gate_launch<float>(g, s);
     if (e != cudaSuccess) {
         snprintf(msg, sizeof msg, "xc_op_gate: %s", cudaGetErrorString(e));
@@ -504,7 +637,7 @@ xc_status xc_op_gate_static(int dtype, int n_cams, int tokens_per_cam, int d, co
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     xc::gate_bind_scratch(g, gg, scratch);
     // the tickets must start at zero; partials and column sums are overwritten
-    cudaError_t e = cudaMemsetAsync(g.slice_ticket, 0, gg.n_tickets * sizeof(unsigned), s);
+    cudaError_t e = cudaMemsetAsync(g.ticket, 0, sizeof(unsigned), s);
     if (e == cudaSuccess) e = dtype == XC_BF16 ? xc::gate_launch<xc::bf16>(g, s) : xc::gate_launch<float>(g, s);
     if (e != cudaSuccess) {
         snprintf(msg, sizeof msg, "xc_op_gate_static: %s", cudaGetErrorString(e));

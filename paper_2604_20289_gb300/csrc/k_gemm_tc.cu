@@ -125,6 +125,24 @@ __device__ __forceinline__ void write_row32(uint8_t *blk, int r, const float (&v
     }
 }
 
+// Persistent tile order: tile t -> (m block, n block).  Tiles go in
+// super-rows of GEMM_GROUP_M m blocks with m varying fastest inside a
+// super-row, so the tiles in flight at one time (one per SM) share
+// GEMM_GROUP_M row blocks of A and a few column blocks of B -- an
+// L2-resident working set -- instead of all of B streaming through L2 for
+// every row of m blocks (row-major order re-read B from DRAM once per 2-3
+// m-block rows on the large-N projections).
+constexpr int GEMM_GROUP_M = 16;
+__device__ __forceinline__ void tile_mn(int tile, int tiles_m, int tiles_n, int &mb, int &nb) {
+    const int per = GEMM_GROUP_M * tiles_n;
+    const int grp = tile / per;
+    const int first = grp * GEMM_GROUP_M;
+    const int gm = min(GEMM_GROUP_M, tiles_m - first);
+    const int loc = tile - grp * per;
+    mb = first + loc % gm;
+    nb = loc / gm;
+}
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(320, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -145,7 +163,8 @@ __global__ void __launch_bounds__(320, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int KT = K / GEMM_BK;
     const int tiles_n = ep.N / BN;
-    const int n_tiles = ((ep.M + GEMM_BM - 1) / GEMM_BM) * tiles_n;
+    const int tiles_m = (ep.M + GEMM_BM - 1) / GEMM_BM;
+    const int n_tiles = tiles_m * tiles_n;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < G::STAGES; ++s) {
@@ -170,7 +189,9 @@ __global__ void __launch_bounds__(320, 1)
             int it = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x) {
-                const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
+                int mb, nb;
+                tile_mn(tile, tiles_m, tiles_n, mb, nb);
+                const int m0 = mb * GEMM_BM, n0 = nb * BN;
                 for (int kt = 0; kt < KT; ++kt, ++it) {
                     const int s = it % G::STAGES;
                     const uint32_t ph = (it / G::STAGES) & 1;
@@ -259,7 +280,9 @@ __global__ void __launch_bounds__(320, 1)
         for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++local) {
             const int buf = local & 1;
             const uint32_t use = (uint32_t)(local >> 1);
-            const int m0 = (tile / tiles_n) * GEMM_BM, n0 = (tile % tiles_n) * BN;
+            int mb, nb;
+            tile_mn(tile, tiles_m, tiles_n, mb, nb);
+            const int m0 = mb * GEMM_BM, n0 = nb * BN;
             const int row = m0 + q * 32 + lane;
             if constexpr (SHARED) {
                 if (lane == 0) bulk_wait_read<0>();

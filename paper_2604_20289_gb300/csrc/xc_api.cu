@@ -189,6 +189,12 @@ struct xc_ctx {
     float *h_stats;                            // pinned [3][B]
     int *d_err;
 
+    // lazy residual chaining: per-camera means of every cached residual
+    // [S][B][V][d]; running chained sample rows [2][n_rows][d] and means
+    // [2][V][d] of the current pass; the chain setting of the last pass
+    float *rmean, *chain_sp, *chain_gm;
+    int chain_last;
+
     // gate scratch (grid and layout in g_geom)
     GateGeom g_geom;
     char *g_scratch;
@@ -257,6 +263,7 @@ bool xc::gate_ok(const xc_gate_params *p, int B, char *why, size_t n) {
     if (p->fp_tokens < 1) return bad("fp_tokens < 1");
     if (p->fp_refresh != 0 && p->fp_refresh != 1) return bad("fp_refresh must be 0 or 1");
     if (p->fp_linear != 0 && p->fp_linear != 1) return bad("fp_linear must be 0 or 1");
+    if (p->chain != 0 && p->chain != 1) return bad("chain must be 0 or 1");
     (void)B;
     return true;
 }
@@ -373,7 +380,7 @@ void ensure_fp(xc_ctx *ctx, int K, int linear) {
         CK(cudaStreamSynchronize(ctx->st));
         drop_graphs(ctx);                        // the captured passes point at the old buffers
         for (auto it = ctx->allocs.begin(); it != ctx->allocs.end();) {
-            if (*it == ctx->fp_rows || *it == ctx->phi) {
+            if (*it == ctx->fp_rows || *it == ctx->phi || *it == ctx->chain_sp) {
                 cudaFree(*it);
                 it = ctx->allocs.erase(it);
             } else {
@@ -384,6 +391,7 @@ void ensure_fp(xc_ctx *ctx, int K, int linear) {
     ctx->fp_rows = dalloc<int>(ctx, rows.size() * sizeof(int));
     CK(cudaMemcpy(ctx->fp_rows, rows.data(), rows.size() * sizeof(int), cudaMemcpyHostToDevice));
     ctx->phi = dalloc<float>(ctx, (size_t)ctx->S * ctx->B * 2 * n_all * sizeof(float));
+    ctx->chain_sp = dalloc<float>(ctx, 2 * rows.size() * (size_t)ctx->d * sizeof(float));
     CK(cudaMemsetAsync(ctx->phi, 0, (size_t)ctx->S * ctx->B * 2 * n_all * sizeof(float), ctx->st));
     CK(cudaMemsetAsync(ctx->cells, 0, (size_t)ctx->S * ctx->B * sizeof(GateCell), ctx->st));
     CK(cudaMemsetAsync(ctx->phi_act, 0, (size_t)ctx->S * ctx->B * 16 * sizeof(float), ctx->st));
@@ -571,6 +579,10 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
 
     const bool gating = p.enabled != 0 && !kv;
     const bool eval_mode = eval_pass(ctx, p, t);
+    // lazy residual chaining (reading c27); a block trace needs every block's
+    // output written, so traced passes do not chain
+    const bool chain = gating && p.chain != 0 && ctx->trace == nullptr;
+    auto gated_at = [&](int b) { return gating && b >= p.front_anchors && b < B - p.back_anchors; };
     T *x1 = reinterpret_cast<T *>(ctx->x1);
     T *hb = reinterpret_cast<T *>(ctx->hbuf);
     T *qb = reinterpret_cast<T *>(ctx->q);
@@ -580,7 +592,7 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
     for (int b = 0; b < B; ++b) {
         T *xin = X[b & 1], *xout = X[(b + 1) & 1];
         const uint8_t *flag = ctx->flags + b;
-        const bool gated = gating && b >= p.front_anchors && b < B - p.back_anchors;
+        const bool gated = gated_at(b);
         const float *mb = ctx->mods + (size_t)b * 6 * d;   // shift1 scale1 gate1 shift2 scale2 gate2
         T *rk = reinterpret_cast<T *>(ctx->ring_k) + ((size_t)b * ctx->Wkv + slot) * Ld;
         T *rv = reinterpret_cast<T *>(ctx->ring_v) + ((size_t)b * ctx->Wkv + slot) * Ld;
@@ -626,8 +638,24 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             g.d_max = ctx->d_max + b;
             g.tau_out = ctx->tau + b;
             gate_bind_scratch(g, ctx->g_geom, ctx->g_scratch);
+            if (chain) {
+                const size_t nsp = (size_t)ctx->n_rows * d, nm = (size_t)ctx->V * d;
+                g.chain = 1;
+                g.prev_flag = b >= 1 && gated_at(b - 1) ? ctx->flags + b - 1 : nullptr;
+                g.rhat_prev = b >= 1 ? reinterpret_cast<const T *>(ctx->rhat) + ((size_t)t * B + b - 1) * Ld : nullptr;
+                g.rmean_prev = b >= 1 ? ctx->rmean + ((size_t)t * B + b - 1) * nm : nullptr;
+                g.csp_in = ctx->chain_sp + (size_t)((b + 1) & 1) * nsp;
+                g.csp_out = ctx->chain_sp + (size_t)(b & 1) * nsp;
+                g.cgm_in = ctx->chain_gm + (size_t)((b + 1) & 1) * nm;
+                g.cgm_out = ctx->chain_gm + (size_t)(b & 1) * nm;
+            }
             LAUNCH(XC_K_GATE, b, 1, gate_launch<T>(g, st));
         }
+        // lazy chaining: write the input of block b if the blocks before it were skipped
+        if (chain && b >= 1)
+            LAUNCH(XC_K_CHAIN, b, 1,
+                   chain_apply<T>(X[0], X[1], reinterpret_cast<const T *>(ctx->rhat) + (size_t)t * B * Ld, ctx->flags,
+                                  b, B, (long)Ld, ctx->n_sm, st));
 
         // ---- recompute path (early-exits when flag[b] == skip)
         LAUNCH(XC_K_LN, b, 1, ln_mod<T>(xin, mb + 0 * d, mb + 1 * d, hb, L, d, ctx->cfg.ln_eps, flag, st));
@@ -759,12 +787,36 @@ void run_pass(xc_ctx *ctx, const float *lat_dev, const float *action, float sigm
             const float *W = reinterpret_cast<const float *>(ctx->f2_wt) + (size_t)b * d * F;
             LAUNCH(XC_K_FFN2, b, 1, gemm_simt(EPI_RESID_CACHE, ep, reinterpret_cast<const float *>(ub), W, F, flag, st));
         }
-        // ---- reuse path (Eq. 4), only when the gate chose skip
-        if (gated) LAUNCH(XC_K_REUSE, b, 1, residual_reuse<T>(xin, rh, xout, (long)Ld, flag, ctx->n_sm, st));
+        // ---- reuse path (Eq. 4), only when the gate chose skip; with lazy
+        // chaining the skipped block writes nothing, and a computed gated
+        // block records the per-camera means of its new residual
+        if (gated && !chain) LAUNCH(XC_K_REUSE, b, 1, residual_reuse<T>(xin, rh, xout, (long)Ld, flag, ctx->n_sm, st));
+        if (gated && chain) {
+            GateArgs gm;
+            memset(&gm, 0, sizeof gm);
+            gm.x = rh;
+            gm.d = d;
+            gm.V = ctx->V;
+            gm.n_groups = ctx->G;
+            for (int q = 0; q < ctx->G; ++q) {
+                gm.g_cam0[q] = ctx->g_cam0[q];
+                gm.g_tok0[q] = ctx->g_tok0[q];
+                gm.g_npc[q] = ctx->g_npc[q];
+            }
+            gm.g_cam0[ctx->G] = ctx->V;
+            gate_bind_scratch(gm, ctx->g_geom, ctx->g_scratch);
+            gm.flag = ctx->flags + b;
+            gm.cam_mean_out = ctx->rmean + ((size_t)t * B + b) * (size_t)ctx->V * d;
+            LAUNCH(XC_K_CHAIN, b, 1, camera_mean_launch<T>(gm, st));
+        }
         if (ctx->trace != nullptr)
             CK(cudaMemcpyAsync(reinterpret_cast<char *>(ctx->trace) + (size_t)b * Ld * sizeof(T), xout,
                                Ld * sizeof(T), cudaMemcpyDeviceToDevice, st));
     }
+    if (chain)
+        LAUNCH(XC_K_CHAIN, -1, 1,
+               chain_apply<T>(X[0], X[1], reinterpret_cast<const T *>(ctx->rhat) + (size_t)t * B * Ld, ctx->flags, B,
+                              B, (long)Ld, ctx->n_sm, st));
     if (!kv_tail_off)
         LAUNCH(XC_K_HEAD, -1, 1, head<T>(X[B & 1], ctx->hmod, ctx->out_w, ctx->out_b, v_dev, L, d, ctx->cfg.ln_eps, st));
     };   // body
@@ -1031,10 +1083,14 @@ xc_status xc_init(const xc_model_cfg *cfg, const xc_weights *w, void *cuda_strea
         ctx->rhat = dalloc<void>(ctx, (size_t)ctx->S * B * Ld * es);
         ctx->cells = dalloc<GateCell>(ctx, (size_t)ctx->S * B * sizeof(GateCell));
         ctx->phi_act = dalloc<float>(ctx, (size_t)ctx->S * B * 16 * sizeof(float));
+        ctx->rmean = dalloc<float>(ctx, (size_t)ctx->S * B * ctx->V * d * sizeof(float));
+        ctx->chain_gm = dalloc<float>(ctx, 2 * (size_t)ctx->V * d * sizeof(float));
+        ctx->chain_last = 0;
         ctx->fp_K = -1;
         ctx->fp_lin = 0;
         ctx->fp_rows = nullptr;
         ctx->phi = nullptr;
+        ctx->chain_sp = nullptr;
         ensure_fp(ctx, 32, 0);
 
         // per pass
@@ -1368,6 +1424,12 @@ xc_status xc_chunk_step(xc_ctx *ctx, const float *latent, const float *action, f
     const int t = kv ? 0 : step_index;
     try {
         ensure_fp(ctx, p.fp_tokens, p.fp_linear);
+        if (p.chain != 0 && ctx->chain_last == 0 && !kv) {
+            // residuals cached before chaining have no per-camera means:
+            // every gate cell starts over (the blocks recompute once)
+            CK(cudaMemsetAsync(ctx->cells, 0, (size_t)ctx->S * ctx->B * sizeof(GateCell), ctx->st));
+        }
+        if (!kv) ctx->chain_last = p.chain;
         const size_t lat_bytes = (size_t)ctx->L * ctx->C * sizeof(float);
         const float *lat_dev = latent;
         if (is_host_ptr(latent)) {

@@ -21,7 +21,7 @@ struct GateArgs {
     int n_groups, n_rows;    // n_rows: sample rows of all cameras
     int g_cam0[XC_MAX_GROUPS + 1], g_tok0[XC_MAX_GROUPS], g_npc[XC_MAX_GROUPS], g_fp0[XC_MAX_GROUPS],
         g_kfp[XC_MAX_GROUPS];
-    int n_slices;            // 64-column slices
+    int n_slices, cw;        // column slices of cw columns
     int R, rows_per;         // row blocks per camera and rows per row block: one CTA per (camera, slice, row block)
     float *phi;
     float *phi_act;
@@ -37,14 +37,24 @@ struct GateArgs {
     uint8_t *flag;
     float *s_cos, *d_max, *tau_out;
     float *part;             // scratch [V * n_slices * R][8] partial metrics
-    float *colsum;           // scratch [V * n_slices * R][64] column sums
-    unsigned *slice_ticket;  // scratch [V * n_slices], zero before the launch (left zero)
     unsigned *ticket;        // scratch, zero before the launch (left zero)
+    // lazy residual chaining (chain = 1): when *prev_flag (the previous
+    // block's decision) is skip, the input is x_{j-1} + the pending residuals:
+    // its sampled rows are csp_in + rhat_prev rows (running fp32 sums, [n_rows][d])
+    // and its per-camera means cgm_in + rmean_prev ([V][d]); every chained
+    // gate writes its own sums to csp_out / cgm_out
+    int chain;
+    const uint8_t *prev_flag;
+    const void *rhat_prev;
+    const float *rmean_prev;
+    const float *csp_in, *cgm_in;
+    float *csp_out, *cgm_out;
+    float *cam_mean_out;     // camera_mean_launch: [V][d] per-camera means of x
 };
 // Grid and scratch layout of one gate launch (k_gate.cu).
 struct GateGeom {
-    int n_slices, R, rows_per, n_ctas;
-    size_t colsum_off, tickets_off, n_tickets, total;
+    int n_slices, cw, R, rows_per, n_ctas;
+    size_t tickets_off, n_tickets, total;
 };
 // One view group of V cameras, npc tokens and kfp sample rows each.
 inline void gate_single_group(GateArgs &g, int V, int npc, int kfp) {
@@ -59,13 +69,23 @@ inline void gate_single_group(GateArgs &g, int V, int npc, int kfp) {
     g.g_kfp[0] = kfp;
 }
 // Gate grid for V cameras of at most max_npc tokens, d columns, n_sm SMs; the
-// scratch holds partials, column sums and tickets (see GateGeom).
+// scratch holds the per-CTA partials and the ticket (see GateGeom).
 GateGeom gate_geometry(int V, int max_npc, int d, int n_sm);
 // Points the scratch fields (and grid fields) of g into `scratch`.
 void gate_bind_scratch(GateArgs &g, const GateGeom &gg, void *scratch);
 // Validates the gate knobs (NaN thresholds, ranges, counts); the reason goes to why.
 bool gate_ok(const xc_gate_params *p, int B, char *why, size_t n);
 template <typename T> cudaError_t gate_launch(const GateArgs &g, cudaStream_t st);
+// Per-camera column means of g.x into g.cam_mean_out (same grid as the gate;
+// exits at once when *g.flag is skip).
+template <typename T> cudaError_t camera_mean_launch(const GateArgs &g, cudaStream_t st);
+// Lazy chaining (reading c27): before block b (b = n_blocks: before the head)
+// computes, when the blocks before it back to j were skipped, writes
+// round(X[j & 1] + rhat[t][j] + ... + rhat[t][b - 1]) (fp32 sum in block
+// order) to X[b & 1].  Exits at once otherwise.
+template <typename T>
+cudaError_t chain_apply(T *x0, T *x1, const T *rhat_t, const uint8_t *flags, int b, int n_blocks, long ld,
+                        int n_sm, cudaStream_t st);
 bool make_tmap_bf16(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 int gemm_tc_bn(int M, int N);
 cudaError_t gemm_tc(int epi, int bn, const CUtensorMap &ta, const CUtensorMap &tb, const EpiParams &ep, int K,

@@ -60,6 +60,7 @@ class GateParams(ctypes.Structure):
                 ("warmup_chunks", ctypes.c_int), ("max_skips", ctypes.c_int),
                 ("protect_step0", ctypes.c_int), ("step0_strict_tau", ctypes.c_float),
                 ("fp_tokens", ctypes.c_int), ("fp_refresh", ctypes.c_int), ("fp_linear", ctypes.c_int),
+                ("chain", ctypes.c_int),
                 ("replay_skip", ctypes.POINTER(ctypes.c_uint8)),
                 ("replay_table", ctypes.c_void_p)]
 
@@ -79,7 +80,7 @@ class ProfileRec(ctypes.Structure):
 
 
 KERNEL_KINDS = ("cond", "embed", "gate", "ln", "qkv", "attn", "oproj", "ffn1", "ffn2", "reuse", "head",
-                "xattn")
+                "xattn", "chain")
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int

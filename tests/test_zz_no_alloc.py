@@ -103,11 +103,11 @@ def test_static_scratch_gate_rejects_geometry_beyond_its_maximum():
     buf = torch.zeros(1024, dtype=torch.uint8, device=DEV)
     p = buf.data_ptr()
     act = np.zeros(2, np.float32)
-    # 64 cameras x d 32768: 32768 (camera, 64-column slice) CTAs, each with 8
-    # partial metrics and 64 column sums in fp32 -- about 9 MiB of scratch
-    need = xb.op_gate_workspace_bytes("bf16", 64, 8, 32768)
-    assert need > 8 * (1 << 20)
-    st = xb.LIB.xc_op_gate_static(xb.XC_BF16, 64, 8, 32768, p, p, 1, p, p, p, act.ctypes.data, 2, 1, 1,
+    # 128 cameras x d 262144: 65536 (camera, column slice) CTAs, each with 8
+    # fp32 partial metrics (32 bytes) -- about 2 MiB of scratch, twice the maximum
+    need = xb.op_gate_workspace_bytes("bf16", 128, 8, 262144)
+    assert need > 2 * (1 << 20)
+    st = xb.LIB.xc_op_gate_static(xb.XC_BF16, 128, 8, 262144, p, p, 1, p, p, p, act.ctypes.data, 2, 1, 1,
                                   None, p, p, p, p, None)
     assert st == xb.XC_EINVAL
     assert "static maximum" in xb.last_error(None)
