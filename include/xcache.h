@@ -305,6 +305,15 @@ long long xc_launch_count(const xc_ctx *ctx);
  * hook off.  Process-wide; for tests of the error paths. */
 void xc_debug_fail_alloc(int n);
 
+/* Runs out one bounded device wait on purpose: a one-thread kernel waits on
+ * a barrier phase that nothing completes, gives up after the library's wait
+ * limit (2 s), records the expiry in the error word of ctx (NULL: the error
+ * word of the operator entry points) and returns -- the path every bounded
+ * wait of the library takes on expiry.  xc_sync(ctx) then reports
+ * XC_ETIMEOUT (xc_op_device_error() a non-zero word) and clears it; the
+ * context stays usable.  For tests of that path. */
+xc_status xc_debug_expire_wait(xc_ctx *ctx);
+
 #ifdef __cplusplus
 }
 #endif

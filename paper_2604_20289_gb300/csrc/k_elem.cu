@@ -2,8 +2,26 @@
 // adaLN-Zero LayerNorm modulation, the reuse path (Eq. 4), the conditioning
 // GEMVs, the output head, the Euler update and weight layout conversion.
 #include "xc_kernels.cuh"
+#include "xc_ptx.cuh"
 
 namespace xc {
+
+// ------------------------------------------------------- bounded-wait test
+// One thread waits on an mbarrier phase that nothing completes: the bounded
+// wait gives up after WAIT_NS, records `code` in *err and the kernel
+// returns (the error path of every wait in the library, made to run out on
+// purpose for its test).
+__global__ void expire_wait_kernel(int *err, int code) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    mbar_fence_init();
+    mbar_wait(&bar, 0, err, code);
+}
+cudaError_t expire_wait(int *err, int code, cudaStream_t st) {
+    expire_wait_kernel<<<1, 32, 0, st>>>(err, code);
+    return cudaGetLastError();
+}
 
 // ------------------------------------------------------------ patch embed
 // X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][16].

@@ -1194,6 +1194,22 @@ int xc_chunk_index(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->n; }
 
 void xc_debug_fail_alloc(int n) { g_fail_alloc.store(n > 0 ? n : 0); }
 
+static int *op_err_word();
+
+xc_status xc_debug_expire_wait(xc_ctx *ctx) {
+    int *err = ctx != nullptr ? ctx->d_err : op_err_word();
+    if (err == nullptr) {
+        set_err(nullptr, "xc_debug_expire_wait: no device error word");
+        return XC_ECUDA;
+    }
+    const cudaError_t e = expire_wait(err, ERR_WAIT_TMA, ctx != nullptr ? ctx->st : nullptr);
+    if (e != cudaSuccess) {
+        set_err(ctx, "xc_debug_expire_wait: %s", cudaGetErrorString(e));
+        return XC_ECUDA;
+    }
+    return XC_OK;
+}
+
 long long xc_launch_count(const xc_ctx *ctx) { return ctx == nullptr ? -1 : ctx->launches; }
 
 static void prof_free(xc_ctx *ctx) {

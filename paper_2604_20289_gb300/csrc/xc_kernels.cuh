@@ -125,6 +125,9 @@ cudaError_t head(const T *x, const float *hm, const float *w, const float *b, fl
                  cudaStream_t st);
 template <typename T> cudaError_t transpose_convert(const float *W, T *Wt, int K, int N, cudaStream_t st);
 cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out, int n, cudaStream_t st);
+// Test of the bounded waits: a one-thread kernel whose wait runs out (after
+// WAIT_NS) and records `code` in *err.
+cudaError_t expire_wait(int *err, int code, cudaStream_t st);
 // Records the message returned by xc_last_error(NULL).
 void set_global_error(const char *msg);
 }  // namespace xc

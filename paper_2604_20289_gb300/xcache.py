@@ -100,6 +100,7 @@ SIGNATURES = {
     "xc_sync": (_I, [_P]),
     "xc_chunk_index": (_I, [_P]),
     "xc_debug_fail_alloc": (None, [_I]),
+    "xc_debug_expire_wait": (_I, [_P]),
     "xc_launch_count": (ctypes.c_longlong, [_P]),
     "xc_profile_start": (_I, [_P, ctypes.c_uint, _I]),
     "xc_profile_stop": (_I, [_P, ctypes.POINTER(ProfileRec), _I, ctypes.POINTER(_I)]),

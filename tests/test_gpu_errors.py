@@ -46,3 +46,32 @@ def test_injected_allocation_failures_in_init():
     xc.sync()
     assert np.isfinite(v.cpu().numpy()).all() and st["chunk"] == 0
     xc.close()
+
+
+def test_expired_device_wait_is_reported_and_the_context_stays_usable():
+    """A bounded wait that runs out (nothing completes the barrier phase it
+    waits for) records its bit in the error word: xc_sync reports
+    XC_ETIMEOUT once, and the same context then runs a pass that gives the
+    same velocity as before."""
+    cfg = X.TINY_F32
+    w = X.make_weights(cfg)
+    traj = X.Trajectory(cfg, n_chunks=1)
+    xc = xb.XCache(cfg, w)
+    x = torch.tensor(traj.noise(0), device="cuda")
+    v0, v1 = torch.empty_like(x), torch.empty_like(x)
+    xc.chunk_step(x, traj.action(0), 1.0, 0, False, xb.gate_params(), v_out=v0)
+    xc.reset()
+    assert xb.LIB.xc_debug_expire_wait(xc.ctx) == xb.XC_OK
+    with pytest.raises(xb.XCacheError) as e:
+        xc.sync()
+    assert e.value.status == xb.XC_ETIMEOUT
+    xc.sync()                                   # reported once, then cleared
+    xc.chunk_step(x, traj.action(0), 1.0, 0, False, xb.gate_params(), v_out=v1)
+    xc.sync()
+    assert torch.equal(v0, v1)
+    xc.close()
+    # the operator entry points' error word
+    assert xb.op_device_error() == 0
+    assert xb.LIB.xc_debug_expire_wait(None) == xb.XC_OK
+    assert xb.op_device_error() != 0
+    assert xb.op_device_error() == 0
