@@ -22,8 +22,8 @@
 //   hd = 128: TMEM is full (S0 S1 O0 O1 = 512 columns); P_i overwrites S_i and
 //             S_{j+1} waits until P_j V has been issued; the two tiles
 //             ping-pong so the tensor core still has the other tile's work.
-// The two softmax warps of each SM sub-partition (one per tile) take turns
-// on the MUFU-bound exponential phase.
+// At head_dim 64 the two softmax warps of each SM sub-partition (one per
+// tile) take turns on the MUFU-bound exponential phase.
 // Online softmax in the exp2 domain with lazy rescaling: a row's O and sum
 // are rescaled only when its running max grows by more than 8 (2^8 headroom
 // in fp32 / bf16).  Score scaling and row sums use packed fp32 pairs
@@ -395,10 +395,15 @@ __global__ void __launch_bounds__(352, 1)
             // overlap the other's loads, max and MMA waits.  The hand-off is
             // per quadrant, so a slower sub-partition does not hold up the
             // others.
-            if (wg == 1 || g > 0) {
-                ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? g : g - 1) & 1, err, ERR_WAIT_SOFTMAX);
-                __syncwarp();
-                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+            // (hd 128: the turns cost more than they save -- the exponential
+            // phase is a smaller share of a key tile's work; 7.27 -> 7.16 ms
+            // at the 14B shape, 1.91 -> 1.85 ms at the 1.3B shape)
+            if constexpr (A::SEP_P) {
+                if (wg == 1 || g > 0) {
+                    ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? g : g - 1) & 1, err, ERR_WAIT_SOFTMAX);
+                    __syncwarp();
+                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                }
             }
             // probabilities p = 2^(s * sl2 - m), packed bf16 pairs + row sum,
             // stored to TMEM in four 32-key quarters
