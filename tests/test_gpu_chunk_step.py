@@ -1,6 +1,6 @@
 """Chunk-step parity: AR rollouts through xc_chunk_step against the CPU oracle.
 
-Tolerances (the benchmark spec): fp32 model max|err| <= 1e-4 x output RMS; bf16
+Tolerances: fp32 model max|err| <= 1e-4 x output RMS; bf16
 model per-block rel-L2 <= 1e-2 and final-latent rel-L2 <= 3e-2; gate
 decisions identical except where the oracle's metric lies within 1e-3
 relative of its threshold.  Numerics are compared in decision-replay mode

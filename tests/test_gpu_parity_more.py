@@ -228,3 +228,28 @@ def test_chained_small_model_matches_per_block_reuse_decisions():
         for sa, sb in zip(ca, cb):
             ok = ~np.isnan(sa["s_cos"])
             np.testing.assert_allclose(sb["s_cos"][ok], sa["s_cos"][ok], rtol=0, atol=5e-3)
+
+
+def test_all_method_options_together_bf16():
+    """View groups (front / side / rear cameras), cross-attention to a
+    varying number of condition tokens, a KV-update pass every second chunk
+    (force-compute chunks) and lazy chaining, on one bf16 model: decisions
+    and final latents against the oracle (decision replay) and free-running
+    decisions."""
+    cfg = X.GROUPS_BF16.replace(name="all_options_bf16_4blk", n_blocks=4, d_ctx=128, max_ctx=64, kv_period=2,
+                                n_chunks=5)
+    op, gp = params(tau_floor=0.9, tau_dev=3.0, back_anchors=1, chain=True)
+    w, xc = model(cfg)
+    traj = X.Trajectory(cfg, n_chunks=cfg.n_chunks)
+    ref = O.rollout(cfg, w, traj, op, cfg.n_chunks)
+    dec = decisions([ch[:cfg.n_steps] for ch in ref["stats"]])
+    assert (dec == O.Decision.SKIP).any()
+    rep = gpu_rollout(xc, traj, cfg.n_chunks, gp, replay=replay_of(ref["stats"]))
+    np.testing.assert_array_equal(decisions([ch[:cfg.n_steps] for ch in rep["stats"]]), dec)
+    for n in range(cfg.n_chunks):
+        assert rel_l2(rep["final"][n], ref["final"][n]) <= 3e-2, (n, rel_l2(rep["final"][n], ref["final"][n]))
+    xc.reset()
+    free = gpu_rollout(xc, traj, cfg.n_chunks, gp)
+    compare_decisions(ref["stats"], free["stats"], op)
+    xc.close()
+    _MODELS_drop(cfg)

@@ -319,7 +319,7 @@ def test_block_adaln_zero_identity():
     np.testing.assert_array_equal(got, x)
 
 
-# ------------------------------------------------ rollout invariants (the benchmark spec)
+# ------------------------------------------------ rollout invariants
 def _run(cfg, params, n_chunks, keep_trace=False, traj=None):
     w = X.make_weights(cfg)
     tr = traj or X.Trajectory(cfg, n_chunks=n_chunks)
