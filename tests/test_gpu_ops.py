@@ -287,3 +287,34 @@ def test_attention_split_all_rows(Lq, Lk, H, hd):
     assert per_row.max() <= 2e-2, per_row.max()
     assert rel_l2(host(o_whole)[rows], want) <= 5e-3
     assert xb.op_device_error() == 0
+
+
+def test_attention_wave_order_remainder_units():
+    """Wave work order: 40 heads x 32 query blocks = 1280 units over 152 SMs
+    (W = 8 whole waves) with K / V of 143 MB (above L2), so the launch runs
+    whole units in waves and splits the 64 remaining units (heads 38 and 39)
+    evenly over the SMs, merged from two or more partials.  Every row of the
+    remaining units is checked, plus sampled rows of the other heads; ragged
+    last query and key tiles."""
+    Lq, Lk, H, hd = 8000, 7000, 40, 128
+    d = H * hd
+    q = rt(f"Wq{Lq}{d}", (Lq, d))
+    k = rt(f"Wk{Lk}{d}", (Lk, d))
+    v = rt(f"Wv{Lk}{d}", (Lk, d))
+    o = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
+    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o, workspace="auto")
+    torch.cuda.synchronize()
+    got = host(o)
+    kk = k.reshape(Lk, H, hd).astype(np.float64)
+    vv = v.reshape(Lk, H, hd).astype(np.float64)
+    for h in (38, 39):
+        cols = slice(h * hd, (h + 1) * hd)
+        want = O.to_bf16(O.attention(q[:, cols].reshape(Lq, 1, hd).astype(np.float64), kk[:, h:h + 1],
+                                     vv[:, h:h + 1]).reshape(Lq, hd))
+        per_row = np.sqrt(((got[:, cols] - want) ** 2).sum(1) / (want ** 2).sum(1))
+        assert rel_l2(got[:, cols], want) <= 5e-3
+        assert per_row.max() <= 2e-2, (h, per_row.max())
+    rows = np.unique(np.r_[0, 255, 256, Lq - 1, np.random.default_rng(6).integers(0, Lq, 40)])
+    want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64), kk, vv).reshape(len(rows), d))
+    assert rel_l2(got[rows], want) <= 5e-3
+    assert xb.op_device_error() == 0
