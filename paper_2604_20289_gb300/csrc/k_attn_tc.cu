@@ -102,7 +102,7 @@ struct AttnSplit {
     __host__ __device__ long long begin2(int c) const { return T2 * c / G; }
 };
 struct TileCursor {
-    int g, seg, k;
+    int g, seg, k;        // contiguous order: seg holds the unit
 };
 // Waves: segments W and W + 1 of CTA c -- first key tile of segment W, end
 // key tiles of both (0: no such segment), and the unit of segment W.
@@ -165,12 +165,16 @@ __global__ void __launch_bounds__(352, 1)
         n_t = (int)(sp.begin(cta + 1) - it0);
     }
     const int u0 = (int)(it0 / nkt);
-    const TileCursor c0{0, 0, (int)(it0 % nkt)};
+    const TileCursor c0{0, WAVE ? 0 : u0, (int)(it0 % nkt)};
     auto seg_k0 = [&](int seg) { return seg < sp.W ? 0 : (seg == sp.W ? rem->k0 : 0); };
     auto seg_k1 = [&](int seg) { return seg < sp.W ? sp.n_kt : (seg == sp.W ? rem->k1a : rem->k1b); };
     auto seg_u = [&](int seg) {
         if constexpr (WAVE) return seg < sp.W ? cta + seg * sp.G : rem->u + (seg - sp.W);
-        else return u0 + seg;
+        else return seg;
+    };
+    auto piece_of = [&](const TileCursor &c) {    // index of the cursor's piece in this CTA
+        if constexpr (WAVE) return c.seg;
+        else return c.seg - u0;
     };
     auto first_of = [&](const TileCursor &c) {
         if constexpr (WAVE) return c.k == seg_k0(c.seg);
@@ -311,11 +315,11 @@ __global__ void __launch_bounds__(352, 1)
             // the producer may replace Q); P V of the first tile of a piece
             // overwrites O, so it waits until the softmax has read O out.
             auto s_ready = [&](const TileCursor &c) -> bool {
-                if (first_of(c) && !wait(q_full, c.seg)) return false;
+                if (first_of(c) && !wait(q_full, piece_of(c))) return false;
                 return wait(&k_full[c.g % A::STAGES], c.g / A::STAGES);
             };
             auto pv_ready = [&](int i, const TileCursor &c) -> bool {
-                if (first_of(c) && c.seg > 0 && !wait(&o_free[i], c.seg - 1)) return false;
+                if (first_of(c) && piece_of(c) > 0 && !wait(&o_free[i], piece_of(c) - 1)) return false;
                 return wait(&p_full[i], c.g) && wait(&v_full[c.g % A::STAGES], c.g / A::STAGES);
             };
             if constexpr (A::SEP_P) {
@@ -396,18 +400,12 @@ __global__ void __launch_bounds__(352, 1)
         const uint32_t tO = tl + A::O_COL(wg);
         const float sl2 = rsqrtf((float)HD) * 1.4426950408889634f;
         const int tail = n_keys - (nkt - 1) * A::BKV;      // valid keys in the last tile
-        bool ok = true;
-        TileCursor cur = c0;
-        while (ok && cur.g < n_t) {
-          // ---- one piece: key tiles [cur.k, ...] of the segment's unit
-          const bool cut_front = WAVE ? cur.k != 0 : (cur.g == 0 && cur.k != 0);   // began in another CTA
-          float m = -INFINITY, l = 0.0f;
-          bool fresh = true;
-          for (;;) {
-            const int g = cur.g;
-            ok = mbar_wait(&s_full[wg], g & 1, err, ERR_WAIT_SOFTMAX);
+        // One key tile g (key tile kt of its unit): S_i -> running max m,
+        // P_i = 2^(S_i sl2 - m) into TMEM, running sum l.  false: a wait ran out.
+        auto tile = [&](int g, int kt, bool fresh, float &m, float &l) -> bool {
+            bool ok = mbar_wait(&s_full[wg], g & 1, err, ERR_WAIT_SOFTMAX);
             __syncwarp();
-            if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+            if (!__all_sync(0xffffffffu, ok)) return false;
             tc_fence_after();
             float s[128];
             tmem_ld128_sync(tS, s);
@@ -415,7 +413,7 @@ __global__ void __launch_bounds__(352, 1)
                 tc_fence_before();
                 mbar_arrive(&s_cons[wg]);
             }
-            if (cur.k == nkt - 1 && tail < A::BKV) {
+            if (kt == nkt - 1 && tail < A::BKV) {
 #pragma unroll
                 for (int c = 0; c < 128; ++c)
                     if (c >= tail) s[c] = -INFINITY;
@@ -441,7 +439,7 @@ __global__ void __launch_bounds__(352, 1)
                 if (g >= 1) {
                     ok = mbar_wait(&pv_done[wg], (g - 1) & 1, err, ERR_WAIT_SOFTMAX);
                     __syncwarp();
-                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                    if (!__all_sync(0xffffffffu, ok)) return false;
                     tc_fence_after();
                 }
             }
@@ -470,7 +468,7 @@ __global__ void __launch_bounds__(352, 1)
                 if (wg == 1 || g > 0) {
                     ok = mbar_wait(&turn[4 * wg + q], (wg == 1 ? g : g - 1) & 1, err, ERR_WAIT_SOFTMAX);
                     __syncwarp();
-                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                    if (!__all_sync(0xffffffffu, ok)) return false;
                 }
             }
             // probabilities p = 2^(s * sl2 - m), packed bf16 pairs + row sum,
@@ -502,47 +500,81 @@ __global__ void __launch_bounds__(352, 1)
             mbar_arrive(&p_full[wg]);
             __syncwarp();
             if (lane == 0) mbar_arrive(&turn[4 * (wg ^ 1) + q]);
-            fresh = false;
-            if (last_of(cur)) break;
+            return true;
+        };
+        // End of a piece (its last tile g, unit u, piece p of this CTA): O_i
+        // complete -> output (whole unit) or partial.
+        auto end_piece = [&](int g, int u, int p, bool head_part, bool cut_front, float m, float l) -> bool {
+            const bool ok = mbar_wait(&pv_done[wg], (A::SEP_P ? g : p) & 1, err, ERR_WAIT_SOFTMAX);
+            __syncwarp();
+            if (!__all_sync(0xffffffffu, ok)) return false;
+            tc_fence_after();
+            const int h = u / sp.n_qblk;
+            const int row = (u % sp.n_qblk) * (A::QT * A::BQ) + r_tile;
+            if (!head_part && !cut_front) {
+                const float inv = 1.0f / l;
+#pragma unroll 1
+                for (int c = 0; c < HD / 16; ++c) {
+                    float t[16];
+                    tmem_ld16_sync(tO + 16 * c, t);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) t[i] *= inv;
+                    if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
+                }
+            } else {
+                const int slot = WAVE ? 2 * cta + (p - sp.W)                       // remainder segment 0 / 1
+                                      : (head_part ? 2 * (cta + 1) : 2 * cta + 1);   // boundary c + 1 head / c tail
+                float *wo = ws_o + ((size_t)slot * (A::QT * A::BQ) + r_tile) * HD;
+#pragma unroll 1
+                for (int c = 0; c < HD / 16; ++c) {
+                    float t[16];
+                    tmem_ld16_sync(tO + 16 * c, t);
+                    store16<float>(wo + 16 * c, t);
+                }
+                ws_ml[(size_t)slot * (A::QT * A::BQ) + r_tile] = make_float2(m, l);
+            }
+            tc_fence_before();
+            mbar_arrive(&o_free[wg]);
+            return true;
+        };
+        bool ok = true;
+        if constexpr (WAVE) {
+          // piece by piece -- key tiles [k0, k1) of the piece's unit, bounds
+          // read once per piece -- so that the tile loop carries only the
+          // tile counter g and the key tile kt
+          int g = 0;
+          for (int seg = 0; ok && g < n_t; ++seg) {
+            int k0 = 0, k1 = nkt;
+            if (seg >= sp.W) {
+                k0 = seg == sp.W ? rem_s.k0 : 0;
+                k1 = seg == sp.W ? rem_s.k1a : rem_s.k1b;
+            }
+            float m = -INFINITY, l = 0.0f;
+            for (int kt = k0;; ++kt, ++g) {
+                ok = tile(g, kt, kt == k0, m, l);
+                if (!ok || kt == k1 - 1) break;
+            }
+            if (!ok) break;
+            ok = end_piece(g, seg_u(seg), seg, k1 != nkt, k0 != 0, m, l);
+            ++g;
+          }
+        } else {
+          TileCursor cur = c0;
+          while (ok && cur.g < n_t) {
+            const bool cut_front = cur.g == 0 && cur.k != 0;      // the unit began in another CTA
+            float m = -INFINITY, l = 0.0f;
+            bool fresh = true;
+            for (;;) {
+                ok = tile(cur.g, cur.k, fresh, m, l);
+                if (!ok) break;
+                fresh = false;
+                if (last_of(cur)) break;
+                next(cur);
+            }
+            if (!ok) break;
+            ok = end_piece(cur.g, cur.seg, cur.seg - u0, cur.k != nkt - 1, cut_front, m, l);
             next(cur);
           }
-          if (!ok) break;
-          {
-                // end of a piece: O_i complete -> output (whole unit) or partial
-                const int g = cur.g, u = seg_u(cur.seg), p = cur.seg;
-                ok = mbar_wait(&pv_done[wg], (A::SEP_P ? g : p) & 1, err, ERR_WAIT_SOFTMAX);
-                __syncwarp();
-                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-                tc_fence_after();
-                const int h = u / sp.n_qblk;
-                const int row = (u % sp.n_qblk) * (A::QT * A::BQ) + r_tile;
-                const bool head_part = cur.k != nkt - 1;                       // unit continues in another CTA
-                if (!head_part && !cut_front) {
-                    const float inv = 1.0f / l;
-#pragma unroll 1
-                    for (int c = 0; c < HD / 16; ++c) {
-                        float t[16];
-                        tmem_ld16_sync(tO + 16 * c, t);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) t[i] *= inv;
-                        if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
-                    }
-                } else {
-                    const int slot = WAVE ? 2 * cta + (cur.seg - sp.W)                 // remainder segment 0 / 1
-                                          : (head_part ? 2 * (cta + 1) : 2 * cta + 1);   // boundary c + 1 head / c tail
-                    float *wo = ws_o + ((size_t)slot * (A::QT * A::BQ) + r_tile) * HD;
-#pragma unroll 1
-                    for (int c = 0; c < HD / 16; ++c) {
-                        float t[16];
-                        tmem_ld16_sync(tO + 16 * c, t);
-                        store16<float>(wo + 16 * c, t);
-                    }
-                    ws_ml[(size_t)slot * (A::QT * A::BQ) + r_tile] = make_float2(m, l);
-                }
-                tc_fence_before();
-                mbar_arrive(&o_free[wg]);
-          }
-          next(cur);
         }
     }
     tc_fence_before();
