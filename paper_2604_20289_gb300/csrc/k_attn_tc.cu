@@ -102,7 +102,8 @@ struct AttnSplit {
     __host__ __device__ long long begin2(int c) const { return T2 * c / G; }
 };
 struct TileCursor {
-    int g, seg, k;        // contiguous order: seg holds the unit
+    int g, u, k;          // tile counter, unit, key tile of the unit
+    int p, du;            // waves: piece index, unit step (G over the waves, 1 in the remainder)
 };
 // Waves: segments W and W + 1 of CTA c -- first key tile of segment W, end
 // key tiles of both (0: no such segment), and the unit of segment W.
@@ -154,8 +155,6 @@ __global__ void __launch_bounds__(352, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nkt = sp.n_kt;
     const int cta = blockIdx.x;
-    __shared__ RemSeg rem_s;                       // waves: the remainder piece (static shared)
-    volatile RemSeg *rem = &rem_s;
     long long it0 = 0;
     int n_t;                                       // key tiles of this CTA (>= 1)
     if constexpr (WAVE) {
@@ -165,48 +164,46 @@ __global__ void __launch_bounds__(352, 1)
         n_t = (int)(sp.begin(cta + 1) - it0);
     }
     const int u0 = (int)(it0 / nkt);
-    const TileCursor c0{0, WAVE ? 0 : u0, (int)(it0 % nkt)};
-    auto seg_k0 = [&](int seg) { return seg < sp.W ? 0 : (seg == sp.W ? rem->k0 : 0); };
-    auto seg_k1 = [&](int seg) { return seg < sp.W ? sp.n_kt : (seg == sp.W ? rem->k1a : rem->k1b); };
-    auto seg_u = [&](int seg) {
-        if constexpr (WAVE) return seg < sp.W ? cta + seg * sp.G : rem->u + (seg - sp.W);
-        else return seg;
-    };
+    // Waves: this CTA's remainder segments (registers of the cursor roles),
+    // and the tile at which its remainder begins.  The cursor steps like the
+    // contiguous one -- next unit after a unit's last key tile -- with a jump
+    // to the remainder at tile gw, so the per-tile tests stay the same.
+    RemSeg rem{0, 0, 0, 0};
+    if constexpr (WAVE) rem = rem_seg(sp, cta);
+    const int gw = WAVE ? sp.W * nkt : -1;
+    TileCursor c0{0, u0, (int)(it0 % nkt), 0, 1};
+    if constexpr (WAVE) c0 = sp.W > 0 ? TileCursor{0, cta, 0, 0, sp.G} : TileCursor{0, rem.u, rem.k0, 0, 1};
     auto piece_of = [&](const TileCursor &c) {    // index of the cursor's piece in this CTA
-        if constexpr (WAVE) return c.seg;
-        else return c.seg - u0;
+        if constexpr (WAVE) return c.p;
+        else return c.u - u0;
     };
     auto first_of = [&](const TileCursor &c) {
-        if constexpr (WAVE) return c.k == seg_k0(c.seg);
+        if constexpr (WAVE) return c.k == 0 || c.g == gw;
         else return c.g == 0 || c.k == 0;
     };
-    auto last_of = [&](const TileCursor &c) {
-        if constexpr (WAVE) return c.k == seg_k1(c.seg) - 1;
-        else return c.g == n_t - 1 || c.k == nkt - 1;
-    };
+    auto last_of = [&](const TileCursor &c) { return c.g == n_t - 1 || c.k == nkt - 1; };
     auto next = [&](TileCursor &c) {
         ++c.g;
-        if constexpr (WAVE) {
-            if (++c.k == seg_k1(c.seg)) {
-                ++c.seg;
-                c.k = seg_k0(c.seg);
+        if (++c.k == nkt) {
+            c.k = 0;
+            if constexpr (WAVE) {
+                c.u += c.du;
+                ++c.p;
+            } else {
+                ++c.u;
             }
-        } else {
-            if (++c.k == nkt) {
-                c.k = 0;
-                ++c.seg;
+        }
+        if constexpr (WAVE) {
+            if (c.g == gw) {
+                c.u = rem.u;
+                c.k = rem.k0;
+                c.du = 1;
+                c.p = sp.W;
             }
         }
     };
 
     if (threadIdx.x == 0) {
-        if constexpr (WAVE) {
-            const RemSeg r = rem_seg(sp, cta);
-            rem->k0 = r.k0;
-            rem->k1a = r.k1a;
-            rem->k1b = r.k1b;
-            rem->u = r.u;
-        }
         mbar_init(q_full, 1);
         mbar_init(q_empty, A::ISSUERS);
         for (int s = 0; s < A::STAGES; ++s) {
@@ -239,7 +236,7 @@ __global__ void __launch_bounds__(352, 1)
             for (TileCursor c = c0; c.g < n_t; next(c)) {
                 const int g = c.g;
                 if (first_of(c)) {
-                    const int u = seg_u(c.seg);
+                    const int u = c.u;
                     h = u / sp.n_qblk;
                     const int q0 = (u % sp.n_qblk) * (A::QT * A::BQ);
                     // the previous piece's Q stays until its last S MMA is done
@@ -538,30 +535,9 @@ __global__ void __launch_bounds__(352, 1)
             return true;
         };
         bool ok = true;
-        if constexpr (WAVE) {
-          // piece by piece -- key tiles [k0, k1) of the piece's unit, bounds
-          // read once per piece -- so that the tile loop carries only the
-          // tile counter g and the key tile kt
-          int g = 0;
-          for (int seg = 0; ok && g < n_t; ++seg) {
-            int k0 = 0, k1 = nkt;
-            if (seg >= sp.W) {
-                k0 = seg == sp.W ? rem_s.k0 : 0;
-                k1 = seg == sp.W ? rem_s.k1a : rem_s.k1b;
-            }
-            float m = -INFINITY, l = 0.0f;
-            for (int kt = k0;; ++kt, ++g) {
-                ok = tile(g, kt, kt == k0, m, l);
-                if (!ok || kt == k1 - 1) break;
-            }
-            if (!ok) break;
-            ok = end_piece(g, seg_u(seg), seg, k1 != nkt, k0 != 0, m, l);
-            ++g;
-          }
-        } else {
-          TileCursor cur = c0;
-          while (ok && cur.g < n_t) {
-            const bool cut_front = cur.g == 0 && cur.k != 0;      // the unit began in another CTA
+        TileCursor cur = c0;
+        while (ok && cur.g < n_t) {
+            const bool cut_front = cur.k != 0;     // the piece's unit began in another CTA
             float m = -INFINITY, l = 0.0f;
             bool fresh = true;
             for (;;) {
@@ -572,9 +548,8 @@ __global__ void __launch_bounds__(352, 1)
                 next(cur);
             }
             if (!ok) break;
-            ok = end_piece(cur.g, cur.seg, cur.seg - u0, cur.k != nkt - 1, cut_front, m, l);
+            ok = end_piece(cur.g, cur.u, piece_of(cur), cur.k != nkt - 1, cut_front, m, l);
             next(cur);
-          }
         }
     }
     tc_fence_before();
