@@ -562,11 +562,14 @@ __global__ void __launch_bounds__(352, 1)
 
 // Merges the partials of the units cut between CTAs (see AttnSplit): m =
 // max_p m_p, O = sum_p O_p 2^(m_p - m) / sum_p l_p 2^(m_p - m).  Contiguous
-// order: one CTA per CTA boundary, two partials (head and tail) of the unit
-// the boundary cuts.  Waves: one CTA per remaining unit, the partials of the
-// CTAs whose pieces touch it, in CTA order.  One thread per query row.
+// order: grid.x = CTA boundaries, two partials (head and tail) of the unit
+// the boundary cuts.  Waves: grid.x = remaining units, the partials of the
+// CTAs whose pieces touch it, in CTA order (up to G / R of them).  grid.y
+// picks 32 of the head's columns, grid.z 64 of the unit's 256 query rows;
+// one thread per row.
+constexpr int COMBINE_ROWS = 64, COMBINE_COLS = 32;
 template <int HD, bool WAVE>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(COMBINE_ROWS)
     attn_combine_kernel(bf16 *__restrict__ o, const int Lq, const int d, const AttnSplit sp,
                         const float *__restrict__ ws_o, const float2 *__restrict__ ws_ml,
                         const uint8_t *__restrict__ skip_flag) {
@@ -593,7 +596,8 @@ __global__ void __launch_bounds__(256)
         c_hi = b;
     }
     const int h = u / sp.n_qblk;
-    const int r = threadIdx.x;
+    const int r = blockIdx.z * COMBINE_ROWS + threadIdx.x;     // row of the unit
+    const int k0 = blockIdx.y * COMBINE_COLS;
     const int row = (u % sp.n_qblk) * 256 + r;
     if (row >= Lq) return;
     // slot of CTA c's partial of this unit
@@ -609,29 +613,32 @@ __global__ void __launch_bounds__(256)
     for (int c = c_lo; c <= c_hi; ++c)
         if (has(c)) mm = fmaxf(mm, ws_ml[(size_t)slot(c) * 256 + r].x);
     float den = 0.0f;
-    for (int c = c_lo; c <= c_hi; ++c)
-        if (has(c)) {
-            const float2 ml = ws_ml[(size_t)slot(c) * 256 + r];
-            den += ml.y * exp2f(ml.x - mm);
-        }
-    const float inv = 1.0f / den;
-#pragma unroll 1
-    for (int k = 0; k < HD; k += 16) {
-        float acc[16];
+    float acc[COMBINE_COLS];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) acc[i] = 0.0f;
-        for (int c = c_lo; c <= c_hi; ++c) {
-            if (!has(c)) continue;
-            const int sl = slot(c);
-            const float w = exp2f(ws_ml[(size_t)sl * 256 + r].x - mm);
+    for (int i = 0; i < COMBINE_COLS; ++i) acc[i] = 0.0f;
+#pragma unroll 2
+    for (int c = c_lo; c <= c_hi; ++c) {
+        if (!has(c)) continue;
+        const int sl = slot(c);
+        const float2 ml = ws_ml[(size_t)sl * 256 + r];
+        const float w = exp2f(ml.x - mm);
+        den += ml.y * w;
+        const float *src = ws_o + ((size_t)sl * 256 + r) * HD + k0;
+#pragma unroll
+        for (int j = 0; j < COMBINE_COLS; j += 16) {
             float x[16];
-            load16<float>(ws_o + ((size_t)sl * 256 + r) * HD + k, x);
+            load16<float>(src + j, x);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = fmaf(x[i], w, acc[i]);
+            for (int i = 0; i < 16; ++i) acc[j + i] = fmaf(x[i], w, acc[j + i]);
         }
+    }
+    const float inv = 1.0f / den;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) acc[i] *= inv;
-        store16<bf16>(o + (size_t)row * d + h * HD + k, acc);
+    for (int j = 0; j < COMBINE_COLS; j += 16) {
+        float y[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) y[i] = acc[j + i] * inv;
+        store16<bf16>(o + (size_t)row * d + h * HD + k0 + j, y);
     }
 }
 
@@ -672,7 +679,8 @@ static cudaError_t launch_attn_(const CUtensorMap &tq, const CUtensorMap &tk, co
     if (e != cudaSuccess) return e;
     if (n_launched) *n_launched = 1;
     if (split && n_combine > 0) {
-        e = launch_pdl(attn_combine_kernel<HD, WAVE>, dim3(n_combine), dim3(256), 0, st, o, Lq, d, sp,
+        e = launch_pdl(attn_combine_kernel<HD, WAVE>, dim3(n_combine, HD / COMBINE_COLS, 256 / COMBINE_ROWS),
+                       dim3(COMBINE_ROWS), 0, st, o, Lq, d, sp,
                        static_cast<const float *>(ws_o), static_cast<const float2 *>(ws_ml), skip);
         if (n_launched) *n_launched = 2;
     }
