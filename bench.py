@@ -408,6 +408,14 @@ def kernel_work(cfg, kind: str, n_keys: int) -> tuple[str, float]:
         return "hbm", float(3 * L * d * es)             # x, r_hat in; x + r_hat out
     if kind == "ln":
         return "hbm", float(2 * L * d * es)
+    C = cfg.c_latent
+    if kind == "embed":                                 # latent + pe_w in, X0 out
+        return "hbm", float(L * C * 4 + C * d * 4 + L * d * es)
+    if kind == "head":                                  # block output + W_out in, velocity out
+        return "hbm", float(L * d * es + d * C * 4 + L * C * 4)
+    if kind == "cond":                                  # the conditioning MLP weights (fp32) + per-block tables
+        B, tf, A = cfg.n_blocks, cfg.t_freq, cfg.action_dim
+        return "hbm", float(4 * (tf * d + A * d + 2 * d * d + 6 * d * d + 2 * d * d) + 2 * 4 * B * 6 * d)
     return "", 0.0
 
 

@@ -23,41 +23,107 @@ cudaError_t expire_wait(int *err, int code, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+static int n_sm_elem() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    }
+    return n;
+}
+
 // ------------------------------------------------------------ patch embed
 // X0[r][c] = round(sum_k z[r][k] * pe_w[k][c] + pe_b[c]), z float32 [L][16].
-// Warp = one 16-column run of 32 consecutive rows (lane = row): every lane
-// needs the same 16 x 16 block of pe_w, so its loads are warp-wide
-// broadcasts, and each lane reads its own 64-byte latent row.
+// Each lane owns 4 columns for the whole kernel and keeps their 16 x 4 block
+// of pe_w and 4 biases in registers; a warp covers 128 consecutive columns
+// and writes 128 columns of a row per store instruction.  CTA = 8 warps over
+// one column block and a range of rows, walked in chunks of 64 latent rows
+// (4 KB) staged in shared memory: the next chunk is loaded into registers
+// (one float4 per thread) while the current one is computed, so the global
+// load latency overlaps the arithmetic.
+constexpr int PE_COLS = 128, PE_WARPS = 8, PE_CHUNK = 64;
 template <typename T>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(PE_WARPS * 32)
     patch_embed_kernel(const float *__restrict__ z, const float *__restrict__ w, const float *__restrict__ b,
-                       T *__restrict__ out, int L, int d) {
+                       T *__restrict__ out, int L, int d, int rows_per_cta) {
     pdl_wait();
     pdl_release();
+    __shared__ __align__(16) float zs[2][PE_CHUNK * 16];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int run = blockIdx.y * 8 + warp;
-    const int row = blockIdx.x * 32 + lane;
-    if (run * 16 >= d || row >= L) return;
-    const int col = run * 16;
-    float zr[16];
-    load16<float>(z + (size_t)row * 16, zr);
-    float acc[16];
-    load16<float>(b + col, acc);
+    const int col = blockIdx.x * PE_COLS + 4 * lane;
+    const bool active = col < d;
+    float wr[16][4], bias[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-        float wr[16];
-        load16<float>(w + (size_t)k * d + col, wr);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) acc[j] = fmaf(zr[k], wr[j], acc[j]);
+        float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (active) t = *reinterpret_cast<const float4 *>(w + (size_t)k * d + col);
+        wr[k][0] = t.x;
+        wr[k][1] = t.y;
+        wr[k][2] = t.z;
+        wr[k][3] = t.w;
     }
-    store16<T>(out + (size_t)row * d + col, acc);
+    if (active) {
+        const float4 t = *reinterpret_cast<const float4 *>(b + col);
+        bias[0] = t.x;
+        bias[1] = t.y;
+        bias[2] = t.z;
+        bias[3] = t.w;
+    }
+    const int r0 = blockIdx.y * rows_per_cta;
+    const int r1 = min(L, r0 + rows_per_cta);
+    // thread t stages float4 t of a chunk: row t / 4, quarter t % 4
+    auto fetch = [&](int c0) {
+        const int row = c0 + (threadIdx.x >> 2);
+        return row < r1 ? __ldg(reinterpret_cast<const float4 *>(z + (size_t)row * 16) + (threadIdx.x & 3))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    float4 nxt = fetch(r0);
+    int buf = 0;
+    for (int c0 = r0; c0 < r1; c0 += PE_CHUNK, buf ^= 1) {
+        reinterpret_cast<float4 *>(zs[buf])[threadIdx.x] = nxt;
+        __syncthreads();
+        if (c0 + PE_CHUNK < r1) nxt = fetch(c0 + PE_CHUNK);
+        const int n = min(PE_CHUNK, r1 - c0);
+        if (active) {
+            for (int rr = warp; rr < n; rr += PE_WARPS) {
+                const float4 *zr = reinterpret_cast<const float4 *>(zs[buf] + rr * 16);
+                float acc[4] = {bias[0], bias[1], bias[2], bias[3]};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 zq = zr[q];
+                    const float zv[4] = {zq.x, zq.y, zq.z, zq.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) acc[j] = fmaf(zv[i], wr[4 * q + i][j], acc[j]);
+                }
+                T *dst = out + (size_t)(c0 + rr) * d + col;
+                if constexpr (sizeof(T) == 2) {
+                    __nv_bfloat162 lo = __floats2bfloat162_rn(acc[0], acc[1]);
+                    __nv_bfloat162 hi = __floats2bfloat162_rn(acc[2], acc[3]);
+                    uint2 pk;
+                    pk.x = *reinterpret_cast<uint32_t *>(&lo);
+                    pk.y = *reinterpret_cast<uint32_t *>(&hi);
+                    *reinterpret_cast<uint2 *>(dst) = pk;
+                } else {
+                    *reinterpret_cast<float4 *>(dst) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+                }
+            }
+        }
+    }
 }
 
 template <typename T>
 cudaError_t patch_embed(const float *z, const float *w, const float *b, T *out, int L, int C, int d, cudaStream_t st) {
     if (C != 16 || d % 16 != 0) return cudaErrorInvalidValue;
-    const dim3 grid((L + 31) / 32, (d / 16 + 7) / 8);
-    return launch_pdl(patch_embed_kernel<T>, grid, dim3(256), 0, st, z, w, b, out, L, d);
+    const int n_sm = n_sm_elem();
+    const int n_cb = (d + PE_COLS - 1) / PE_COLS;
+    int n_rb = (16 * n_sm + n_cb - 1) / n_cb;          // many short CTAs: no tail wave to speak of
+    const int rows = ((L + n_rb - 1) / n_rb + PE_CHUNK - 1) / PE_CHUNK * PE_CHUNK;
+    n_rb = (L + rows - 1) / rows;
+    return launch_pdl(patch_embed_kernel<T>, dim3(n_cb, n_rb < 1 ? 1 : n_rb), dim3(PE_WARPS * 32), 0, st, z, w, b,
+                      out, L, d, rows);
 }
 template cudaError_t patch_embed<float>(const float *, const float *, const float *, float *, int, int, int, cudaStream_t);
 template cudaError_t patch_embed<bf16>(const float *, const float *, const float *, bf16 *, int, int, int, cudaStream_t);
@@ -328,16 +394,6 @@ static cudaError_t ln_mod_cta(const T *x, const float *shift, const float *scale
                               const uint8_t *skip, cudaStream_t st) {
     return launch_pdl(ln_mod_cta_kernel<T, KMAX>, dim3(M), dim3(LN_CTA), 0, st, x, shift, scale, out, M, d, eps,
                       skip);
-}
-
-static int n_sm_elem() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
-    }
-    return n;
 }
 
 template <typename T, int NCH>
@@ -618,39 +674,61 @@ cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out,
 // ------------------------------------------------------------------- head
 // Output head (a10): v = round(LN(x) * (1 + scale) + shift) W_out + b,
 // W_out [d][16].  CTA = 32 rows, 256 threads.  Pass 1: warp w reduces the
-// moments of rows 4w..4w+3.  Pass 2 walks the columns in chunks of 256: the
-// CTA writes the modulated chunk h[32][256] (rounded to the storage type) to
-// shared memory, then warp w multiplies its 32-column slice: lane (r4, c4)
-// accumulates rows 4 r4..4 r4+3 x outputs 4 c4..4 c4+3, reading W_out rows
-// as float4 (shared by the 8 lanes with the same c4) and h as broadcasts
-// (row stride 257 words: the 8 row groups fall in distinct banks).  The 8
-// warps' partial sums are then added in shared memory.
-constexpr int HEAD_ROWS = 32, HEAD_CH = 256;
+// moments of rows 4w..4w+3 (two loads in flight per lane).  Pass 2 walks the
+// columns in chunks of 128 (the next chunk's loads in flight meanwhile): the
+// CTA writes the modulated chunk h (rounded to the storage type) to shared
+// memory transposed, hT[k][row] (lane = row when staging, so the stores are
+// conflict-free), and the chunk's 128 x 16 block of W_out beside it; warp w
+// then takes keys 16w..16w+15 of the chunk, lane (r4, c4) accumulating rows
+// 4 r4..4 r4+3 x outputs 4 c4..4 c4+3 from one float4 of hT and one of W_out
+// per key (16 FMA per two shared loads).  The 8 warps' partial sums are
+// added in shared memory at the end, in warp order.
+__device__ __forceinline__ void fma4(float (&a)[4], float h, const float4 &w) {
+    a[0] = fmaf(h, w.x, a[0]);
+    a[1] = fmaf(h, w.y, a[1]);
+    a[2] = fmaf(h, w.z, a[2]);
+    a[3] = fmaf(h, w.w, a[3]);
+}
+constexpr int HEAD_ROWS = 32, HEAD_CH = 128, HEAD_LD = HEAD_ROWS + 4;
 template <typename T>
 __global__ void __launch_bounds__(256)
     head_kernel(const T *__restrict__ x, const float *__restrict__ hm, const float *__restrict__ w,
                 const float *__restrict__ b, float *__restrict__ v, int L, int d, float eps) {
     pdl_wait();
     pdl_release();
-    __shared__ float hs[HEAD_ROWS * (HEAD_CH + 1)];
+    __shared__ __align__(16) float hT[HEAD_CH * HEAD_LD];
+    __shared__ __align__(16) float ws[HEAD_CH * 16];
     __shared__ float2 stats[HEAD_ROWS];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int row0 = blockIdx.x * HEAD_ROWS;
     const int runs = d / 16;
+    // moments of one 16-element run, merged into mo
+    auto add_run = [](Moments &mo, const float (&t)[16]) {
+        float sum = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sum += t[i];
+        Moments m1{16.0f, sum * (1.0f / 16.0f), 0.0f};
+#pragma unroll
+        for (int i = 0; i < 16; ++i) m1.m2 += (t[i] - m1.mean) * (t[i] - m1.mean);
+        mo = merge(mo, m1);
+    };
     for (int rr = 0; rr < 4; ++rr) {
         const int r = warp * 4 + rr, row = row0 + r;
         Moments mo{0.0f, 0.0f, 0.0f};
         if (row < L) {
-            for (int run = lane; run < runs; run += 32) {
-                float t[16];
-                load16<T>(x + (size_t)row * d + 16 * run, t);
-                float sum = 0.0f;
-#pragma unroll
-                for (int i = 0; i < 16; ++i) sum += t[i];
-                Moments m1{16.0f, sum * (1.0f / 16.0f), 0.0f};
-#pragma unroll
-                for (int i = 0; i < 16; ++i) m1.m2 += (t[i] - m1.mean) * (t[i] - m1.mean);
-                mo = merge(mo, m1);
+            const T *xr = x + (size_t)row * d;
+            int run = lane;
+            for (; run + 32 < runs; run += 64) {         // two runs in flight
+                float t0[16], t1[16];
+                load16<T>(xr + 16 * run, t0);
+                load16<T>(xr + 16 * (run + 32), t1);
+                add_run(mo, t0);
+                add_run(mo, t1);
+            }
+            if (run < runs) {
+                float t0[16];
+                load16<T>(xr + 16 * run, t0);
+                add_run(mo, t0);
             }
         }
         mo = warp_moments(mo);
@@ -664,44 +742,57 @@ __global__ void __launch_bounds__(256)
     for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+    const int my_row = row0 + lane;
+    const float2 my_st = stats[lane];
+    // warp w stages keys [16 w, 16 w + 16) of each chunk for its lane's row;
+    // the next chunk's values are loaded while the current one is computed
+    float xn[16];
+    auto fetch = [&](int c0) {
+        if (my_row < L && c0 + warp * 16 < d) {
+            load16<T>(x + (size_t)my_row * d + c0 + warp * 16, xn);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) xn[i] = 0.0f;
+        }
+    };
+    fetch(0);
     for (int c0 = 0; c0 < d; c0 += HEAD_CH) {
         const int n = d - c0 < HEAD_CH ? d - c0 : HEAD_CH;      // multiple of 16
-        const int nr = n / 16;
-        for (int idx = threadIdx.x; idx < HEAD_ROWS * nr; idx += blockDim.x) {
-            const int r = idx / nr, cr = (idx - r * nr) * 16, row = row0 + r;
+        const int k16 = warp * 16;
+        if (k16 < n) {
             float t[16];
-            if (row < L) {
+            if (my_row < L) {
                 float sc[16], sh[16];
-                load16<T>(x + (size_t)row * d + c0 + cr, t);
-                load16<float>(scale + c0 + cr, sc);
-                load16<float>(shift + c0 + cr, sh);
-                const float2 st = stats[r];
+                load16<float>(scale + c0 + k16, sc);
+                load16<float>(shift + c0 + k16, sh);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) t[i] = round_to<T>((t[i] - st.x) * st.y * (1.0f + sc[i]) + sh[i]);
+                for (int i = 0; i < 16; ++i)
+                    t[i] = round_to<T>((xn[i] - my_st.x) * my_st.y * (1.0f + sc[i]) + sh[i]);
             } else {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) t[i] = 0.0f;
             }
 #pragma unroll
-            for (int i = 0; i < 16; ++i) hs[r * (HEAD_CH + 1) + cr + i] = t[i];
+            for (int i = 0; i < 16; ++i) hT[(k16 + i) * HEAD_LD + lane] = t[i];
         }
+        for (int i = threadIdx.x; i < n * 4; i += blockDim.x)
+            reinterpret_cast<float4 *>(ws)[i] = reinterpret_cast<const float4 *>(w + (size_t)c0 * 16)[i];
         __syncthreads();
-        const int k_end = 32 * warp + 32 < n ? 32 * warp + 32 : n;
-        for (int k = 32 * warp; k < k_end; ++k) {
-            const float4 wv = *reinterpret_cast<const float4 *>(w + (size_t)(c0 + k) * 16 + 4 * c4);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float hv = hs[(4 * r4 + i) * (HEAD_CH + 1) + k];
-                acc[i][0] = fmaf(hv, wv.x, acc[i][0]);
-                acc[i][1] = fmaf(hv, wv.y, acc[i][1]);
-                acc[i][2] = fmaf(hv, wv.z, acc[i][2]);
-                acc[i][3] = fmaf(hv, wv.w, acc[i][3]);
-            }
+        if (c0 + HEAD_CH < d) fetch(c0 + HEAD_CH);
+        const int k_end = 16 * warp + 16 < n ? 16 * warp + 16 : n;
+#pragma unroll 4
+        for (int k = 16 * warp; k < k_end; ++k) {
+            const float4 hv = *reinterpret_cast<const float4 *>(hT + k * HEAD_LD + 4 * r4);
+            const float4 wv = *reinterpret_cast<const float4 *>(ws + k * 16 + 4 * c4);
+            fma4(acc[0], hv.x, wv);
+            fma4(acc[1], hv.y, wv);
+            fma4(acc[2], hv.z, wv);
+            fma4(acc[3], hv.w, wv);
         }
         __syncthreads();
     }
-    // partial sums of the 8 warps -> shared memory (reuses hs), then add
-    float *red = hs;                                          // [8][32][16] = 4096 floats
+    // partial sums of the 8 warps -> shared memory (reuses hT), then add
+    float *red = hT;                                          // [8][32][16] = 4096 floats
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
