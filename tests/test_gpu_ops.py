@@ -318,3 +318,33 @@ def test_attention_wave_order_remainder_units():
     want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64), kk, vv).reshape(len(rows), d))
     assert rel_l2(got[rows], want) <= 5e-3
     assert xb.op_device_error() == 0
+
+
+def test_attention_wave_order_head_dim_64():
+    """Wave work order at head_dim 64: 64 heads x 32 query blocks = 2048
+    units (W = 13 waves on 152 SMs) over 9000 keys (K / V 147 MB, above L2),
+    ragged last query and key tiles; every row of heads 61-63 (the 72
+    remaining units start at head 61, query block 24) and sampled rows of all
+    heads."""
+    Lq, Lk, H, hd = 8000, 9000, 64, 64
+    d = H * hd
+    q = rt(f"Wq{Lq}{d}", (Lq, d))
+    k = rt(f"Wk{Lk}{d}", (Lk, d))
+    v = rt(f"Wv{Lk}{d}", (Lk, d))
+    o = torch.empty(Lq, d, device=DEV, dtype=torch.bfloat16)
+    xb.op_attention("bf16", H, hd, dev(q, "bf16"), dev(k, "bf16"), dev(v, "bf16"), o, workspace="auto")
+    torch.cuda.synchronize()
+    got = host(o)
+    kk = k.reshape(Lk, H, hd).astype(np.float64)
+    vv = v.reshape(Lk, H, hd).astype(np.float64)
+    for h in (61, 62, 63):
+        cols = slice(h * hd, (h + 1) * hd)
+        want = O.to_bf16(O.attention(q[:, cols].reshape(Lq, 1, hd).astype(np.float64), kk[:, h:h + 1],
+                                     vv[:, h:h + 1]).reshape(Lq, hd))
+        per_row = np.sqrt(((got[:, cols] - want) ** 2).sum(1) / (want ** 2).sum(1))
+        assert rel_l2(got[:, cols], want) <= 5e-3
+        assert per_row.max() <= 2e-2, (h, per_row.max())
+    rows = np.unique(np.r_[0, 255, 256, Lq - 1, np.random.default_rng(7).integers(0, Lq, 24)])
+    want = O.to_bf16(O.attention(q[rows].reshape(-1, H, hd).astype(np.float64), kk, vv).reshape(len(rows), d))
+    assert rel_l2(got[rows], want) <= 5e-3
+    assert xb.op_device_error() == 0
