@@ -53,22 +53,18 @@ __global__ void __launch_bounds__(PE_WARPS * 32)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int col = blockIdx.x * PE_COLS + 4 * lane;
     const bool active = col < d;
-    float wr[16][4], bias[4] = {0.f, 0.f, 0.f, 0.f};
+    float2 wr[16][2], bias[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
         float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
         if (active) t = *reinterpret_cast<const float4 *>(w + (size_t)k * d + col);
-        wr[k][0] = t.x;
-        wr[k][1] = t.y;
-        wr[k][2] = t.z;
-        wr[k][3] = t.w;
+        wr[k][0] = make_float2(t.x, t.y);
+        wr[k][1] = make_float2(t.z, t.w);
     }
     if (active) {
         const float4 t = *reinterpret_cast<const float4 *>(b + col);
-        bias[0] = t.x;
-        bias[1] = t.y;
-        bias[2] = t.z;
-        bias[3] = t.w;
+        bias[0] = make_float2(t.x, t.y);
+        bias[1] = make_float2(t.z, t.w);
     }
     const int r0 = blockIdx.y * rows_per_cta;
     const int r1 = min(L, r0 + rows_per_cta);
@@ -88,16 +84,19 @@ __global__ void __launch_bounds__(PE_WARPS * 32)
         if (active) {
             for (int rr = warp; rr < n; rr += PE_WARPS) {
                 const float4 *zr = reinterpret_cast<const float4 *>(zs[buf] + rr * 16);
-                float acc[4] = {bias[0], bias[1], bias[2], bias[3]};
+                float2 a01 = bias[0], a23 = bias[1];           // packed fp32 pairs: two FMAs per instruction
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     const float4 zq = zr[q];
                     const float zv[4] = {zq.x, zq.y, zq.z, zq.w};
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) acc[j] = fmaf(zv[i], wr[4 * q + i][j], acc[j]);
+                    for (int i = 0; i < 4; ++i) {
+                        const float2 zz = make_float2(zv[i], zv[i]);
+                        a01 = __ffma2_rn(zz, wr[4 * q + i][0], a01);
+                        a23 = __ffma2_rn(zz, wr[4 * q + i][1], a23);
+                    }
                 }
+                const float acc[4] = {a01.x, a01.y, a23.x, a23.y};
                 T *dst = out + (size_t)(c0 + rr) * d + col;
                 if constexpr (sizeof(T) == 2) {
                     __nv_bfloat162 lo = __floats2bfloat162_rn(acc[0], acc[1]);
@@ -681,13 +680,12 @@ cudaError_t rope_table(int hd, double theta, int frame0, int4 npos, float2 *out,
 // conflict-free), and the chunk's 128 x 16 block of W_out beside it; warp w
 // then takes keys 16w..16w+15 of the chunk, lane (r4, c4) accumulating rows
 // 4 r4..4 r4+3 x outputs 4 c4..4 c4+3 from one float4 of hT and one of W_out
-// per key (16 FMA per two shared loads).  The 8 warps' partial sums are
+// per key (16 FMA, as 8 packed fp32-pair FMAs, per two shared loads).  The 8 warps' partial sums are
 // added in shared memory at the end, in warp order.
-__device__ __forceinline__ void fma4(float (&a)[4], float h, const float4 &w) {
-    a[0] = fmaf(h, w.x, a[0]);
-    a[1] = fmaf(h, w.y, a[1]);
-    a[2] = fmaf(h, w.z, a[2]);
-    a[3] = fmaf(h, w.w, a[3]);
+__device__ __forceinline__ void fma4(float2 (&a)[2], float h, const float4 &w) {
+    const float2 hh = make_float2(h, h);
+    a[0] = __ffma2_rn(hh, make_float2(w.x, w.y), a[0]);
+    a[1] = __ffma2_rn(hh, make_float2(w.z, w.w), a[1]);
 }
 constexpr int HEAD_ROWS = 32, HEAD_CH = 128, HEAD_LD = HEAD_ROWS + 4;
 template <typename T>
@@ -737,11 +735,9 @@ __global__ void __launch_bounds__(256)
     __syncthreads();
     const float *shift = hm, *scale = hm + d;
     const int r4 = lane >> 2, c4 = lane & 3;
-    float acc[4][4];
+    float2 acc[4][2];                                     // [row][column pair]
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+    for (int i = 0; i < 4; ++i) acc[i][0] = acc[i][1] = make_float2(0.f, 0.f);
     const int my_row = row0 + lane;
     const float2 my_st = stats[lane];
     // warp w stages keys [16 w, 16 w + 16) of each chunk for its lane's row;
@@ -794,9 +790,13 @@ __global__ void __launch_bounds__(256)
     // partial sums of the 8 warps -> shared memory (reuses hT), then add
     float *red = hT;                                          // [8][32][16] = 4096 floats
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) red[(warp * HEAD_ROWS + 4 * r4 + i) * 16 + 4 * c4 + j] = acc[i][j];
+    for (int i = 0; i < 4; ++i) {
+        float *dst = red + (warp * HEAD_ROWS + 4 * r4 + i) * 16 + 4 * c4;
+        dst[0] = acc[i][0].x;
+        dst[1] = acc[i][0].y;
+        dst[2] = acc[i][1].x;
+        dst[3] = acc[i][1].y;
+    }
     __syncthreads();
     for (int o = threadIdx.x; o < HEAD_ROWS * 16; o += blockDim.x) {
         const int r = o >> 4, c = o & 15;
