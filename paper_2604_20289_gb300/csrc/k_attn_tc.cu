@@ -90,10 +90,11 @@ __device__ __forceinline__ float ex2_approx(float x) {
 //    each K / V tile comes from DRAM once per wave -- then the R = n_units -
 //    W G remaining units, T2 = R n_kt key tiles, are split evenly: CTA c
 //    takes [c T2 / G, (c + 1) T2 / G), less than one unit, touching at most
-//    two units (its segments W and W + 1, partial slots 2 c and 2 c + 1),
+//    two units (its pieces W and W + 1, partial slots 2 c and 2 c + 1),
 //    merged per remaining unit by attn_combine_kernel.
-// Each role walks the CTA's key tiles with a cursor: tile counter g, segment
-// (piece) index seg, key tile k.
+// Each role walks the CTA's key tiles with a cursor (TileCursor): tile
+// counter g, unit u and its key tile k; in the wave order also the piece
+// index p and the unit step du.
 struct AttnSplit {
     long long T;          // contiguous: total iterations
     long long T2;         // waves: key tiles of the remaining units
@@ -105,8 +106,9 @@ struct TileCursor {
     int g, u, k;          // tile counter, unit, key tile of the unit
     int p, du;            // waves: piece index, unit step (G over the waves, 1 in the remainder)
 };
-// Waves: segments W and W + 1 of CTA c -- first key tile of segment W, end
-// key tiles of both (0: no such segment), and the unit of segment W.
+// Waves: pieces W and W + 1 of CTA c (its share of the remaining units) --
+// first key tile of piece W, end key tiles of both (0: no such piece), and
+// the unit of piece W.
 struct RemSeg {
     int k0, k1a, k1b, u;
 };
@@ -164,7 +166,7 @@ __global__ void __launch_bounds__(352, 1)
         n_t = (int)(sp.begin(cta + 1) - it0);
     }
     const int u0 = (int)(it0 / nkt);
-    // Waves: this CTA's remainder segments (registers of the cursor roles),
+    // Waves: this CTA's remainder pieces (registers of the cursor roles),
     // and the tile at which its remainder begins.  The cursor steps like the
     // contiguous one -- next unit after a unit's last key tile -- with a jump
     // to the remainder at tile gw, so the per-tile tests stay the same.
@@ -519,7 +521,7 @@ __global__ void __launch_bounds__(352, 1)
                     if (row < Lq) store16<bf16>(o + (size_t)row * d + h * HD + 16 * c, t);
                 }
             } else {
-                const int slot = WAVE ? 2 * cta + (p - sp.W)                       // remainder segment 0 / 1
+                const int slot = WAVE ? 2 * cta + (p - sp.W)                       // remainder piece 0 / 1
                                       : (head_part ? 2 * (cta + 1) : 2 * cta + 1);   // boundary c + 1 head / c tail
                 float *wo = ws_o + ((size_t)slot * (A::QT * A::BQ) + r_tile) * HD;
 #pragma unroll 1
