@@ -417,15 +417,18 @@ __global__ void __launch_bounds__(352, 1)
                 for (int c = 0; c < 128; ++c)
                     if (c >= tail) s[c] = -INFINITY;
             }
-            // row max: 16 independent chains of three-input max, then a tree
+            // row max: 16 independent chains of three-input max over columns
+            // 0..111, the last 16 columns, then a tree
             float mx[16];
 #pragma unroll
             for (int k = 0; k < 16; ++k) mx[k] = s[k];
 #pragma unroll
-            for (int c = 16; c < 128; c += 32) {
+            for (int c = 16; c < 112; c += 32) {
 #pragma unroll
                 for (int k = 0; k < 16; ++k) mx[k] = fmax3(mx[k], s[c + k], s[c + 16 + k]);
             }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) mx[k] = fmaxf(mx[k], s[112 + k]);
 #pragma unroll
             for (int k = 0; k < 5; ++k) mx[k] = fmax3(mx[k], mx[k + 5], mx[k + 10]);
             const float m_new = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[15]), mx[0]) * sl2;
