@@ -53,11 +53,14 @@ xc_status xc_op_qkv_rope(int dtype, int n_cams, int frames, int gh, int gw, int 
  * keys).  q, o [Lq][H*hd]; k, v [n_keys][H*hd] (bf16: 16-byte aligned rows).
  *   workspace  device, optional.  With at least
  *              xc_op_attention_workspace_bytes() bytes and more (head,
- *              256-query) units than SMs, the key range is split evenly over
- *              the SMs and units cut between two SMs are merged by a second
- *              kernel; with NULL (or too small) every unit runs whole on one
- *              SM.  Contents on entry are ignored; it must not be shared by
- *              calls that overlap in time.
+ *              256-query) units than SMs, the work is spread evenly over the
+ *              SMs: either the (unit, key tile) space is cut into equal
+ *              shares, or -- with 8 or more waves of units and the K / V of
+ *              all heads larger than L2 -- whole units run in waves and only
+ *              the remaining units are cut; a second kernel merges the
+ *              partials of the cut units.  With NULL (or too small) every
+ *              unit runs whole on one SM.  Contents on entry are ignored; it
+ *              must not be shared by calls that overlap in time.
  * bf16 needs head_dim 64 or 128; fp32 head_dim 16, 32 or 64. */
 size_t xc_op_attention_workspace_bytes(int dtype, int head_dim);
 xc_status xc_op_attention(int dtype, int Lq, int n_keys, int n_heads, int head_dim,
